@@ -1,0 +1,115 @@
+"""Attention, total variation, the Tier-A bound, the e-form meter and the gate.
+
+Test infrastructure only (see ``oracle/__init__.py``).  All arithmetic is
+float64 and follows the definitions in the order the paper states them.
+
+§3 setup: p and p~ are the softmax distributions over the cached tokens
+computed from exact and compressed keys; eps_t is token t's logit error;
+c_t >= |eps_t| is any per-token bound; TV(p, p~) = 1/2 sum_t |p_t - p~_t|.
+The machine-checked statement (Appendix A, "L1 main theorem") fixes the
+sign convention p_t = p~_t exp(-eps_t) / Z, i.e. eps_t = z~_t - z_t.
+
+§3 Thm. "Sound replacement": A = E_p~[e^c] and TV <= 1/2 (A^2 - 1).
+The meter is reported as min(1, .) (§4.3) and evaluated without truncating
+c; +inf on overflow is sound and counts as over threshold (§6.2.3
+telemetry).  Here 1/2 (A^2 - 1) is computed as 1/2 D (D + 2) with
+D = A - 1 = E_p~[expm1(c)], which is the same number without the
+cancellation of A^2 - 1 for small c (reading: the paper only asks for a
+numerically careful evaluation, "in the log domain").
+
+§4.1 Thm. "Sound black-box logit bound": |eps_t| = |q . r_t| / sqrt(d)
+<= (1/sqrt(d)) sum_b ||q_b|| w_{t,b} =: c_t.
+
+Gate (§6 meter-loop box; §4.3 certified vs risk-ranked): a (layer, head)
+falls back when its meter exceeds tau.  Reading: keep the compressed path
+iff meter_raw <= tau (so equality keeps, NaN falls back), evaluated in
+float32 on the float32 meter_raw; a KV head keeps its compressed cache only
+if all G query heads sharing it keep (any-of-G fallback, §5 statistics "at
+KV-head any-of-G granularity").
+"""
+
+import numpy as np
+
+from . import quantizer
+
+
+def softmax(z):
+    z = np.asarray(z, dtype=np.float64)
+    m = np.max(z, axis=-1, keepdims=True)
+    e = np.exp(z - m)
+    return e / np.sum(e, axis=-1, keepdims=True)
+
+
+def total_variation(p, p_tilde):
+    return 0.5 * np.sum(np.abs(np.asarray(p) - np.asarray(p_tilde)), axis=-1)
+
+
+def perturbed(p_tilde, eps):
+    """p_t = p~_t exp(-eps_t) / Z (Appendix A, L1 hypothesis)."""
+    w = np.asarray(p_tilde, dtype=np.float64) * np.exp(-np.asarray(eps, dtype=np.float64))
+    return w / np.sum(w, axis=-1, keepdims=True)
+
+
+def flawed_bound(p_tilde, c):
+    """§3 Eq. (flawed): 1/2 e^{2 cmax} (E|c - cbar| + cbar (e^{cmax} - 1)).
+
+    Unsound; kept only so the tests can show the paper's counterexample.
+    """
+    p_tilde = np.asarray(p_tilde, dtype=np.float64)
+    c = np.asarray(c, dtype=np.float64)
+    cbar = np.sum(p_tilde * c, axis=-1)
+    cmax = np.max(c, axis=-1)
+    disp = np.sum(p_tilde * np.abs(c - cbar[..., None]), axis=-1)
+    return 0.5 * np.exp(2 * cmax) * (disp + cbar * np.expm1(cmax))
+
+
+def eform_meter(p_tilde, c):
+    """Returns (meter, meter_raw, A) for A = E_p~[e^c]."""
+    p_tilde = np.asarray(p_tilde, dtype=np.float64)
+    c = np.asarray(c, dtype=np.float64)
+    with np.errstate(over="ignore", invalid="ignore"):
+        terms = p_tilde * np.expm1(c)
+        terms = np.where(p_tilde == 0, 0.0, terms)      # 0 * e^huge is 0 mass
+        D = np.sum(terms, axis=-1)
+        raw = 0.5 * D * (D + 2.0)
+    raw = np.where(np.isnan(raw), np.inf, raw)
+    return np.minimum(1.0, raw), raw, 1.0 + D
+
+
+def tier_a_bound(q, w, num_bands, rope_layout):
+    """c_t = (1/sqrt(d)) sum_b ||q_b|| w_{t,b}.
+
+    q: [..., d]; w: [..., S, B] stored witness; returns [..., S].
+    """
+    q = np.asarray(q, dtype=np.float64)
+    d = q.shape[-1]
+    qn = quantizer.band_norms(q, num_bands, rope_layout)          # [..., B]
+    w = np.asarray(w, dtype=np.float64)
+    return np.einsum("...b,...sb->...s", qn, w) / np.sqrt(d)
+
+
+def logits(q, k):
+    """z_t = q . k_t / sqrt(d); q [..., d], k [..., S, d] -> [..., S]."""
+    q = np.asarray(q, dtype=np.float64)
+    k = np.asarray(k, dtype=np.float64)
+    return np.einsum("...d,...sd->...s", q, k) / np.sqrt(q.shape[-1])
+
+
+def attend(p, v):
+    """y = sum_t p_t v_t."""
+    return np.einsum("...s,...sd->...d", np.asarray(p, np.float64), np.asarray(v, np.float64))
+
+
+def gate(meter_raw, tau, group):
+    """Keep/fallback decisions from float32 meter_raw [..., n_cells].
+
+    Returns keep_q (bool, per query-head cell), keep_kv (bool, per group of
+    ``group`` consecutive cells) and the two kept counts.
+    """
+    mr = np.asarray(meter_raw, dtype=np.float32)
+    keep_q = mr <= np.float32(tau)
+    n = keep_q.shape[-1]
+    if n % group:
+        raise ValueError("cells must come in whole groups")
+    keep_kv = np.all(keep_q.reshape(keep_q.shape[:-1] + (n // group, group)), axis=-1)
+    return keep_q, keep_kv, int(np.sum(keep_q)), int(np.sum(keep_kv))

@@ -1,0 +1,146 @@
+"""The write path over a paged cache and one metered decode step.
+
+Test infrastructure only (see ``oracle/__init__.py``).
+
+Paged cache (PagedAttention-style token slots, §6.2.3; 16-token pages as in
+the serving runs of §6.2 and Table "serving"): slot = page * P + offset with
+P = page_size; per layer the arrays are
+
+  k_codes, v_codes  [num_pages, Hkv, P, d]   int8 (dither) or uint8 (fp8 bytes)
+  k_scale, v_scale  [num_pages, Hkv, P]      fp16 (dither scheme only)
+  k_witness         [num_pages, Hkv, P, B]   fp16
+
+The meter loop (§6 box): write path quantizes k -> k^ and stores the
+witness; the read path computes the compressed attention and
+A = sum_t p~_t e^{c_t}; meter = min(1, 1/2 (A^2 - 1)); the gate compares it
+with tau.  The query head h_q reads KV head h_q // G (grouped-query
+attention, G = Hq / Hkv).
+"""
+
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import meter as M
+from . import fp, philox, quantizer
+
+SCHEME_DITHER_INT8 = 0
+SCHEME_FP8_E4M3 = 1
+
+
+@dataclass
+class Desc:
+    head_dim: int = 128
+    num_q_heads: int = 8
+    num_kv_heads: int = 2
+    num_bands: int = 8
+    page_size: int = 16
+    num_pages: int = 256
+    scheme: int = SCHEME_DITHER_INT8
+    rope_layout: int = quantizer.ROPE_HALF
+    dither_bits: int = 8
+    seed: int = 0
+
+
+def empty_cache(desc):
+    shp = (desc.num_pages, desc.num_kv_heads, desc.page_size)
+    code_t = np.int8 if desc.scheme == SCHEME_DITHER_INT8 else np.uint8
+    cache = {
+        "k_codes": np.zeros(shp + (desc.head_dim,), code_t),
+        "v_codes": np.zeros(shp + (desc.head_dim,), code_t),
+        "k_witness": np.zeros(shp + (desc.num_bands,), np.float16),
+    }
+    if desc.scheme == SCHEME_DITHER_INT8:
+        cache["k_scale"] = np.zeros(shp, np.float16)
+        cache["v_scale"] = np.zeros(shp, np.float16)
+    return cache
+
+
+def quantize_rows(desc, layer, kv_head, rows16, slots, tag):
+    """Quantize fp16 rows [n, d] written to ``slots``.
+
+    Returns (codes, scale or None, reconstruction float64 [n, d]).
+    """
+    if desc.scheme == SCHEME_DITHER_INT8:
+        s = quantizer.int8_scale(rows16)
+        j = philox.dither_integers(desc.seed, layer, kv_head, slots, tag,
+                                   desc.head_dim, desc.dither_bits)
+        xi = philox.dither_values(j, desc.dither_bits)
+        code = quantizer.dither_code(rows16, s, xi)
+        return code, s, quantizer.dither_reconstruct(code, s, xi)
+    code, rec = quantizer.fp8_quantize(rows16)
+    return code, None, rec
+
+
+def write_tokens(desc, layer, k16, v16, slot_mapping, cache):
+    """kv_quantize_witness: k16, v16 [n_tok, Hkv, d] fp16; slot < 0 skips."""
+    slot_mapping = np.asarray(slot_mapping, dtype=np.int64)
+    live = slot_mapping >= 0
+    slots = slot_mapping[live]
+    page, off = slots // desc.page_size, slots % desc.page_size
+    for h in range(desc.num_kv_heads):
+        kr = np.asarray(k16)[live, h, :]
+        vr = np.asarray(v16)[live, h, :]
+        kc, ks, khat = quantize_rows(desc, layer, h, kr, slots, 0)
+        vc, vs, _ = quantize_rows(desc, layer, h, vr, slots, 1)
+        cache["k_codes"][page, h, off] = kc
+        cache["v_codes"][page, h, off] = vc
+        if ks is not None:
+            cache["k_scale"][page, h, off] = ks
+            cache["v_scale"][page, h, off] = vs
+        resid = khat - kr.astype(np.float64)
+        cache["k_witness"][page, h, off] = quantizer.witness(
+            resid, desc.num_bands, desc.rope_layout)
+
+
+def slots_of(desc, block_table_row, ctx_len):
+    t = np.arange(ctx_len)
+    return np.asarray(block_table_row)[t // desc.page_size] * desc.page_size + t % desc.page_size
+
+
+def reconstruct(desc, layer, kv_head, slots, cache):
+    """Dequantized k^, v^ [S, d] float64 and the stored witness [S, B]."""
+    page, off = slots // desc.page_size, slots % desc.page_size
+    kc = cache["k_codes"][page, kv_head, off]
+    vc = cache["v_codes"][page, kv_head, off]
+    if desc.scheme == SCHEME_DITHER_INT8:
+        xk = philox.dither_values(philox.dither_integers(
+            desc.seed, layer, kv_head, slots, 0, desc.head_dim, desc.dither_bits), desc.dither_bits)
+        xv = philox.dither_values(philox.dither_integers(
+            desc.seed, layer, kv_head, slots, 1, desc.head_dim, desc.dither_bits), desc.dither_bits)
+        khat = quantizer.dither_reconstruct(kc, cache["k_scale"][page, kv_head, off], xk)
+        vhat = quantizer.dither_reconstruct(vc, cache["v_scale"][page, kv_head, off], xv)
+    else:
+        khat, vhat = fp.e4m3_decode(kc), fp.e4m3_decode(vc)
+    return khat, vhat, cache["k_witness"][page, kv_head, off]
+
+
+def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
+                    k_exact=None, v_exact=None):
+    """metered_decode_attention for one sequence: q16 [Hq, d] post-RoPE.
+
+    Returns a dict with float64 ``out`` [Hq, d], ``meter``/``meter_raw``
+    [Hq]; with the exact fp16 keys/values [S, Hkv, d] also ``tv`` [Hq]
+    (the true TV between exact and compressed attention) and
+    ``out_exact`` [Hq, d].
+    """
+    G = desc.num_q_heads // desc.num_kv_heads
+    d = desc.head_dim
+    slots = slots_of(desc, block_table_row, ctx_len)
+    res = {k: np.zeros((desc.num_q_heads, d)) for k in ("out", "out_exact")}
+    for k in ("meter", "meter_raw", "tv", "A"):
+        res[k] = np.zeros(desc.num_q_heads)
+    for h in range(desc.num_kv_heads):
+        khat, vhat, w = reconstruct(desc, layer, h, slots, cache)
+        for g in range(G):
+            hq = h * G + g
+            q = np.asarray(q16[hq], dtype=np.float64)
+            p_tilde = M.softmax(M.logits(q, khat))
+            c = M.tier_a_bound(q, w, desc.num_bands, desc.rope_layout)
+            res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.eform_meter(p_tilde, c)
+            res["out"][hq] = M.attend(p_tilde, vhat)
+            if k_exact is not None:
+                p = M.softmax(M.logits(q, np.asarray(k_exact)[:ctx_len, h]))
+                res["tv"][hq] = M.total_variation(p, p_tilde)
+                res["out_exact"][hq] = M.attend(p, np.asarray(v_exact)[:ctx_len, h])
+    return res
