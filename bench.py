@@ -1,0 +1,427 @@
+"""Benchmark of the WitCert hot path on GB300: metered decode KV tokens/s,
+achieved HBM GB/s against the measured peak, and witness-write GB/s.
+
+One step = one decode step of the workload: for every layer, write the
+newest token of every sequence (quantize + witness) and run the metered
+decode attention over the whole context; then gate all (layer, sequence,
+query head) meters at tau.  The step is captured once in a CUDA graph and
+replayed.  Default workload: 28 layers, 28 query / 4 KV heads, head_dim 128,
+one sequence of 32768 tokens, dithered INT8 cache, tau = 0.1.
+
+    python bench.py [--gpus N --steps K --warmup W] [--config 1..5] [--impl ours|reference]
+
+Multi-GPU (torchrun): every rank runs its own sequences (different seeds)
+with no collective on the data path; a barrier brackets the timed region and
+the slowest rank's time is used (weak scaling).
+"""
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import workloads as W  # noqa: E402
+
+BYTES_PER_TOKEN_HEAD = {0: 276, 1: 272}     # decode bytes read per token per KV head
+WRITE_BYTES_PER_TOKEN_HEAD = {0: 512 + 276, 1: 512 + 272}
+METRIC = "metered decode KV tokens/s & HBM GB/s vs 8 TB/s; witness-write GB/s"
+
+
+def _peaks():
+    try:
+        return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling during the timed region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except FileNotFoundError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc:
+            time.sleep(0.2)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---------------------------------------------------------------------------
+# our arm
+# ---------------------------------------------------------------------------
+
+class Setup:
+    """Caches, queries and the per-step buffers of one workload on one GPU."""
+
+    def __init__(self, wl, dither_bits=8):
+        import paper_2607_28699_gb300 as wc
+        self.wc, self.wl = wc, wl
+        self.desc = wc.CacheDesc(num_q_heads=wl.n_q_heads, num_kv_heads=wl.n_kv_heads,
+                                 num_pages=wl.num_pages, scheme=wl.scheme, dither_bits=dither_bits,
+                                 seed=wl.seed * 7919 + 1)
+        bt = W.block_tables(wl)
+        sm = W.slot_mapping(wl, bt)
+        self.bt = torch.from_numpy(bt).cuda()
+        self.sm = torch.from_numpy(sm).cuda()
+        self.ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+        last = np.cumsum(wl.ctx_lens) - 1                       # index of each sequence's newest token
+        self.new_slots = self.sm[torch.from_numpy(last).cuda()].contiguous()
+        self.caches, self.k_new, self.v_new = [], [], []
+        self.prefill_write_s = 0.0
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        for layer in range(wl.n_layers):
+            k, v = W.layer_kv(wl, layer, device="cuda")
+            cache = wc.LayerCache.empty(self.desc)
+            torch.cuda.synchronize()
+            s.record()
+            wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, cache)
+            e.record()
+            e.synchronize()
+            self.prefill_write_s += s.elapsed_time(e) / 1e3
+            self.caches.append(cache)
+            li = torch.from_numpy(last).cuda()
+            self.k_new.append(k[li].contiguous())
+            self.v_new.append(v[li].contiguous())
+            del k, v
+        self.q = torch.stack([W.layer_queries(wl, layer, device="cuda") for layer in range(wl.n_layers)])
+        self.ws = wc.Workspace(self.desc, wl.batch, wl.max_pages)
+        L, B, Hq = wl.n_layers, wl.batch, wl.n_q_heads
+        self.out = torch.empty(L, B, Hq, 128, dtype=torch.float32, device="cuda")
+        self.meter = torch.empty(L, B, Hq, dtype=torch.float32, device="cuda")
+        self.raw = torch.empty(L, B, Hq, dtype=torch.float32, device="cuda")
+        self.keep_q = torch.empty(L * B * Hq, dtype=torch.uint8, device="cuda")
+        self.keep_kv = torch.empty(L * B * Hq // wl.group, dtype=torch.uint8, device="cuda")
+        self.n_kept = torch.empty(2, dtype=torch.int32, device="cuda")
+        self.ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                   for _ in range(L)]
+        self.tau = wl.taus[0]
+
+    def step(self, timed_events=True):
+        wc, wl = self.wc, self.wl
+        for layer in range(wl.n_layers):
+            wc.kv_quantize_witness(self.desc, layer, self.k_new[layer], self.v_new[layer], self.new_slots,
+                                   self.caches[layer])
+            if timed_events:
+                self.ev[layer][0].record()
+            wc.metered_decode_attention(self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer],
+                                        self.ws, out=self.out[layer], meter=self.meter[layer],
+                                        meter_raw=self.raw[layer])
+            if timed_events:
+                self.ev[layer][1].record()
+        wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
+
+    def launches_per_step(self):
+        return 2 * self.wl.n_layers + 1
+
+    def decode_bytes_per_launch(self):
+        return sum(self.wl.ctx_lens) * self.wl.n_kv_heads * BYTES_PER_TOKEN_HEAD[self.wl.scheme]
+
+
+def capture(fn, stream):
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.stream(stream):
+        fn()                                   # warm once outside capture (lazy init)
+    torch.cuda.synchronize()
+    with torch.cuda.graph(g, stream=stream):
+        fn()
+    torch.cuda.synchronize()
+    return g
+
+
+def run_ours(args, rank, world, local):
+    wl = W.config(args.config, seed=args.seed + rank)
+    if args.layers:
+        wl.n_layers = args.layers
+    st = Setup(wl, dither_bits=args.dither_bits)
+    stream = torch.cuda.Stream()
+    graph = capture(st.step, stream)
+
+    # ---- device-resident timed region ----------------------------------
+    for _ in range(args.warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clk:
+        torch.cuda.synchronize()
+        t0.record(stream)
+        for _ in range(args.steps):
+            graph.replay()
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    ms = t0.elapsed_time(t1) / args.steps
+    ms = max_over_ranks(ms, world)
+    dec_ms = [a.elapsed_time(b) for a, b in st.ev]            # last replay, per layer
+    dec_avg_ms = sum(dec_ms) / len(dec_ms)
+    st.wc.read_status(st.ws)
+
+    kv_tokens_step = wl.kv_tokens
+    value = kv_tokens_step * world / (ms / 1e3)
+    algo_bytes = st.decode_bytes_per_launch()
+    peaks = _peaks() or {}
+    peak = peaks.get("hbm_gbs", 6800.0)
+    achieved = algo_bytes / (dec_avg_ms / 1e3) / 1e9
+    step_gbs = algo_bytes * wl.n_layers / (ms / 1e3) / 1e9
+
+    # ---- end-to-end: host buffers, copies inside the timed region --------
+    e2e = run_e2e(st, args, stream, world)
+
+    # ---- write path: full prefill write of the cache ---------------------
+    write_th = sum(wl.ctx_lens) * wl.n_layers * wl.n_kv_heads
+    write_gbs = write_th * WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme] / st.prefill_write_s / 1e9
+
+    # ---- gate summary ---------------------------------------------------------
+    kept = st.n_kept.cpu().tolist()
+    ncell = wl.n_layers * wl.batch * wl.n_q_heads
+    coverage = {"tau": st.tau, "kept_q_frac": kept[0] / ncell, "kept_kv_frac": kept[1] / (ncell // wl.group)}
+    meters = st.raw.reshape(-1).cpu().numpy()
+    coverage["meter_raw_median"] = float(np.median(meters))
+    coverage["overflow_cells"] = int(np.sum(~np.isfinite(meters)))
+
+    res = {
+        "metric": METRIC, "value": value, "unit": "KV tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int8-dither+fp16-mma/fp32" if wl.scheme == 0 else "fp8-e4m3+fp16-mma/fp32",
+        "data": "synthetic (seeded; log-normal outlier channels, 8x sink token, RoPE theta 1e4)",
+        "config": {"workload": wl.name, "layers": wl.n_layers, "q_heads": wl.n_q_heads,
+                   "kv_heads": wl.n_kv_heads, "head_dim": 128, "batch": wl.batch,
+                   "ctx_tokens": sum(wl.ctx_lens), "page": 16, "dither_bits": args.dither_bits,
+                   "tau": st.tau, "parallelism": f"replica-per-gpu x{world}",
+                   "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step > 129 MB L2; no flush"},
+        "hbm_gbs_step": step_gbs,
+        "decode_kernel_ms": dec_avg_ms,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "traffic": None,
+                     "frac_of_nominal_8tbs": achieved / 8000.0,
+                     "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peaks else "fallback 6.8 TB/s",
+                     "algorithmic_bytes_per_launch": algo_bytes},
+        "witness_write": {"gbs": write_gbs, "token_heads_per_s": write_th / st.prefill_write_s,
+                          "bytes_per_token_head": WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme]},
+        "gate": coverage,
+        "gpu_launches": st.launches_per_step() * args.steps,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline(wl, args)
+    return res
+
+
+def run_e2e(st, args, stream, world):
+    """Same step with inputs copied from pinned host memory and results read back."""
+    wl = st.wl
+    host_q = st.q.cpu().pin_memory()
+    host_k = torch.stack(st.k_new).cpu().pin_memory()
+    host_v = torch.stack(st.v_new).cpu().pin_memory()
+    host_ctx = st.ctx.cpu().pin_memory()
+    dev_k = torch.stack(st.k_new)
+    dev_v = torch.stack(st.v_new)
+    out_h = torch.empty_like(st.out, device="cpu").pin_memory()
+    raw_h = torch.empty_like(st.raw, device="cpu").pin_memory()
+    meter_h = torch.empty_like(st.meter, device="cpu").pin_memory()
+    keep_h = torch.empty_like(st.keep_q, device="cpu").pin_memory()
+    kept_h = torch.empty_like(st.n_kept, device="cpu").pin_memory()
+
+    def e2e_step():
+        st.q.copy_(host_q, non_blocking=True)
+        dev_k.copy_(host_k, non_blocking=True)
+        dev_v.copy_(host_v, non_blocking=True)
+        st.ctx.copy_(host_ctx, non_blocking=True)
+        for layer in range(wl.n_layers):
+            st.k_new[layer].copy_(dev_k[layer], non_blocking=True)
+            st.v_new[layer].copy_(dev_v[layer], non_blocking=True)
+        st.step(timed_events=False)
+        out_h.copy_(st.out, non_blocking=True)
+        raw_h.copy_(st.raw, non_blocking=True)
+        meter_h.copy_(st.meter, non_blocking=True)
+        keep_h.copy_(st.keep_q, non_blocking=True)
+        kept_h.copy_(st.n_kept, non_blocking=True)
+
+    g = capture(e2e_step, stream)
+    for _ in range(max(3, args.warmup)):
+        g.replay()
+    torch.cuda.synchronize()
+    barrier(world)
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        g.replay()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier(world)
+    ms = max_over_ranks(t0.elapsed_time(t1) / args.steps, world)
+    bi = sum(t.numel() * t.element_size() for t in (host_q, host_k, host_v, host_ctx))
+    bo = sum(t.numel() * t.element_size() for t in (out_h, raw_h, meter_h, keep_h, kept_h))
+    return {"value": wl.kv_tokens * world / (ms / 1e3), "unit": "KV tokens/s", "ms_per_step": ms,
+            "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo}
+
+
+# ---------------------------------------------------------------------------
+# oracle legs (CPU)
+# ---------------------------------------------------------------------------
+
+def _oracle_sample(wl, budget_s, seed_layer=0):
+    """Time the oracle's decode of whole layers (all KV heads) of the
+    workload until ``budget_s`` of CPU time is spent; returns KV tokens/s."""
+    from oracle import pipeline as OP
+    od = OP.Desc(num_q_heads=wl.n_q_heads, num_kv_heads=wl.n_kv_heads, num_pages=wl.num_pages,
+                 scheme=wl.scheme, dither_bits=8, seed=wl.seed * 7919 + 1)
+    bt = W.block_tables(wl)
+    sm = W.slot_mapping(wl, bt)
+    done_tokens, spent, layers = 0, 0.0, 0
+    seqs = min(wl.batch, 2)
+    while spent < budget_s and layers < wl.n_layers:
+        layer = (seed_layer + layers) % wl.n_layers
+        k, v = W.layer_kv(wl, layer, seq_range=(0, seqs))
+        q = W.layer_queries(wl, layer)
+        cache = OP.empty_cache(od)
+        n = sum(wl.ctx_lens[:seqs])
+        OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm[:n], cache)
+        t = time.perf_counter()
+        for b in range(seqs):
+            OP.decode_sequence(od, layer, q[b].numpy(), bt[b], wl.ctx_lens[b], cache)
+        spent += time.perf_counter() - t
+        done_tokens += n
+        layers += 1
+    return done_tokens / spent, f"oracle decode of {layers} layer(s) x {seqs} sequence(s) x all KV heads " \
+                                f"({done_tokens} KV tokens), {spent:.1f} s", spent
+
+
+def cpu_baseline(wl, args):
+    tok_s, sample, _ = _oracle_sample(wl, args.cpu_budget)
+    return {"value": tok_s, "unit": "KV tokens/s", "cores": 1, "kind": "oracle", "sample": sample,
+            "host_cores_available": os.cpu_count()}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return None
+    wl = W.config(args.config, seed=args.seed)
+    per_step = []
+    sample = ""
+    for _ in range(args.warmup):
+        _oracle_sample(wl, 0.0)
+    for i in range(args.steps):
+        tok_s, sample, spent = _oracle_sample(wl, args.cpu_budget / max(args.steps, 1), seed_layer=i)
+        per_step.append(tok_s)
+    value = statistics.median(per_step)
+    ms = wl.kv_tokens / value * 1e3
+    return {"metric": METRIC, "value": value, "unit": "KV tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded)", "impl": "reference",
+            "config": {"workload": wl.name, "parallelism": "single CPU process (oracle)"},
+            "cpu_baseline": {"value": value, "unit": "KV tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": "KV tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--config", type=int, default=2)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling only)")
+    ap.add_argument("--dither-bits", type=int, default=8)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        res = run_reference(args, rank, world)
+        if res is not None:
+            print(json.dumps(res))
+        return
+    torch.cuda.set_device(local)
+    if world > 1:
+        torch.distributed.init_process_group("nccl")
+    res = run_ours(args, rank, world, local)
+    if rank == 0:
+        print(json.dumps(res))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

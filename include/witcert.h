@@ -1,0 +1,203 @@
+/*
+ * witcert.h -- C ABI of the WitCert metered-KV-cache library for GB300
+ * (sm_103a).  Paper: "WitCert: Sound Runtime Risk Observability and Gating
+ * for KV-Cache Quantization", arxiv 2607.28699.
+ *
+ * The library implements the meter loop of §6 (box "The meter loop"): a
+ * write path that quantizes post-RoPE keys/values and stores a per-token
+ * band-norm residual witness, a fused decode-attention read path that also
+ * computes the per-(layer, head, step) total-variation meter, and a gate.
+ *
+ * Conventions shared by every entry point
+ *  - All tensor arguments are DEVICE pointers owned by the caller; the
+ *    library allocates no memory and never synchronises the host with the
+ *    device (kernels are enqueued on the caller's stream).  The only
+ *    exception is wc_read_status, which synchronises the given stream.
+ *  - Arguments are validated on the host before any launch.  On failure the
+ *    call returns a non-zero wc_status, launches nothing and leaves a message
+ *    for wc_last_error() (thread-local).
+ *  - Faults that only the device can see (a page index outside the pool, a
+ *    slot outside the pool, an asynchronous copy that did not complete within
+ *    its bounded wait) are never trapped: the offending token or page is
+ *    skipped and a bit is OR-ed into a caller-visible 32-bit status word.
+ *  - All tensors are dense, row-major, 16-byte aligned (the decode kernel
+ *    stages pages with bulk asynchronous copies).
+ *  - head_dim = 128, page_size = 16, num_bands = 8 and 1 <= G <= 8 query heads
+ *    per KV head are the supported shapes (the paper's 7B-class shapes).
+ *
+ * Paged cache layout for ONE layer (PagedAttention-style token slots; a
+ * slot is page * 16 + offset; §6.2.3 "Storage side"):
+ *   k_codes, v_codes [num_pages][Hkv][16][128]  int8 (WC_SCHEME_DITHER_INT8)
+ *                                               or fp8 e4m3fn bytes (WC_SCHEME_FP8_E4M3)
+ *   k_scale, v_scale [num_pages][Hkv][16]       fp16, dither scheme only (else NULL)
+ *   k_witness        [num_pages][Hkv][16][8]    fp16, per-band residual norms
+ */
+#ifndef WITCERT_H
+#define WITCERT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int wc_status;
+enum {
+    WC_OK = 0,
+    WC_ERR_INVALID_ARG = 1,   /* null pointer, bad size or misaligned tensor      */
+    WC_ERR_UNSUPPORTED = 2,   /* a shape or option this build does not implement  */
+    WC_ERR_CUDA = 3,          /* a CUDA runtime call failed (message has details) */
+    WC_ERR_WORKSPACE = 4,     /* workspace smaller than wc_workspace_size()       */
+    WC_ERR_DEVICE_CHECK = 5   /* wc_read_status found device-side fault bits      */
+};
+
+/* Device status bits (wc_read_status, or the word a write call points to). */
+enum {
+    WC_DEV_BAD_SLOT = 1u,     /* write: slot >= num_pages * 16; token skipped    */
+    WC_DEV_BAD_PAGE = 2u,     /* decode: block-table page outside [0, num_pages)  */
+    WC_DEV_BAD_CTX = 4u,      /* decode: context length < 0 or > max_pages * 16   */
+    WC_DEV_TIMEOUT = 8u       /* decode: a bounded wait for staged data gave up   */
+};
+
+typedef enum {
+    /* Controlled quantizer of §4.2 ("Subtractive dither"): per token and KV
+     * head, s = fp16_rn(fp32(amax) / 126.5f), code = round-half-even of the
+     * exact x/s + xi clamped to [-127, 127], reconstruction s * (code - xi). */
+    WC_SCHEME_DITHER_INT8 = 0,
+    /* Black-box raw cast to fp8 e4m3fn (round to nearest even, saturating
+     * finite overflow to +-448), no scale, no dither (§4.1, Fig. f5). */
+    WC_SCHEME_FP8_E4M3 = 1
+} wc_scheme;
+
+typedef enum {
+    /* RoPE frequency pair j occupies dims (j, j + 64) (half rotation). */
+    WC_ROPE_HALF = 0,
+    /* RoPE frequency pair j occupies dims (2j, 2j + 1) (interleaved). */
+    WC_ROPE_INTERLEAVED = 1
+} wc_rope_layout;
+
+/* Static description of one model's paged cache. */
+typedef struct {
+    int32_t head_dim;       /* must be 128                                        */
+    int32_t num_q_heads;    /* Hq; Hq % Hkv == 0 and Hq / Hkv <= 8                 */
+    int32_t num_kv_heads;   /* Hkv, 1 .. 65535                                     */
+    int32_t num_bands;      /* B, must be 8: 64 RoPE pairs in 8 contiguous bands   */
+    int32_t page_size;      /* must be 16                                          */
+    int32_t num_pages;      /* pages in each layer's pool                          */
+    int32_t scheme;         /* wc_scheme                                           */
+    int32_t rope_layout;    /* wc_rope_layout                                      */
+    int32_t dither_bits;    /* 8 or 10 (dither scheme): resolution of xi           */
+    int32_t reserved;       /* must be 0                                           */
+    uint64_t seed;          /* Philox key (lo, hi 32 bits)                         */
+} wc_cache_desc;
+
+/*
+ * Write path ("write kernel", §6.2.1; witness Eq. (witness), §4.1).
+ *
+ * For each token t < n_tok and KV head h, quantizes the post-RoPE fp16 rows
+ * k[t][h][:] and v[t][h][:] with desc->scheme, writes the codes (and fp16
+ * scales for the dither scheme) to slot slot_mapping[t] of this layer's
+ * cache, and stores the K witness w_b = fp16_round_up(||k^_b - k_b||) for
+ * the 8 RoPE bands.  The dither xi is Philox4x32-10 under key
+ * (seed lo, seed hi) at counter (slot, layer * 65536 + h, group, tag), tag 0
+ * for K and 1 for V; with dither_bits = 8 one counter covers 16 channels
+ * (channel i of group g is byte i % 4 of word i / 4), with 10 it covers 8
+ * (bits 16 * (i % 2) .. +9 of word i / 2); integer j maps to
+ * xi = (j + 1/2) / 2^bits - 1/2.  The witness may exceed the exactly rounded
+ * norm by one fp16 ulp (it is computed in fp32 and rounded up with margin),
+ * never fall below it.
+ *
+ *   layer          0 .. 65535, keys the dither
+ *   k, v           [n_tok][Hkv][128] fp16, device
+ *   slot_mapping   [n_tok] int32, device; a negative slot skips the token,
+ *                  a slot >= num_pages * 16 skips it and sets WC_DEV_BAD_SLOT
+ *   k_scale,v_scale NULL for WC_SCHEME_FP8_E4M3
+ *   dev_status     optional device uint32 that collects WC_DEV_* bits (OR)
+ * Rows written by the same call must have distinct slots.
+ */
+wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer,
+                                 const void* k, const void* v,
+                                 const int32_t* slot_mapping, int32_t n_tok,
+                                 void* k_codes, void* v_codes,
+                                 void* k_scale, void* v_scale, void* k_witness,
+                                 uint32_t* dev_status, void* stream);
+
+/*
+ * Bytes of workspace wc_metered_decode_attention needs for `batch`
+ * sequences whose block tables hold `max_pages` pages, on the current
+ * device (the split count depends on its SM count).  Returns 0 and sets
+ * wc_last_error() on invalid arguments.  The workspace must be zero-filled
+ * once after allocation; each call leaves it ready for the next one.
+ */
+size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_pages);
+
+/*
+ * Metered decode attention (read path, §6.2.1-§6.2.2; Thm. "Sound black-box
+ * logit bound"; Thm. "Sound replacement").
+ *
+ * For every sequence b and query head hq (KV head hq / G) over the
+ * ctx_lens[b] cached tokens of this layer:
+ *   out[b][hq][:]   = sum_t p~_t v^_t, p~ = softmax_t(q . k^_t / sqrt(128))
+ *   c_t             = (1/sqrt(128)) sum_b ||q_b|| w_{t,b}
+ *   meter_raw[b][hq] = 1/2 (A^2 - 1), A = sum_t p~_t e^{c_t}  (+inf on fp32 overflow)
+ *   meter[b][hq]    = min(1, meter_raw)
+ * The context is split across CTAs; partial softmax, output and A
+ * accumulators are merged under log-sum-exp weights (A is a p~-weighted mean,
+ * §6.2.2), by the last CTA of each (sequence, KV head).  A sequence with
+ * ctx_len 0 gets out = 0 and meter = meter_raw = 0.
+ *
+ *   q            [batch][Hq][128] fp16 post-RoPE queries, device
+ *   block_table  [batch][max_pages] int32 physical page of each logical page
+ *   ctx_lens     [batch] int32, 0 .. max_pages * 16
+ *   out          [batch][Hq][128] fp32; meter, meter_raw [batch][Hq] fp32
+ *   workspace    >= wc_workspace_size(desc, batch, max_pages) bytes, zeroed
+ *                once; holds the device status word (wc_read_status)
+ * Calls sharing one workspace must be ordered on one stream.
+ */
+wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer,
+                                      const void* q, const int32_t* block_table,
+                                      int32_t max_pages, const int32_t* ctx_lens,
+                                      int32_t batch,
+                                      const void* k_codes, const void* v_codes,
+                                      const void* k_scale, const void* v_scale,
+                                      const void* k_witness,
+                                      float* out, float* meter, float* meter_raw,
+                                      void* workspace, size_t workspace_bytes,
+                                      void* stream);
+
+/*
+ * Gate (§6 meter-loop box; certified tau < 1 vs risk-ranked tau >= 1, §4.3).
+ *
+ * keep_q[i] = (meter_raw[i] <= tau) in fp32 (equality keeps the compressed
+ * path; +inf and NaN fall back).  Cells come in groups of `group`
+ * consecutive query heads sharing one KV head; keep_kv[i / group] = AND of
+ * its group (any-of-G fallback).  n_kept[0] = kept query-head cells,
+ * n_kept[1] = kept KV-head cells.  One CTA; no atomics; n_kept need not be
+ * zeroed.
+ *   meter_raw [n_cells] fp32; keep_q [n_cells] uint8; keep_kv [n_cells/group]
+ *   uint8; n_kept [2] int32 -- all device.
+ */
+wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau,
+                  uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept, void* stream);
+
+/*
+ * Synchronises `stream`, copies the device status word held in `workspace`
+ * (or pointed to by a write call's dev_status, when `is_status_word` != 0)
+ * to *bits, clears it on the device, and returns WC_ERR_DEVICE_CHECK if
+ * any bit was set.  Diagnostic only: the other calls never synchronise.
+ */
+wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word,
+                         uint32_t* bits, void* stream);
+
+/* Thread-local description of the last non-OK status on this thread. */
+const char* wc_last_error(void);
+
+/* Library version, (major << 16) | minor. */
+int32_t wc_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WITCERT_H */

@@ -1,0 +1,228 @@
+"""Python binding of the WitCert GB300 library (ctypes over ``include/witcert.h``).
+
+Argument marshalling only: every function passes device pointers, sizes and
+the current CUDA stream to the C ABI, where all work runs in the library's
+CUDA kernels.  PyTorch supplies device memory and streams.  There is no CPU
+fallback: importing this package without the compiled library raises.
+
+    import paper_2607_28699_gb300 as wc
+    desc = wc.CacheDesc(num_q_heads=28, num_kv_heads=4, num_pages=n)
+    cache = wc.LayerCache.empty(desc, device="cuda")
+    wc.kv_quantize_witness(desc, layer, k, v, slot_mapping, cache)
+    ws = wc.Workspace(desc, batch, max_pages)
+    out, meter, meter_raw = wc.metered_decode_attention(desc, layer, q, block_table,
+                                                        ctx_lens, cache, ws)
+    keep_q, keep_kv, n_kept = wc.gate(meter_raw, group, tau)
+"""
+
+import ctypes
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libwitcert.so")
+
+SCHEME_DITHER_INT8 = 0
+SCHEME_FP8_E4M3 = 1
+ROPE_HALF = 0
+ROPE_INTERLEAVED = 1
+DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT = 1, 2, 4, 8
+EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
+           "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
+
+
+class WitCertError(RuntimeError):
+    def __init__(self, status, message):
+        super().__init__(f"witcert status {status}: {message}")
+        self.status = status
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with "
+                          "`python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32, u64 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_uint64
+    lib.wc_kv_quantize_witness.argtypes = [vp, i32, vp, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp]
+    lib.wc_kv_quantize_witness.restype = ctypes.c_int
+    lib.wc_workspace_size.argtypes = [vp, i32, i32]
+    lib.wc_workspace_size.restype = ctypes.c_size_t
+    lib.wc_metered_decode_attention.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp,
+                                                vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.wc_metered_decode_attention.restype = ctypes.c_int
+    lib.wc_gate.argtypes = [vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]
+    lib.wc_gate.restype = ctypes.c_int
+    lib.wc_read_status.argtypes = [vp, i32, vp, vp]
+    lib.wc_read_status.restype = ctypes.c_int
+    lib.wc_last_error.argtypes = []
+    lib.wc_last_error.restype = ctypes.c_char_p
+    lib.wc_version.restype = ctypes.c_int32
+    del u64
+    return lib
+
+
+lib = _load()
+
+
+class _Desc(ctypes.Structure):
+    _fields_ = [("head_dim", ctypes.c_int32), ("num_q_heads", ctypes.c_int32),
+                ("num_kv_heads", ctypes.c_int32), ("num_bands", ctypes.c_int32),
+                ("page_size", ctypes.c_int32), ("num_pages", ctypes.c_int32),
+                ("scheme", ctypes.c_int32), ("rope_layout", ctypes.c_int32),
+                ("dither_bits", ctypes.c_int32), ("reserved", ctypes.c_int32),
+                ("seed", ctypes.c_uint64)]
+
+
+@dataclass
+class CacheDesc:
+    """Mirror of ``wc_cache_desc``."""
+    num_q_heads: int
+    num_kv_heads: int
+    num_pages: int
+    scheme: int = SCHEME_DITHER_INT8
+    rope_layout: int = ROPE_HALF
+    dither_bits: int = 8
+    seed: int = 0
+    head_dim: int = 128
+    num_bands: int = 8
+    page_size: int = 16
+
+    @property
+    def group(self):
+        return self.num_q_heads // self.num_kv_heads
+
+    def c(self):
+        return _Desc(self.head_dim, self.num_q_heads, self.num_kv_heads, self.num_bands,
+                     self.page_size, self.num_pages, self.scheme, self.rope_layout,
+                     self.dither_bits, 0, self.seed & (2 ** 64 - 1))
+
+
+def _check(status):
+    if status != 0:
+        raise WitCertError(status, lib.wc_last_error().decode())
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_contiguous():
+        raise ValueError("tensors passed to the library must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+@dataclass
+class LayerCache:
+    """One layer's paged cache tensors (layout in ``include/witcert.h``)."""
+    k_codes: torch.Tensor
+    v_codes: torch.Tensor
+    k_scale: Optional[torch.Tensor]
+    v_scale: Optional[torch.Tensor]
+    k_witness: torch.Tensor
+
+    @staticmethod
+    def empty(desc: CacheDesc, device="cuda"):
+        shp = (desc.num_pages, desc.num_kv_heads, desc.page_size)
+        code_t = torch.int8 if desc.scheme == SCHEME_DITHER_INT8 else torch.uint8
+        dither = desc.scheme == SCHEME_DITHER_INT8
+        return LayerCache(
+            torch.zeros(shp + (desc.head_dim,), dtype=code_t, device=device),
+            torch.zeros(shp + (desc.head_dim,), dtype=code_t, device=device),
+            torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
+            torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
+            torch.zeros(shp + (desc.num_bands,), dtype=torch.float16, device=device))
+
+    def nbytes(self):
+        return sum(t.numel() * t.element_size() for t in
+                   (self.k_codes, self.v_codes, self.k_scale, self.v_scale, self.k_witness) if t is not None)
+
+
+def kv_quantize_witness(desc: CacheDesc, layer: int, k: torch.Tensor, v: torch.Tensor,
+                        slot_mapping: torch.Tensor, cache: LayerCache,
+                        dev_status: Optional[torch.Tensor] = None, stream=None):
+    """``wc_kv_quantize_witness``: k, v fp16 [n_tok, Hkv, 128]; slots int32 [n_tok]."""
+    d = desc.c()
+    _check(lib.wc_kv_quantize_witness(
+        ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(dev_status), _stream(stream)))
+
+
+def workspace_size(desc: CacheDesc, batch: int, max_pages: int) -> int:
+    d = desc.c()
+    n = lib.wc_workspace_size(ctypes.byref(d), batch, max_pages)
+    if n == 0:
+        raise WitCertError(1, lib.wc_last_error().decode())
+    return n
+
+
+class Workspace:
+    """Zero-filled device workspace for ``metered_decode_attention``."""
+
+    def __init__(self, desc: CacheDesc, batch: int, max_pages: int, device="cuda"):
+        self.nbytes = workspace_size(desc, batch, max_pages)
+        self.buf = torch.zeros(self.nbytes + 256, dtype=torch.uint8, device=device)
+        off = (-self.buf.data_ptr()) % 256
+        self.view = self.buf[off:off + self.nbytes]
+
+    def ptr(self):
+        return ctypes.c_void_p(self.view.data_ptr())
+
+
+def metered_decode_attention(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
+                             ctx_lens: torch.Tensor, cache: LayerCache, ws: Workspace,
+                             out=None, meter=None, meter_raw=None, stream=None):
+    """``wc_metered_decode_attention``; returns (out [B,Hq,128], meter [B,Hq], meter_raw [B,Hq]) fp32."""
+    batch, max_pages = block_table.shape
+    dev = q.device
+    if out is None:
+        out = torch.empty(batch, desc.num_q_heads, desc.head_dim, dtype=torch.float32, device=dev)
+    if meter is None:
+        meter = torch.empty(batch, desc.num_q_heads, dtype=torch.float32, device=dev)
+    if meter_raw is None:
+        meter_raw = torch.empty(batch, desc.num_q_heads, dtype=torch.float32, device=dev)
+    d = desc.c()
+    _check(lib.wc_metered_decode_attention(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(out), _ptr(meter), _ptr(meter_raw), ws.ptr(), ws.nbytes,
+        _stream(stream)))
+    return out, meter, meter_raw
+
+
+def gate(meter_raw: torch.Tensor, group: int, tau: float, keep_q=None, keep_kv=None, n_kept=None,
+         stream=None):
+    """``wc_gate``: returns (keep_q uint8 [n], keep_kv uint8 [n/group], n_kept int32 [2])."""
+    n = meter_raw.numel()
+    dev = meter_raw.device
+    keep_q = torch.empty(n, dtype=torch.uint8, device=dev) if keep_q is None else keep_q
+    keep_kv = torch.empty(n // group, dtype=torch.uint8, device=dev) if keep_kv is None else keep_kv
+    n_kept = torch.empty(2, dtype=torch.int32, device=dev) if n_kept is None else n_kept
+    _check(lib.wc_gate(_ptr(meter_raw), n, group, float(tau), _ptr(keep_q), _ptr(keep_kv),
+                       _ptr(n_kept), _stream(stream)))
+    return keep_q, keep_kv, n_kept
+
+
+def read_status(ws_or_word, stream=None) -> int:
+    """Synchronising read-and-clear of the device status word; returns the bits."""
+    if isinstance(ws_or_word, Workspace):
+        p, is_word = ws_or_word.ptr(), 0
+    else:
+        p, is_word = _ptr(ws_or_word), 1
+    bits = ctypes.c_uint32(0)
+    st = lib.wc_read_status(p, is_word, ctypes.byref(bits), _stream(stream))
+    if st not in (0, 5):
+        _check(st)
+    return bits.value
+
+
+def version():
+    v = lib.wc_version()
+    return (v >> 16, v & 0xFFFF)

@@ -1,0 +1,212 @@
+// extern "C" boundary: host-side argument checks and kernel launches.
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <string>
+
+#include "wc_kernels.cuh"
+
+namespace {
+
+thread_local std::string g_last_error;
+
+wc_status fail(wc_status st, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+wc_status fail(wc_status st, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return st;
+}
+
+wc_status cuda_fail(cudaError_t e, const char* what) {
+    return fail(WC_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+wc_status check_desc(const wc_cache_desc* d) {
+    if (!d) return fail(WC_ERR_INVALID_ARG, "desc is NULL");
+    if (d->head_dim != wc::kHeadDim) return fail(WC_ERR_UNSUPPORTED, "head_dim must be 128 (got %d)", d->head_dim);
+    if (d->page_size != wc::kPage) return fail(WC_ERR_UNSUPPORTED, "page_size must be 16 (got %d)", d->page_size);
+    if (d->num_bands != wc::kBands) return fail(WC_ERR_UNSUPPORTED, "num_bands must be 8 (got %d)", d->num_bands);
+    if (d->num_kv_heads < 1 || d->num_kv_heads > 65535)
+        return fail(WC_ERR_INVALID_ARG, "num_kv_heads must be in [1, 65535] (got %d)", d->num_kv_heads);
+    if (d->num_q_heads < 1 || d->num_q_heads % d->num_kv_heads != 0)
+        return fail(WC_ERR_INVALID_ARG, "num_q_heads (%d) must be a positive multiple of num_kv_heads (%d)",
+                    d->num_q_heads, d->num_kv_heads);
+    if (d->num_q_heads / d->num_kv_heads > wc::kMaxGroup)
+        return fail(WC_ERR_UNSUPPORTED, "at most %d query heads per KV head (got %d)", wc::kMaxGroup,
+                    d->num_q_heads / d->num_kv_heads);
+    if (d->num_pages < 1) return fail(WC_ERR_INVALID_ARG, "num_pages must be positive (got %d)", d->num_pages);
+    if ((long long)d->num_pages * wc::kPage > 0x7FFFFFFFLL)
+        return fail(WC_ERR_UNSUPPORTED, "num_pages * 16 must fit in int32");
+    if (d->scheme != WC_SCHEME_DITHER_INT8 && d->scheme != WC_SCHEME_FP8_E4M3)
+        return fail(WC_ERR_UNSUPPORTED, "unknown scheme %d", d->scheme);
+    if (d->rope_layout != WC_ROPE_HALF && d->rope_layout != WC_ROPE_INTERLEAVED)
+        return fail(WC_ERR_UNSUPPORTED, "unknown rope_layout %d", d->rope_layout);
+    if (d->scheme == WC_SCHEME_DITHER_INT8 && d->dither_bits != 8 && d->dither_bits != 10)
+        return fail(WC_ERR_UNSUPPORTED, "dither_bits must be 8 or 10 (got %d)", d->dither_bits);
+    if (d->reserved != 0) return fail(WC_ERR_INVALID_ARG, "reserved must be 0");
+    return WC_OK;
+}
+
+wc_status check_cache(const wc_cache_desc* d, const void* kc, const void* vc, const void* ks, const void* vs,
+                      const void* kw) {
+    if (!kc || !vc || !kw) return fail(WC_ERR_INVALID_ARG, "cache pointers must not be NULL");
+    if (!aligned16(kc) || !aligned16(vc) || !aligned16(kw))
+        return fail(WC_ERR_INVALID_ARG, "cache arrays must be 16-byte aligned");
+    if (d->scheme == WC_SCHEME_DITHER_INT8) {
+        if (!ks || !vs) return fail(WC_ERR_INVALID_ARG, "k_scale/v_scale are required by the dither scheme");
+        if (!aligned16(ks) || !aligned16(vs)) return fail(WC_ERR_INVALID_ARG, "scale arrays must be 16-byte aligned");
+    } else if (ks || vs) {
+        return fail(WC_ERR_INVALID_ARG, "k_scale/v_scale must be NULL for the fp8 scheme");
+    }
+    return WC_OK;
+}
+
+int current_sm_count(int* out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+    if (cudaDeviceGetAttribute(out, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return -1;
+    return 0;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t wc_version(void) { return (1 << 16) | 0; }
+
+const char* wc_last_error(void) { return g_last_error.c_str(); }
+
+wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
+                                 const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
+                                 void* k_scale, void* v_scale, void* k_witness, uint32_t* dev_status,
+                                 void* stream) {
+    if (wc_status st = check_desc(desc)) return st;
+    if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
+    if (n_tok < 0) return fail(WC_ERR_INVALID_ARG, "n_tok must be >= 0 (got %d)", n_tok);
+    if ((long long)n_tok * desc->num_kv_heads > 0x7FFFFFFFLL - 8)
+        return fail(WC_ERR_UNSUPPORTED, "n_tok * num_kv_heads must fit in int32");
+    if (n_tok > 0 && (!k || !v || !slot_mapping)) return fail(WC_ERR_INVALID_ARG, "k, v, slot_mapping must not be NULL");
+    if (!aligned16(k) || !aligned16(v)) return fail(WC_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
+    if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
+    if (n_tok == 0) return WC_OK;
+    wc::WriteParams p;
+    p.k = static_cast<const __half*>(k);
+    p.v = static_cast<const __half*>(v);
+    p.slot_mapping = slot_mapping;
+    p.k_codes = k_codes;
+    p.v_codes = v_codes;
+    p.k_scale = static_cast<__half*>(k_scale);
+    p.v_scale = static_cast<__half*>(v_scale);
+    p.k_witness = static_cast<__half*>(k_witness);
+    p.dev_status = dev_status;
+    p.n_tok = n_tok;
+    p.num_kv_heads = desc->num_kv_heads;
+    p.num_pages = desc->num_pages;
+    p.layer = layer;
+    p.rope_layout = desc->rope_layout;
+    p.keys = wc::make_philox_keys(desc->seed);
+    cudaError_t e = wc::launch_write(p, desc->scheme, desc->dither_bits, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "write kernel launch");
+}
+
+size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_pages) {
+    if (check_desc(desc) != WC_OK) return 0;
+    if (batch < 1 || max_pages < 1) {
+        fail(WC_ERR_INVALID_ARG, "batch and max_pages must be positive");
+        return 0;
+    }
+    int sms = 0;
+    if (current_sm_count(&sms) != 0) {
+        fail(WC_ERR_CUDA, "no current CUDA device to size the workspace for");
+        return 0;
+    }
+    return wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms).total;
+}
+
+wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                      const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                      int32_t batch, const void* k_codes, const void* v_codes,
+                                      const void* k_scale, const void* v_scale, const void* k_witness,
+                                      float* out, float* meter, float* meter_raw, void* workspace,
+                                      size_t workspace_bytes, void* stream) {
+    if (wc_status st = check_desc(desc)) return st;
+    if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
+    if (batch < 0 || batch > 65535) return fail(WC_ERR_INVALID_ARG, "batch must be in [0, 65535] (got %d)", batch);
+    if (max_pages < 1) return fail(WC_ERR_INVALID_ARG, "max_pages must be positive (got %d)", max_pages);
+    if ((long long)max_pages * wc::kPage > 0x7FFFFFFFLL) return fail(WC_ERR_UNSUPPORTED, "max_pages too large");
+    if (batch == 0) return WC_OK;
+    if (!q || !block_table || !ctx_lens || !out || !meter || !meter_raw || !workspace)
+        return fail(WC_ERR_INVALID_ARG, "q, block_table, ctx_lens, out, meter, meter_raw, workspace must not be NULL");
+    if (!aligned16(q)) return fail(WC_ERR_INVALID_ARG, "q must be 16-byte aligned");
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0)
+        return fail(WC_ERR_INVALID_ARG, "workspace must be 256-byte aligned");
+    if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
+    int sms = 0;
+    if (current_sm_count(&sms) != 0) return fail(WC_ERR_CUDA, "cannot query the current device");
+    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms);
+    if (workspace_bytes < pl.total)
+        return fail(WC_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, pl.total);
+    uint8_t* ws = static_cast<uint8_t*>(workspace);
+    wc::DecodeParams p;
+    p.q = static_cast<const __half*>(q);
+    p.block_table = block_table;
+    p.ctx_lens = ctx_lens;
+    p.k_codes = static_cast<const uint8_t*>(k_codes);
+    p.v_codes = static_cast<const uint8_t*>(v_codes);
+    p.k_scale = static_cast<const __half*>(k_scale);
+    p.v_scale = static_cast<const __half*>(v_scale);
+    p.k_witness = static_cast<const __half*>(k_witness);
+    p.out = out;
+    p.meter = meter;
+    p.meter_raw = meter_raw;
+    p.status = reinterpret_cast<uint32_t*>(ws);
+    p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
+    p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
+    p.batch = batch;
+    p.max_pages = max_pages;
+    p.num_q_heads = desc->num_q_heads;
+    p.num_kv_heads = desc->num_kv_heads;
+    p.group = desc->num_q_heads / desc->num_kv_heads;
+    p.num_pages = desc->num_pages;
+    p.layer = layer;
+    p.rope_layout = desc->rope_layout;
+    p.splits = pl.splits;
+    p.pages_per_split = pl.pages_per_split;
+    p.keys = wc::make_philox_keys(desc->seed);
+    cudaError_t e = wc::launch_decode(p, desc->scheme, desc->dither_bits, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "decode kernel launch");
+}
+
+wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau, uint8_t* keep_q,
+                  uint8_t* keep_kv, int32_t* n_kept, void* stream) {
+    if (n_cells < 0 || group < 1 || n_cells % group != 0)
+        return fail(WC_ERR_INVALID_ARG, "n_cells (%d) must be a non-negative multiple of group (%d)", n_cells, group);
+    if (!n_kept) return fail(WC_ERR_INVALID_ARG, "n_kept must not be NULL");
+    if (n_cells > 0 && (!meter_raw || !keep_q || !keep_kv))
+        return fail(WC_ERR_INVALID_ARG, "meter_raw, keep_q, keep_kv must not be NULL");
+    cudaError_t e = wc::launch_gate(meter_raw, n_cells, group, tau, keep_q, keep_kv, n_kept,
+                                    static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "gate kernel launch");
+}
+
+wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word, uint32_t* bits, void* stream) {
+    (void)is_status_word;   // the status word sits at offset 0 of a workspace
+    if (!workspace_or_word || !bits) return fail(WC_ERR_INVALID_ARG, "pointers must not be NULL");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    uint32_t host = 0;
+    cudaError_t e = cudaMemcpyAsync(&host, workspace_or_word, sizeof host, cudaMemcpyDeviceToHost, s);
+    if (e == cudaSuccess) e = cudaMemsetAsync(workspace_or_word, 0, sizeof host, s);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device status word");
+    *bits = host;
+    if (host) return fail(WC_ERR_DEVICE_CHECK, "device status bits 0x%x", host);
+    return WC_OK;
+}
+
+}  // extern "C"

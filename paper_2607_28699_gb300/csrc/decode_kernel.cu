@@ -1,0 +1,554 @@
+// Metered decode attention (§6 meter loop, read path; §6.2.1-§6.2.2):
+// dequantize the paged cache, compute the compressed attention output, and in
+// the same pass accumulate the Tier-A e-form meter
+//   c_t = (1/sqrt d) sum_b ||q_b|| w_{t,b}        (Thm. "Sound black-box logit bound")
+//   A   = sum_t p~_t e^{c_t},  meter = min(1, (A^2 - 1)/2)   (Thm. "Sound replacement")
+// merged across context splits under log-sum-exp weights (A is a p~-weighted
+// mean, so it merges exactly like the output; §6.2.2).
+//
+// Grid (splits, Hkv, batch); 4 warps per CTA.  Each warp owns a 4-stage ring
+// of page buffers in shared memory filled by bulk asynchronous copies
+// (cp.async.bulk + mbarrier) that its lane 0 issues ahead of use; a page is
+// 16 tokens of one KV head (2 KiB K codes, 2 KiB V codes, scales, witness).
+//
+// Per page a warp computes, with mma.m16n8k16 (fp16 in, fp32 accumulate):
+//   QK:  D[head][token] = q . code - q . h'   (A = q, B = codes / dither),
+//   PV:  acc[dim][head] += code^T P - h'^T P (A = V codes / dither, B = P),
+// and the bound C[head][token] = a[head][band] . W[token][band] with
+// mma.m16n8k8 (a split into two fp16 terms).  Integer codes and the dither
+// (h' = 4 + j/256 for 8-bit, 1 + j/1024 for 10-bit; xi = h' - kappa) are
+// exact fp16 operands, so code - xi = code - h' + kappa is carried exactly
+// until the fp32 accumulators.
+#include <algorithm>
+#include <climits>
+
+#include "wc_kernels.cuh"
+
+namespace wc {
+
+namespace {
+
+constexpr int kWarps = 4;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kStages = 4;
+constexpr int kStageBytes = 4416;   // K codes | V codes | K scale | V scale | witness
+constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
+constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8 + 16;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;  // log2(e)/sqrt(128)
+
+constexpr uint32_t kSel01 = 0x4140u, kSel23 = 0x4342u;   // [x0,K,x1,K], [x2,K,x3,K]
+
+__device__ __forceinline__ uint32_t sel_interleave(int p) {  // [a_p, b_p, a_p+1, b_p+1]
+    return p == 0 ? 0x5140u : 0x7362u;
+}
+
+template <int kBits>
+struct DitherConst;
+template <>
+struct DitherConst<8> {  // xi = (j + 1/2)/256 - 1/2 = h' - kappa, h' = 4 + j/256
+    static constexpr float kappa = 4.498046875f;
+};
+template <>
+struct DitherConst<10> {  // xi = (j + 1/2)/1024 - 1/2 = h' - kappa, h' = 1 + j/1024
+    static constexpr float kappa = 1.49951171875f;
+};
+
+// h' pair (fp16) for two 8-bit dithers: bytes of x at the selector.
+__device__ __forceinline__ uint32_t h8(uint32_t x, uint32_t sel) { return prmt(x, 0x44444444u, sel); }
+// h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
+__device__ __forceinline__ uint32_t h10(uint32_t x) { return (x & 0x03FF03FFu) | 0x3C003C00u; }
+
+// 2^n for -126 <= n <= 127.
+__device__ __forceinline__ float pow2(int n) { return __int_as_float((127 + n) << 23); }
+
+__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
+    return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+}
+
+template <int kScheme, int kBits>
+__global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecodeParams p) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int g = lane >> 2, c = lane & 3;
+    const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int G = p.group;
+    constexpr bool kInt8 = (kScheme == WC_SCHEME_DITHER_INT8);
+
+    uint8_t* my_stages = smem + warp * kStages * kStageBytes;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageBytes) + warp * kStages;
+    __shared__ int s_is_last;
+
+    int ctx = __ldg(p.ctx_lens + b);
+    if (ctx < 0 || ctx > p.max_pages * kPage) {
+        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+        ctx = max(0, min(ctx, p.max_pages * kPage));
+    }
+    const int npages = (ctx + kPage - 1) / kPage;
+    const int p0 = split * p.pages_per_split;
+    const int p1 = min(p0 + p.pages_per_split, npages);
+    const int n_my = (p1 - p0 - warp > 0) ? (p1 - p0 - warp + kWarps - 1) / kWarps : 0;
+    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+    const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
+
+    // ---- stage issue -----------------------------------------------------
+    if (lane == 0)
+        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
+    fence_barrier_init();
+    __syncwarp();
+
+    auto issue = [&](int k) {
+        if (k >= n_my || lane != 0) return;
+        const int lp = p0 + warp + kWarps * k;
+        const int phys = __ldg(bt_row + lp);
+        uint64_t* bar = &bars[k % kStages];
+        if (phys < 0 || phys >= p.num_pages) {
+            atomicOr(p.status, WC_DEV_BAD_PAGE);
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+            return;
+        }
+        uint8_t* st = my_stages + (k % kStages) * kStageBytes;
+        const size_t ph = (size_t)phys * p.num_kv_heads + h;
+        constexpr uint32_t bytes = kInt8 ? kStageBytes : (2048 + 2048 + 256);
+        mbar_arrive_expect_tx(bar, bytes);
+        bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, bar);
+        bulk_g2s(st + kOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, bar);
+        if constexpr (kInt8) {
+            bulk_g2s(st + kOffKs, p.k_scale + ph * kPage, 32, bar);
+            bulk_g2s(st + kOffVs, p.v_scale + ph * kPage, 32, bar);
+        }
+        bulk_g2s(st + kOffW, p.k_witness + ph * (kPage * kBands), 256, bar);
+    };
+    for (int k = 0; k < kStages; ++k) issue(k);
+
+    // ---- query fragments, band norms --------------------------------------
+    const bool row_valid = g < G;
+    uint32_t qw[16];
+    {
+        const uint4* qsrc = reinterpret_cast<const uint4*>(
+            p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
+            qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+        }
+    }
+    float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {   // word i = channels 32c + 2i, +1
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[i]));
+        qsum += f.x + f.y;
+        part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));   // 8 channels per part
+    }
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+    float band_a, band_b;   // squared norms of bands 2c and 2c+1 of head g
+    if (p.rope_layout == WC_ROPE_HALF) {
+        // lane c holds first (c < 2) or second (c >= 2) halves of bands 4(c&1) + i
+#pragma unroll
+        for (int i = 0; i < 4; ++i) part[i] += __shfl_xor_sync(0xffffffffu, part[i], 2);
+        const int src = (lane & ~3) | (c >> 1);
+        float v[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __shfl_sync(0xffffffffu, part[i], src);
+        band_a = (c & 1) ? v[2] : v[0];
+        band_b = (c & 1) ? v[3] : v[1];
+    } else {
+        band_a = part[0] + part[1];   // dims 32c .. 32c+15 = band 2c
+        band_b = part[2] + part[3];
+    }
+    uint32_t a_hi = 0, a_lo = 0;   // A fragment rows g (rows g+8 are zero)
+    if (row_valid) {
+        const float x0 = sqrtf(band_a) * 0.08838834764831845f, x1 = sqrtf(band_b) * 0.08838834764831845f;
+        const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+        a_hi = pack_h2(__half2float(h0), __half2float(h1));
+        a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
+    }
+    const float zoff = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa * qsum : 0.f;
+
+    // ---- running state -----------------------------------------------------
+    float m_run = -INFINITY;                 // log2-domain running max, head g
+    float l_part = 0.f, d_part = 0.f, spv_part = 0.f;
+    float acc[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+    int lam_exp = kInt8 ? INT_MIN : 14;      // P * s_v * 2^lam_exp < 2^14 (fp16 range)
+    bool failed = false;
+    int consumed = 0;
+
+    for (int k = 0; k < n_my; ++k) {
+        const int lp = p0 + warp + kWarps * k;
+        const int phys = __ldg(bt_row + lp);
+        const bool page_ok = phys >= 0 && phys < p.num_pages;
+        const bool landed = mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
+        if (!__all_sync(0xffffffffu, landed)) {   // warp-uniform decision
+            if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+            failed = true;
+            break;
+        }
+        consumed = k + 1;
+        if (page_ok) {
+            const uint8_t* st = my_stages + (k % kStages) * kStageBytes;
+            const uint32_t slot0 = (uint32_t)phys * kPage;
+            const int nvalid = min(kPage, ctx - lp * kPage);
+
+            // ---------------- QK ------------------------------------------
+            float dc[2][4], dd[2][4];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) dc[nt][e] = dd[nt][e] = 0.f;
+            uint4 kq[2][2];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                const uint4* src = reinterpret_cast<const uint4*>(st + (8 * nt + g) * kHeadDim + 32 * c);
+                kq[nt][0] = src[0];
+                kq[nt][1] = src[1];
+            }
+            constexpr int kGroupsK = (kBits == 10) ? 4 : 2;   // Philox calls per token
+#pragma unroll
+            for (int gp = 0; gp < (kInt8 ? kGroupsK : 1); ++gp) {
+                uint4 dk[2];
+                if constexpr (kInt8) {
+#pragma unroll
+                    for (int nt = 0; nt < 2; ++nt)
+                        dk[nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kGroupsK * c + gp), 0u, p.keys);
+                }
+                constexpr int kStepsPerGroup = kInt8 ? 8 / kGroupsK : 8;
+#pragma unroll
+                for (int kk = 0; kk < kStepsPerGroup; ++kk) {
+                    const int ks = gp * kStepsPerGroup + kk;
+                    const uint32_t A[4] = {qw[2 * ks], 0u, qw[2 * ks + 1], 0u};
+#pragma unroll
+                    for (int nt = 0; nt < 2; ++nt) {
+                        const uint32_t w = word_of(kq[nt][ks >> 2], ks & 3);
+                        if constexpr (kInt8) {
+                            const uint32_t wx = w ^ 0x80808080u;
+                            mma16816(dc[nt], A, s8x2_to_h2(wx, kSel01), s8x2_to_h2(wx, kSel23));
+                            uint32_t h0, h1;
+                            if constexpr (kBits == 8) {
+                                const uint32_t dw = word_of(dk[nt], kk);
+                                h0 = h8(dw, kSel01);
+                                h1 = h8(dw, kSel23);
+                            } else {
+                                h0 = h10(word_of(dk[nt], 2 * kk));
+                                h1 = h10(word_of(dk[nt], 2 * kk + 1));
+                            }
+                            mma16816(dd[nt], A, h0, h1);
+                        } else {
+                            mma16816(dc[nt], A, e4m3x2_to_h2(w), e4m3x2_to_h2(w >> 16));
+                        }
+                    }
+                }
+            }
+
+            // ---------------- logits, bound, softmax ----------------------
+            float y[2][2], cb[2][2], sv[2][2];
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt) {
+                float db[4] = {0.f, 0.f, 0.f, 0.f};
+                const uint32_t wreg = *reinterpret_cast<const uint32_t*>(
+                    st + kOffW + ((8 * nt + g) * kBands + 2 * c) * 2);
+                mma1688(db, a_hi, 0u, wreg);
+                mma1688(db, a_lo, 0u, wreg);
+                float sk0 = 1.f, sk1 = 1.f;
+                if constexpr (kInt8) {
+                    const float2 sk = __half22float2(
+                        *reinterpret_cast<const __half2*>(st + kOffKs + (8 * nt + 2 * c) * 2));
+                    const float2 vv = __half22float2(
+                        *reinterpret_cast<const __half2*>(st + kOffVs + (8 * nt + 2 * c) * 2));
+                    sk0 = sk.x; sk1 = sk.y;
+                    sv[nt][0] = vv.x; sv[nt][1] = vv.y;
+                } else {
+                    sv[nt][0] = sv[nt][1] = 1.f;
+                }
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const int t = 8 * nt + 2 * c + e;
+                    const float raw = kInt8 ? (dc[nt][e] - dd[nt][e] + zoff) : dc[nt][e];
+                    const float yy = raw * (e ? sk1 : sk0) * kRsdLog2e;
+                    const bool ok = t < nvalid;
+                    y[nt][e] = ok ? yy : -INFINITY;
+                    cb[nt][e] = ok ? db[e] : 0.f;   // tail slots may hold any bits
+                    if (!ok) sv[nt][e] = 0.f;
+                }
+            }
+            float mx = fmaxf(fmaxf(y[0][0], y[0][1]), fmaxf(y[1][0], y[1][1]));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
+            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
+            const float m_new = fmaxf(m_run, mx);
+            const bool grow = m_new > m_run;
+            if (__any_sync(0xffffffffu, grow)) {
+                const float alpha = grow ? (m_run == -INFINITY ? 0.f : fast_exp2(m_run - m_new)) : 1.f;
+                l_part *= alpha;
+                d_part *= alpha;
+                spv_part *= alpha;
+                const float a0 = __shfl_sync(0xffffffffu, alpha, 8 * c);      // head 2c
+                const float a1 = __shfl_sync(0xffffffffu, alpha, 8 * c + 4);  // head 2c+1
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    acc[mt][0] *= a0; acc[mt][2] *= a0;
+                    acc[mt][1] *= a1; acc[mt][3] *= a1;
+                }
+                m_run = m_new;
+            }
+            float P[2][2];
+            float smax = 0.f;
+#pragma unroll
+            for (int nt = 0; nt < 2; ++nt)
+#pragma unroll
+                for (int e = 0; e < 2; ++e) {
+                    const float pe = fast_exp2(y[nt][e] - m_run);    // 0 for masked tokens
+                    P[nt][e] = pe;
+                    l_part += pe;
+                    d_part = fmaf(pe, fast_exp2(cb[nt][e] * kLog2e) - 1.f, d_part);
+                    const float pv = pe * sv[nt][e];
+                    spv_part += pv;
+                    P[nt][e] = pv;
+                    smax = fmaxf(smax, sv[nt][e]);
+                }
+            if constexpr (kInt8) {
+                // keep s_v * 2^lam_exp below 2^14 so P s_v 2^lam_exp fits fp16
+                const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
+                if (wmax > 0.f) {
+                    const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
+                    const int want = 14 - e;
+                    if (lam_exp == INT_MIN) {
+                        lam_exp = want;
+                    } else if (want < lam_exp) {
+                        const float f = pow2(want - lam_exp);
+#pragma unroll
+                        for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+                            for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
+                        lam_exp = want;
+                    }
+                }
+            }
+            const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
+            const uint32_t bp0 = pack_h2(P[0][0] * lam, P[0][1] * lam);   // tokens 2c, 2c+1
+            const uint32_t bp1 = pack_h2(P[1][0] * lam, P[1][1] * lam);   // tokens 8+2c, 9+2c
+
+            // ---------------- PV ------------------------------------------
+            const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+            uint4 vq[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                vq[j] = *reinterpret_cast<const uint4*>(st + kOffV + tv[j] * kHeadDim + 16 * g);
+                // an fp8 NaN byte in an unused tail slot would poison P = 0 columns
+                if (!kInt8 && tv[j] >= nvalid) vq[j] = make_uint4(0, 0, 0, 0);
+            }
+            if constexpr (kInt8) {
+                const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
+                constexpr int kHalves = (kBits == 10) ? 2 : 1;
+#pragma unroll
+                for (int hf = 0; hf < kHalves; ++hf) {
+                    uint4 dv[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        dv[j] = philox(slot0 + tv[j], c1,
+                                       (uint32_t)((kBits == 10) ? 2 * g + hf : g), 1u, p.keys);
+#pragma unroll
+                    for (int mm = 0; mm < 8 / kHalves; ++mm) {
+                        const int mt = hf * (8 / kHalves) + mm;
+                        const int wi = mt >> 1, pos = 2 * (mt & 1);
+                        uint32_t A[4];
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
+                                                    word_of(vq[2 * pr + 1], wi) ^ 0x80808080u,
+                                                    sel_interleave(pos));
+                            A[2 * pr] = s8x2_to_h2(X, kSel01);
+                            A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
+                        }
+                        mma16816(acc[mt], A, bp0, bp1);
+                        uint32_t H[4];
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            if constexpr (kBits == 8) {
+                                const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
+                                                        sel_interleave(pos));
+                                H[2 * pr] = h8(Y, kSel01);
+                                H[2 * pr + 1] = h8(Y, kSel23);
+                            } else {
+                                const uint32_t wa = word_of(dv[2 * pr], mt & 3), wb = word_of(dv[2 * pr + 1], mt & 3);
+                                H[2 * pr] = h10(prmt(wa, wb, 0x5410u));
+                                H[2 * pr + 1] = h10(prmt(wa, wb, 0x7632u));
+                            }
+                        }
+                        mma16816(acc[mt], H, bn0, bn1);
+                    }
+                }
+            } else {
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int wi = mt >> 1, pos = 2 * (mt & 1);
+                    uint32_t A[4];
+#pragma unroll
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const uint32_t X = prmt(word_of(vq[2 * pr], wi), word_of(vq[2 * pr + 1], wi),
+                                                sel_interleave(pos));
+                        A[2 * pr] = e4m3x2_to_h2(X);
+                        A[2 * pr + 1] = e4m3x2_to_h2(X >> 16);
+                    }
+                    mma16816(acc[mt], A, bp0, bp1);
+                }
+            }
+        }
+        __syncwarp();
+        issue(k + kStages);
+    }
+    if (failed) {
+        // let copies still in flight land before the CTA's smem is released
+        for (int k = consumed; k < min(n_my, consumed + kStages); ++k)
+            (void)mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
+    }
+
+    // ---- warp partials -> shared, merge the 4 warps ---------------------------
+#pragma unroll
+    for (int o = 1; o < 4; o <<= 1) {
+        l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
+        d_part += __shfl_xor_sync(0xffffffffu, d_part, o);
+        spv_part += __shfl_xor_sync(0xffffffffu, spv_part, o);
+    }
+    const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-14);
+    const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
+    const float spv0 = __shfl_sync(0xffffffffu, spv_part, 8 * c);
+    const float spv1 = __shfl_sync(0xffffffffu, spv_part, 8 * c + 4);
+    __syncthreads();   // stage buffers are reused below
+    float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
+    {
+        float* wb = mbuf + warp * kMaxGroup * kPartialStride;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+            const int d0 = 16 * g + 2 * mt;
+            wb[(2 * c) * kPartialStride + d0] = fmaf(acc[mt][0], inv_lam, kap * spv0);
+            wb[(2 * c + 1) * kPartialStride + d0] = fmaf(acc[mt][1], inv_lam, kap * spv1);
+            wb[(2 * c) * kPartialStride + d0 + 1] = fmaf(acc[mt][2], inv_lam, kap * spv0);
+            wb[(2 * c + 1) * kPartialStride + d0 + 1] = fmaf(acc[mt][3], inv_lam, kap * spv1);
+        }
+        if (c == 0) {
+            wb[g * kPartialStride + kHeadDim + 0] = m_run;
+            wb[g * kPartialStride + kHeadDim + 1] = l_part;
+            wb[g * kPartialStride + kHeadDim + 2] = d_part;
+        }
+    }
+    __syncthreads();
+    const size_t unit = (size_t)b * p.num_kv_heads + h;
+    float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
+    for (int idx = threadIdx.x; idx < G * (kHeadDim + 3); idx += kThreads) {
+        const int hh = idx / (kHeadDim + 3), col = idx % (kHeadDim + 3);
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim]);
+        float v = M;
+        if (col != kHeadDim) {
+            v = 0.f;
+#pragma unroll
+            for (int w = 0; w < kWarps; ++w) {
+                const float* wb = mbuf + (w * kMaxGroup + hh) * kPartialStride;
+                const float sc = (wb[kHeadDim] == -INFINITY) ? 0.f : fast_exp2(wb[kHeadDim] - M);
+                v = fmaf(sc, wb[col], v);
+            }
+        }
+        __stcg(part_out + hh * kPartialStride + col, v);
+    }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned prev = atomicAdd(p.counters + unit, 1u);
+        s_is_last = (prev == (unsigned)(p.splits - 1));
+    }
+    __syncthreads();
+    if (!s_is_last) return;
+    __threadfence();
+
+    // ---- last CTA of this (sequence, KV head): merge all splits -------------
+    float* stat = mbuf;   // [head][M, L, D]
+    const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride);
+    if (threadIdx.x < G) {
+        const int hh = threadIdx.x;
+        float M = -INFINITY;
+        for (int s = 0; s < p.splits; ++s)
+            M = fmaxf(M, __ldcg(base + (s * kMaxGroup + hh) * kPartialStride + kHeadDim));
+        float L = 0.f, Dn = 0.f;
+        if (M != -INFINITY)
+            for (int s = 0; s < p.splits; ++s) {
+                const float* ps = base + (s * kMaxGroup + hh) * kPartialStride;
+                const float ms = __ldcg(ps + kHeadDim);
+                if (ms == -INFINITY) continue;
+                const float sc = fast_exp2(ms - M);
+                L = fmaf(sc, __ldcg(ps + kHeadDim + 1), L);
+                Dn = fmaf(sc, __ldcg(ps + kHeadDim + 2), Dn);
+            }
+        stat[hh * 3 + 0] = M;
+        stat[hh * 3 + 1] = L;
+        stat[hh * 3 + 2] = Dn;
+        const size_t cell = (size_t)b * p.num_q_heads + (size_t)h * G + hh;
+        float raw = 0.f;
+        if (L > 0.f) {
+            const float D = Dn / L;                 // A - 1
+            raw = 0.5f * D * (D + 2.0f);            // (A^2 - 1) / 2, +inf on overflow
+        }
+        p.meter_raw[cell] = raw;
+        p.meter[cell] = fminf(1.0f, raw);
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < G * kHeadDim; idx += kThreads) {
+        const int hh = idx / kHeadDim, d = idx % kHeadDim;
+        const float M = stat[hh * 3], L = stat[hh * 3 + 1];
+        float v = 0.f;
+        if (L > 0.f) {
+            for (int s = 0; s < p.splits; ++s) {
+                const float* ps = base + (s * kMaxGroup + hh) * kPartialStride;
+                const float ms = __ldcg(ps + kHeadDim);
+                if (ms == -INFINITY) continue;
+                v = fmaf(fast_exp2(ms - M), __ldcg(ps + d), v);
+            }
+            v /= L;
+        }
+        p.out[((size_t)b * p.num_q_heads + (size_t)h * G + hh) * kHeadDim + d] = v;
+    }
+    if (threadIdx.x == 0) p.counters[unit] = 0u;   // ready for the next call
+}
+
+}  // namespace
+
+DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms) {
+    DecodePlan pl;
+    const long units = (long)batch * num_kv_heads;
+    const long target = (long)num_sms * 3;   // resident CTAs
+    long pps = (max_pages * units + target - 1) / target;
+    pps = std::max<long>(pps, 8);
+    pps = std::min<long>(pps, std::max(max_pages, 1));
+    pl.pages_per_split = (int)pps;
+    pl.splits = (int)std::max<long>(1, (max_pages + pps - 1) / pps);
+    auto align = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    pl.counters_off = 256;
+    pl.partials_off = align(pl.counters_off + sizeof(uint32_t) * units);
+    pl.total = align(pl.partials_off + sizeof(float) * (size_t)units * pl.splits * kMaxGroup * kPartialStride);
+    return pl;
+}
+
+template <int kScheme, int kBits>
+static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
+    static bool configured = false;   // per process; attribute is per function
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    dim3 grid(p.splits, p.num_kv_heads, p.batch);
+    decode_kernel<kScheme, kBits><<<grid, kThreads, kSmemBytes, stream>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
+    if (p.batch == 0) return cudaSuccess;
+    if (scheme == WC_SCHEME_FP8_E4M3) return launch_one<WC_SCHEME_FP8_E4M3, 8>(p, stream);
+    if (bits == 8) return launch_one<WC_SCHEME_DITHER_INT8, 8>(p, stream);
+    return launch_one<WC_SCHEME_DITHER_INT8, 10>(p, stream);
+}
+
+}  // namespace wc

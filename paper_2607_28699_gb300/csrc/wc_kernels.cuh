@@ -1,0 +1,62 @@
+// Launch parameters and launchers of the WitCert kernels (host + device).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include "wc_common.cuh"
+
+namespace wc {
+
+struct WriteParams {
+    const __half* k;
+    const __half* v;
+    const int32_t* slot_mapping;
+    void* k_codes;
+    void* v_codes;
+    __half* k_scale;
+    __half* v_scale;
+    __half* k_witness;
+    uint32_t* dev_status;
+    int32_t n_tok, num_kv_heads, num_pages, layer, rope_layout;
+    PhiloxKeys keys;
+};
+
+struct DecodeParams {
+    const __half* q;
+    const int32_t* block_table;
+    const int32_t* ctx_lens;
+    const uint8_t* k_codes;
+    const uint8_t* v_codes;
+    const __half* k_scale;
+    const __half* v_scale;
+    const __half* k_witness;
+    float* out;
+    float* meter;
+    float* meter_raw;
+    uint32_t* status;     // workspace word
+    uint32_t* counters;   // [batch * Hkv], zero between calls
+    float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
+    int32_t batch, max_pages, num_q_heads, num_kv_heads, group, num_pages, layer, rope_layout;
+    int32_t splits, pages_per_split;
+    PhiloxKeys keys;
+};
+
+// Per (query head, split) partial: acc[128] | m | l | D | pad.
+constexpr int kPartialStride = kHeadDim + 4;
+
+// Workspace layout (bytes): [0, 256) status word, then counters, then
+// partials, each 256-byte aligned.
+struct DecodePlan {
+    int splits;
+    int pages_per_split;
+    size_t counters_off, partials_off, total;
+};
+
+DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms);
+
+cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
+cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
+cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float tau, uint8_t* keep_q,
+                        uint8_t* keep_kv, int32_t* n_kept, cudaStream_t stream);
+
+}  // namespace wc

@@ -1,0 +1,66 @@
+"""Shared helpers for the GPU parity tests: run the oracle and the CUDA path
+on the same seeded inputs and compare."""
+
+import numpy as np
+import torch
+
+import workloads as W
+from oracle import pipeline as OP
+
+RTOL, ATOL = 1e-3, 1e-5     # fp32 outputs, meters, band norms
+
+
+def close(gpu, ref, rtol=RTOL, atol=ATOL):
+    gpu = np.asarray(gpu, dtype=np.float64)
+    ref = np.asarray(ref, dtype=np.float64)
+    both_inf = np.isinf(gpu) & np.isinf(ref) & (np.sign(gpu) == np.sign(ref))
+    ok = both_inf | (np.abs(gpu - ref) <= atol + rtol * np.abs(ref))
+    return ok
+
+
+def assert_close(gpu, ref, what, rtol=RTOL, atol=ATOL):
+    ok = close(gpu, ref, rtol, atol)
+    if not np.all(ok):
+        g, r = np.asarray(gpu, np.float64), np.asarray(ref, np.float64)
+        idx = np.argwhere(~ok)[:5]
+        raise AssertionError(f"{what}: {int((~ok).sum())}/{ok.size} outside tol; first {idx.tolist()} "
+                             f"gpu={g[tuple(idx.T)]} ref={r[tuple(idx.T)]}")
+
+
+def descs(n_q, n_kv, num_pages, scheme=0, bits=8, layout=0, seed=0):
+    import paper_2607_28699_gb300 as wc
+    o = OP.Desc(num_q_heads=n_q, num_kv_heads=n_kv, num_pages=num_pages, scheme=scheme,
+                dither_bits=bits, rope_layout=layout, seed=seed)
+    g = wc.CacheDesc(num_q_heads=n_q, num_kv_heads=n_kv, num_pages=num_pages, scheme=scheme,
+                     dither_bits=bits, rope_layout=layout, seed=seed)
+    return o, g
+
+
+def gpu_cache_to_numpy(cache):
+    out = {"k_codes": cache.k_codes.cpu().numpy(), "v_codes": cache.v_codes.cpu().numpy(),
+           "k_witness": cache.k_witness.cpu().numpy()}
+    if cache.k_scale is not None:
+        out["k_scale"] = cache.k_scale.cpu().numpy()
+        out["v_scale"] = cache.v_scale.cpu().numpy()
+    return out
+
+
+def numpy_cache_to_gpu(cache, desc_g):
+    import paper_2607_28699_gb300 as wc
+    c = wc.LayerCache.empty(desc_g)
+    c.k_codes.copy_(torch.from_numpy(cache["k_codes"]))
+    c.v_codes.copy_(torch.from_numpy(cache["v_codes"]))
+    c.k_witness.copy_(torch.from_numpy(cache["k_witness"]))
+    if "k_scale" in cache:
+        c.k_scale.copy_(torch.from_numpy(cache["k_scale"]))
+        c.v_scale.copy_(torch.from_numpy(cache["v_scale"]))
+    return c
+
+
+def make_inputs(wl, layer=0):
+    """CPU-drawn inputs (identical for both sides)."""
+    bt = W.block_tables(wl)
+    sm = W.slot_mapping(wl, bt)
+    k, v = W.layer_kv(wl, layer)
+    q = W.layer_queries(wl, layer)
+    return bt, sm, k, v, q

@@ -1,0 +1,147 @@
+"""GPU parity of metered decode attention (wc_metered_decode_attention)
+against the oracle: outputs, meters and raw meters within 1e-3 relative /
+1e-5 absolute; the meter bounds the true TV; device status checks."""
+
+import numpy as np
+import pytest
+import torch
+
+import workloads as W
+from oracle import pipeline as OP
+from tests._parity import assert_close, descs, make_inputs, numpy_cache_to_gpu
+
+pytestmark = pytest.mark.gpu
+
+
+def _oracle_decode(od, layer, q, bt, ctx_lens, ocache, k=None, v=None, seq_offsets=None):
+    outs, meters, raws, tvs = [], [], [], []
+    for b, S in enumerate(ctx_lens):
+        ke = ve = None
+        if k is not None:
+            o = seq_offsets[b]
+            ke, ve = k[o:o + S], v[o:o + S]
+        r = OP.decode_sequence(od, layer, q[b], bt[b], S, ocache, ke, ve)
+        outs.append(r["out"]); meters.append(r["meter"]); raws.append(r["meter_raw"]); tvs.append(r["tv"])
+    return np.stack(outs), np.stack(meters), np.stack(raws), np.stack(tvs)
+
+
+def _run(wl, scheme=0, bits=8, layout=0, layer=0, seed=1, gpu_writes=True):
+    import paper_2607_28699_gb300 as wc
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    od, gd = descs(wl.n_q_heads, wl.n_kv_heads, wl.num_pages, scheme, bits, layout, seed)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
+    if gpu_writes:
+        gcache = wc.LayerCache.empty(gd)
+        wc.kv_quantize_witness(gd, layer, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), gcache)
+    else:
+        gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    out, meter, raw = wc.metered_decode_attention(gd, layer, q.cuda(), torch.from_numpy(bt).cuda(), ctx,
+                                                  gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    offs = np.concatenate([[0], np.cumsum(wl.ctx_lens)[:-1]])
+    o_out, o_meter, o_raw, o_tv = _oracle_decode(od, layer, q.numpy(), bt, wl.ctx_lens, ocache,
+                                                 k.numpy(), v.numpy(), offs)
+    return (out.cpu().numpy(), meter.cpu().numpy(), raw.cpu().numpy()), (o_out, o_meter, o_raw, o_tv)
+
+
+def _compare(g, o):
+    assert_close(g[0], o[0], "out")
+    assert_close(g[1], o[1], "meter")
+    assert_close(g[2], o[2], "meter_raw")
+    assert np.all(g[2] >= o[3] * (1 - 1e-3)), "GPU meter below the true TV"
+
+
+@pytest.mark.parametrize("scheme,bits,layout", [(0, 8, 0), (0, 10, 0), (0, 8, 1), (1, 8, 0)])
+@pytest.mark.parametrize("gpu_writes", [False, True])
+def test_decode_matches_oracle_config1_shape(scheme, bits, layout, gpu_writes):
+    wl = W.config(1, ctx_scale=0.5)               # S = 2048 + ragged? (2048) -> also test ragged below
+    g, o = _run(wl, scheme, bits, layout, gpu_writes=gpu_writes)
+    _compare(g, o)
+
+
+@pytest.mark.parametrize("ctx", [1, 15, 16, 17, 127, 128, 129, 1000, 3001])
+def test_decode_ragged_contexts(ctx):
+    wl = W.Workload("r", 1, 8, 2, [ctx], seed=4)
+    g, o = _run(wl)
+    _compare(g, o)
+
+
+def test_decode_batch_mixed_shuffled_gqa7():
+    wl = W.Workload("m", 1, 28, 4, [4100, 77, 1, 2500, 16, 999], shuffle_pages=True, seed=6)
+    for scheme in (0, 1):
+        g, o = _run(wl, scheme=scheme, layer=3)
+        _compare(g, o)
+
+
+def test_decode_many_splits_long_context():
+    wl = W.Workload("long", 1, 28, 4, [20011], seed=8)
+    g, o = _run(wl, bits=10, layer=5)
+    _compare(g, o)
+
+
+def test_decode_zero_context_and_repeat_calls():
+    """ctx 0 gives out = 0 and meter 0; the workspace is reusable call after call."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("z", 1, 8, 2, [300, 40], seed=2)
+    bt, sm, k, v, q = make_inputs(wl)
+    od, gd = descs(8, 2, wl.num_pages)
+    cache = wc.LayerCache.empty(gd)
+    wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
+    ws = wc.Workspace(gd, 2, wl.max_pages)
+    btg = torch.from_numpy(bt).cuda()
+    first = None
+    for it in range(3):
+        ctx = torch.tensor([300, 0] if it == 1 else [300, 40], dtype=torch.int32, device="cuda")
+        out, meter, raw = wc.metered_decode_attention(gd, 0, q.cuda(), btg, ctx, cache, ws)
+        torch.cuda.synchronize()
+        if it == 1:
+            assert torch.all(out[1] == 0) and torch.all(meter[1] == 0) and torch.all(raw[1] == 0)
+        elif first is None:
+            first = (out.clone(), raw.clone())
+        else:
+            assert torch.equal(out, first[0]) and torch.equal(raw, first[1])   # deterministic
+    assert wc.read_status(ws) == 0
+
+
+def test_decode_bad_page_and_bad_ctx_set_status():
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("b", 1, 8, 2, [64], seed=2)
+    bt, sm, k, v, q = make_inputs(wl)
+    od, gd = descs(8, 2, wl.num_pages)
+    cache = wc.LayerCache.empty(gd)
+    wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
+    ws = wc.Workspace(gd, 1, wl.max_pages)
+    bt_bad = torch.from_numpy(bt).cuda().clone()
+    bt_bad[0, 1] = 10_000
+    ctx = torch.tensor([64], dtype=torch.int32, device="cuda")
+    wc.metered_decode_attention(gd, 0, q.cuda(), bt_bad, ctx, cache, ws)
+    assert wc.read_status(ws) & wc.DEV_BAD_PAGE
+    ctx_bad = torch.tensor([65], dtype=torch.int32, device="cuda")    # > max_pages * 16
+    wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx_bad, cache, ws)
+    assert wc.read_status(ws) & wc.DEV_BAD_CTX
+
+
+def test_decode_host_validation():
+    import paper_2607_28699_gb300 as wc
+    _, gd = descs(8, 2, 4)
+    cache = wc.LayerCache.empty(gd)
+    q = torch.zeros(1, 8, 128, dtype=torch.float16, device="cuda")
+    bt = torch.zeros(1, 4, dtype=torch.int32, device="cuda")
+    ctx = torch.ones(1, dtype=torch.int32, device="cuda")
+    ws = wc.Workspace(gd, 1, 4)
+    small = wc.Workspace(gd, 1, 4)
+    small.nbytes = 256
+    with pytest.raises(wc.WitCertError) as e:
+        wc.metered_decode_attention(gd, 0, q, bt, ctx, cache, small)
+    assert e.value.status == 4
+    bad = wc.CacheDesc(num_q_heads=12, num_kv_heads=8, num_pages=4)
+    with pytest.raises(wc.WitCertError):
+        wc.metered_decode_attention(bad, 0, q, bt, ctx, cache, ws)
+    wide = wc.CacheDesc(num_q_heads=36, num_kv_heads=2, num_pages=4)   # G = 18 > 8
+    with pytest.raises(wc.WitCertError) as e:
+        wc.metered_decode_attention(wide, 0, q, bt, ctx, cache, ws)
+    assert e.value.status == 2
