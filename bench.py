@@ -168,8 +168,8 @@ class Setup:
         self.keep_q = torch.empty(L * B * Hq, dtype=torch.uint8, device="cuda")
         self.keep_kv = torch.empty(L * B * Hq // wl.group, dtype=torch.uint8, device="cuda")
         self.n_kept = torch.empty(2, dtype=torch.int32, device="cuda")
-        self.ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                   for _ in range(L)]
+        # events recorded inside the captured graph must be "external" records
+        self.ev = [(_graph_event(), _graph_event()) for _ in range(L)]
         self.tau = wl.taus[0]
 
     def step(self, timed_events=True):
@@ -191,6 +191,13 @@ class Setup:
 
     def decode_bytes_per_launch(self):
         return sum(self.wl.ctx_lens) * self.wl.n_kv_heads * BYTES_PER_TOKEN_HEAD[self.wl.scheme]
+
+
+def _graph_event():
+    try:
+        return torch.cuda.Event(enable_timing=True, external=True)
+    except TypeError:
+        return torch.cuda.Event(enable_timing=True)
 
 
 def capture(fn, stream):

@@ -326,8 +326,19 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                 }
             }
             const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
-            const uint32_t bp0 = pack_h2(P[0][0] * lam, P[0][1] * lam);   // tokens 2c, 2c+1
-            const uint32_t bp1 = pack_h2(P[1][0] * lam, P[1][1] * lam);   // tokens 8+2c, 9+2c
+            // B = P^T as a sum of two fp16 terms (hi + lo): the output is a
+            // sum with heavy cancellation, so one fp16 rounding of P is not
+            // accurate enough.  Tokens 2c, 2c+1 (bp*0) and 8+2c, 9+2c (bp*1).
+            uint32_t bp0, bp1, bl0, bl1;
+            {
+                const float x00 = P[0][0] * lam, x01 = P[0][1] * lam, x10 = P[1][0] * lam, x11 = P[1][1] * lam;
+                bp0 = pack_h2(x00, x01);
+                bp1 = pack_h2(x10, x11);
+                const float2 r0 = __half22float2(*reinterpret_cast<const __half2*>(&bp0));
+                const float2 r1 = __half22float2(*reinterpret_cast<const __half2*>(&bp1));
+                bl0 = pack_h2(x00 - r0.x, x01 - r0.y);
+                bl1 = pack_h2(x10 - r1.x, x11 - r1.y);
+            }
 
             // ---------------- PV ------------------------------------------
             const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
@@ -340,6 +351,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
             }
             if constexpr (kInt8) {
                 const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
+                const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
                 constexpr int kHalves = (kBits == 10) ? 2 : 1;
 #pragma unroll
                 for (int hf = 0; hf < kHalves; ++hf) {
@@ -362,6 +374,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                             A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
                         }
                         mma16816(acc[mt], A, bp0, bp1);
+                        mma16816(acc[mt], A, bl0, bl1);
                         uint32_t H[4];
 #pragma unroll
                         for (int pr = 0; pr < 2; ++pr) {
@@ -377,6 +390,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                             }
                         }
                         mma16816(acc[mt], H, bn0, bn1);
+                        mma16816(acc[mt], H, bm0, bm1);
                     }
                 }
             } else {
@@ -392,6 +406,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                         A[2 * pr + 1] = e4m3x2_to_h2(X >> 16);
                     }
                     mma16816(acc[mt], A, bp0, bp1);
+                    mma16816(acc[mt], A, bl0, bl1);
                 }
             }
         }
