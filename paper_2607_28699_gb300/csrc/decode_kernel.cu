@@ -28,9 +28,10 @@ namespace wc {
 
 namespace {
 
-constexpr int kWarps = 4;
+constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
-constexpr int kStages = 4;
+constexpr int kStages = 3;
+constexpr int kMinBlocks = 2;            // two CTAs (16 warps) per SM
 constexpr int kStageBytes = 4416;   // K codes | V codes | K scale | V scale | witness
 constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
 constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8 + 16;
@@ -54,6 +55,12 @@ struct DitherConst<10> {  // xi = (j + 1/2)/1024 - 1/2 = h' - kappa, h' = 1 + j/
     static constexpr float kappa = 1.49951171875f;
 };
 
+// Two int8 codes as the fp16 pair 1152 + code (exact): (code ^ 0x80) in the
+// low mantissa byte of 1024.0.  The constant 1152 is removed once per logit.
+__device__ __forceinline__ uint32_t s8x2_biased(uint32_t w_xor80, uint32_t sel) {
+    return prmt(w_xor80, 0x64646464u, sel);
+}
+
 // h' pair (fp16) for two 8-bit dithers: bytes of x at the selector.
 __device__ __forceinline__ uint32_t h8(uint32_t x, uint32_t sel) { return prmt(x, 0x44444444u, sel); }
 // h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
@@ -67,7 +74,7 @@ __device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
 }
 
 template <int kScheme, int kBits>
-__global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_constant__ DecodeParams p) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecodeParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
@@ -77,7 +84,6 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
 
     uint8_t* my_stages = smem + warp * kStages * kStageBytes;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageBytes) + warp * kStages;
-    __shared__ int s_is_last;
 
     int ctx = __ldg(p.ctx_lens + b);
     if (ctx < 0 || ctx > p.max_pages * kPage) {
@@ -91,7 +97,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
     const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
     const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
 
-    // ---- stage issue -----------------------------------------------------
+    // ---- per-warp stage ring -------------------------------------------------
     if (lane == 0)
         for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
     fence_barrier_init();
@@ -99,8 +105,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
 
     auto issue = [&](int k) {
         if (k >= n_my || lane != 0) return;
-        const int lp = p0 + warp + kWarps * k;
-        const int phys = __ldg(bt_row + lp);
+        const int phys = __ldg(bt_row + p0 + warp + kWarps * k);
         uint64_t* bar = &bars[k % kStages];
         if (phys < 0 || phys >= p.num_pages) {
             atomicOr(p.status, WC_DEV_BAD_PAGE);
@@ -121,9 +126,9 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
     };
     for (int k = 0; k < kStages; ++k) issue(k);
 
-    // ---- query fragments, band norms --------------------------------------
+    // ---- query fragments, band norms ------------------------------------------
     const bool row_valid = g < G;
-    uint32_t qw[16];
+    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
     {
         const uint4* qsrc = reinterpret_cast<const uint4*>(
             p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
@@ -135,16 +140,16 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
     }
     float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {   // word i = channels 32c + 2i, +1
+    for (int i = 0; i < 16; ++i) {
         const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[i]));
         qsum += f.x + f.y;
-        part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));   // 8 channels per part
+        part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));   // channels 32c + 8(i>>2) .. +7
     }
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
     float band_a, band_b;   // squared norms of bands 2c and 2c+1 of head g
     if (p.rope_layout == WC_ROPE_HALF) {
-        // lane c holds first (c < 2) or second (c >= 2) halves of bands 4(c&1) + i
+        // lane c holds the first (c < 2) or second (c >= 2) halves of bands 4(c&1) + i
 #pragma unroll
         for (int i = 0; i < 4; ++i) part[i] += __shfl_xor_sync(0xffffffffu, part[i], 2);
         const int src = (lane & ~3) | (c >> 1);
@@ -157,28 +162,34 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
         band_a = part[0] + part[1];   // dims 32c .. 32c+15 = band 2c
         band_b = part[2] + part[3];
     }
-    uint32_t a_hi = 0, a_lo = 0;   // A fragment rows g (rows g+8 are zero)
+    uint32_t a_hi = 0, a_lo = 0;   // bound A fragment, rows g (rows g+8 are zero)
     if (row_valid) {
         const float x0 = sqrtf(band_a) * 0.08838834764831845f, x1 = sqrtf(band_b) * 0.08838834764831845f;
         const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
         a_hi = pack_h2(__half2float(h0), __half2float(h1));
         a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
     }
-    const float zoff = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa * qsum : 0.f;
+    // q . (code - xi) = q . (code + 1152) - q . h' + (kappa - 1152) sum(q)
+    const float zoff = kInt8 ? (DitherConst<kBits == 10 ? 10 : 8>::kappa - 1152.0f) * qsum : 0.f;
 
-    // ---- running state -----------------------------------------------------
-    float m_run = -INFINITY;                 // log2-domain running max, head g
+    // ---- running state -----------------------------------------------------------
+    // Log2-domain softmax reference m_run, moved lazily: only when a page's max
+    // exceeds it by more than 8 (P may reach 2^8 in between).
+    float m_run = -INFINITY;
     float l_part = 0.f, d_part = 0.f, spv_part = 0.f;
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-    int lam_exp = kInt8 ? INT_MIN : 14;      // P * s_v * 2^lam_exp < 2^14 (fp16 range)
+    // P * s_v * 2^lam_exp stays below 2^14 (fp16): s_v * 2^lam_exp < 2^6.
+    int lam_exp = kInt8 ? INT_MIN : 6;
     bool failed = false;
     int consumed = 0;
+    int phys_next = n_my > 0 ? __ldg(bt_row + p0 + warp) : 0;
 
     for (int k = 0; k < n_my; ++k) {
         const int lp = p0 + warp + kWarps * k;
-        const int phys = __ldg(bt_row + lp);
+        const int phys = phys_next;
+        if (k + 1 < n_my) phys_next = __ldg(bt_row + lp + kWarps);
         const bool page_ok = phys >= 0 && phys < p.num_pages;
         const bool landed = mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
         if (!__all_sync(0xffffffffu, landed)) {   // warp-uniform decision
@@ -192,39 +203,50 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
             const uint32_t slot0 = (uint32_t)phys * kPage;
             const int nvalid = min(kPage, ctx - lp * kPage);
 
-            // ---------------- QK ------------------------------------------
+            // ---------------- QK: D[head][token] ------------------------------
             float dc[2][4], dd[2][4];
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) dc[nt][e] = dd[nt][e] = 0.f;
-            uint4 kq[2][2];
+            // codes first, then the dither: their operands are never live together
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
-                const uint4* src = reinterpret_cast<const uint4*>(st + (8 * nt + g) * kHeadDim + 32 * c);
-                kq[nt][0] = src[0];
-                kq[nt][1] = src[1];
-            }
-            constexpr int kGroupsK = (kBits == 10) ? 4 : 2;   // Philox calls per token
+            for (int gp = 0; gp < 2; ++gp) {                 // channels 32c + 16gp .. +15
+                uint4 kq[2];
 #pragma unroll
-            for (int gp = 0; gp < (kInt8 ? kGroupsK : 1); ++gp) {
-                uint4 dk[2];
-                if constexpr (kInt8) {
+                for (int nt = 0; nt < 2; ++nt)
+                    kq[nt] = *reinterpret_cast<const uint4*>(st + (8 * nt + g) * kHeadDim + 32 * c + 16 * gp);
 #pragma unroll
-                    for (int nt = 0; nt < 2; ++nt)
-                        dk[nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kGroupsK * c + gp), 0u, p.keys);
-                }
-                constexpr int kStepsPerGroup = kInt8 ? 8 / kGroupsK : 8;
-#pragma unroll
-                for (int kk = 0; kk < kStepsPerGroup; ++kk) {
-                    const int ks = gp * kStepsPerGroup + kk;
+                for (int kk = 0; kk < 4; ++kk) {
+                    const int ks = 4 * gp + kk;              // channels 32c + 4ks .. +3
                     const uint32_t A[4] = {qw[2 * ks], 0u, qw[2 * ks + 1], 0u};
 #pragma unroll
                     for (int nt = 0; nt < 2; ++nt) {
-                        const uint32_t w = word_of(kq[nt][ks >> 2], ks & 3);
+                        const uint32_t w = word_of(kq[nt], kk);
                         if constexpr (kInt8) {
                             const uint32_t wx = w ^ 0x80808080u;
-                            mma16816(dc[nt], A, s8x2_to_h2(wx, kSel01), s8x2_to_h2(wx, kSel23));
+                            mma16816(dc[nt], A, s8x2_biased(wx, kSel01), s8x2_biased(wx, kSel23));
+                        } else {
+                            mma16816(dc[nt], A, e4m3x2_to_h2(w), e4m3x2_to_h2(w >> 16));
+                        }
+                    }
+                }
+            }
+            if constexpr (kInt8) {
+                constexpr int kCalls = (kBits == 10) ? 4 : 2;     // Philox calls per token
+#pragma unroll
+                for (int gi = 0; gi < kCalls; ++gi) {
+                    uint4 dk[2];
+#pragma unroll
+                    for (int nt = 0; nt < 2; ++nt)
+                        dk[nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kCalls * c + gi), 0u, p.keys);
+                    constexpr int kSteps = 8 / kCalls;            // k-steps covered by one call
+#pragma unroll
+                    for (int kk = 0; kk < kSteps; ++kk) {
+                        const int ks = kSteps * gi + kk;
+                        const uint32_t A[4] = {qw[2 * ks], 0u, qw[2 * ks + 1], 0u};
+#pragma unroll
+                        for (int nt = 0; nt < 2; ++nt) {
                             uint32_t h0, h1;
                             if constexpr (kBits == 8) {
                                 const uint32_t dw = word_of(dk[nt], kk);
@@ -235,14 +257,12 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                                 h1 = h10(word_of(dk[nt], 2 * kk + 1));
                             }
                             mma16816(dd[nt], A, h0, h1);
-                        } else {
-                            mma16816(dc[nt], A, e4m3x2_to_h2(w), e4m3x2_to_h2(w >> 16));
                         }
                     }
                 }
             }
 
-            // ---------------- logits, bound, softmax ----------------------
+            // ---------------- logits, bound, softmax --------------------------
             float y[2][2], cb[2][2], sv[2][2];
 #pragma unroll
             for (int nt = 0; nt < 2; ++nt) {
@@ -266,9 +286,8 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                 for (int e = 0; e < 2; ++e) {
                     const int t = 8 * nt + 2 * c + e;
                     const float raw = kInt8 ? (dc[nt][e] - dd[nt][e] + zoff) : dc[nt][e];
-                    const float yy = raw * (e ? sk1 : sk0) * kRsdLog2e;
                     const bool ok = t < nvalid;
-                    y[nt][e] = ok ? yy : -INFINITY;
+                    y[nt][e] = ok ? raw * ((e ? sk1 : sk0) * kRsdLog2e) : -INFINITY;
                     cb[nt][e] = ok ? db[e] : 0.f;   // tail slots may hold any bits
                     if (!ok) sv[nt][e] = 0.f;
                 }
@@ -276,10 +295,10 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
             float mx = fmaxf(fmaxf(y[0][0], y[0][1]), fmaxf(y[1][0], y[1][1]));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
             mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            const float m_new = fmaxf(m_run, mx);
-            const bool grow = m_new > m_run;
-            if (__any_sync(0xffffffffu, grow)) {
-                const float alpha = grow ? (m_run == -INFINITY ? 0.f : fast_exp2(m_run - m_new)) : 1.f;
+            const bool move = mx > m_run + 8.0f;
+            if (__any_sync(0xffffffffu, move)) {
+                const float alpha = move ? (m_run == -INFINITY ? 0.f : fast_exp2(m_run - mx)) : 1.f;
+                if (move) m_run = mx;
                 l_part *= alpha;
                 d_part *= alpha;
                 spv_part *= alpha;
@@ -290,7 +309,6 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
                     acc[mt][1] *= a1; acc[mt][3] *= a1;
                 }
-                m_run = m_new;
             }
             float P[2][2];
             float smax = 0.f;
@@ -299,7 +317,6 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
 #pragma unroll
                 for (int e = 0; e < 2; ++e) {
                     const float pe = fast_exp2(y[nt][e] - m_run);    // 0 for masked tokens
-                    P[nt][e] = pe;
                     l_part += pe;
                     d_part = fmaf(pe, fast_exp2(cb[nt][e] * kLog2e) - 1.f, d_part);
                     const float pv = pe * sv[nt][e];
@@ -308,11 +325,10 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                     smax = fmaxf(smax, sv[nt][e]);
                 }
             if constexpr (kInt8) {
-                // keep s_v * 2^lam_exp below 2^14 so P s_v 2^lam_exp fits fp16
                 const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
                 if (wmax > 0.f) {
                     const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
-                    const int want = 14 - e;
+                    const int want = 6 - e;
                     if (lam_exp == INT_MIN) {
                         lam_exp = want;
                     } else if (want < lam_exp) {
@@ -328,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
             const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
             // B = P^T as a sum of two fp16 terms (hi + lo): the output is a
             // sum with heavy cancellation, so one fp16 rounding of P is not
-            // accurate enough.  Tokens 2c, 2c+1 (bp*0) and 8+2c, 9+2c (bp*1).
+            // accurate enough.  Tokens 2c, 2c+1 (b*0) and 8+2c, 9+2c (b*1).
             uint32_t bp0, bp1, bl0, bl1;
             {
                 const float x00 = P[0][0] * lam, x01 = P[0][1] * lam, x10 = P[1][0] * lam, x11 = P[1][1] * lam;
@@ -340,7 +356,7 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                 bl1 = pack_h2(x10 - r1.x, x11 - r1.y);
             }
 
-            // ---------------- PV ------------------------------------------
+            // ---------------- PV: acc[dim][head] ------------------------------
             const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
             uint4 vq[4];
 #pragma unroll
@@ -350,6 +366,20 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                 if (!kInt8 && tv[j] >= nvalid) vq[j] = make_uint4(0, 0, 0, 0);
             }
             if constexpr (kInt8) {
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int wi = mt >> 1, pos = 2 * (mt & 1);
+                    uint32_t A[4];
+#pragma unroll
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
+                                                word_of(vq[2 * pr + 1], wi) ^ 0x80808080u, sel_interleave(pos));
+                        A[2 * pr] = s8x2_to_h2(X, kSel01);
+                        A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
+                    }
+                    mma16816(acc[mt], A, bp0, bp1);
+                    mma16816(acc[mt], A, bl0, bl1);
+                }
                 const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
                 const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
                 constexpr int kHalves = (kBits == 10) ? 2 : 1;
@@ -358,23 +388,11 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                     uint4 dv[4];
 #pragma unroll
                     for (int j = 0; j < 4; ++j)
-                        dv[j] = philox(slot0 + tv[j], c1,
-                                       (uint32_t)((kBits == 10) ? 2 * g + hf : g), 1u, p.keys);
+                        dv[j] = philox(slot0 + tv[j], c1, (uint32_t)((kBits == 10) ? 2 * g + hf : g), 1u, p.keys);
 #pragma unroll
                     for (int mm = 0; mm < 8 / kHalves; ++mm) {
                         const int mt = hf * (8 / kHalves) + mm;
                         const int wi = mt >> 1, pos = 2 * (mt & 1);
-                        uint32_t A[4];
-#pragma unroll
-                        for (int pr = 0; pr < 2; ++pr) {
-                            const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
-                                                    word_of(vq[2 * pr + 1], wi) ^ 0x80808080u,
-                                                    sel_interleave(pos));
-                            A[2 * pr] = s8x2_to_h2(X, kSel01);
-                            A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
-                        }
-                        mma16816(acc[mt], A, bp0, bp1);
-                        mma16816(acc[mt], A, bl0, bl1);
                         uint32_t H[4];
 #pragma unroll
                         for (int pr = 0; pr < 2; ++pr) {
@@ -419,14 +437,14 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
             (void)mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
     }
 
-    // ---- warp partials -> shared, merge the 4 warps ---------------------------
+    // ---- warp partials -> shared, merge the warps of this CTA ----------------------
 #pragma unroll
     for (int o = 1; o < 4; o <<= 1) {
         l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
         d_part += __shfl_xor_sync(0xffffffffu, d_part, o);
         spv_part += __shfl_xor_sync(0xffffffffu, spv_part, o);
     }
-    const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-14);
+    const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
     const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
     const float spv0 = __shfl_sync(0xffffffffu, spv_part, 8 * c);
     const float spv1 = __shfl_sync(0xffffffffu, spv_part, 8 * c + 4);
@@ -466,65 +484,79 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
                 v = fmaf(sc, wb[col], v);
             }
         }
-        __stcg(part_out + hh * kPartialStride + col, v);
+        part_out[hh * kPartialStride + col] = v;
     }
-    __threadfence();
+    // the merge kernel (launched as a programmatic dependent) may start now;
+    // it waits for this whole grid before reading the partials
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
+// Merge of the per-split partials of one (sequence, query head), 32 output
+// dims per CTA: out = sum_s w_s acc_s / sum_s w_s l_s with w_s = 2^(m_s - M),
+// D = sum_s w_s D_s / sum_s w_s l_s, meter_raw = D (D + 2) / 2 (§6.2.2: the
+// meter accumulator merges under the same LSE weights as the output).
+constexpr int kMergeWarps = 8;
+
+__global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_constant__ DecodeParams p) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int chunk = blockIdx.x, hq = blockIdx.y, b = blockIdx.z;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int h = hq / p.group, hh = hq % p.group;
+    const size_t unit = (size_t)b * p.num_kv_heads + h;
+    const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride) + hh * kPartialStride;
+    const size_t split_stride = kMaxGroup * kPartialStride;
+    __shared__ float red[kMergeWarps][36];
+    __shared__ float sM;
+
+    float M = -INFINITY;
+    for (int s = warp; s < p.splits; s += kMergeWarps) M = fmaxf(M, __ldcg(base + s * split_stride + kHeadDim));
+    if (lane == 0) red[warp][0] = M;
     __syncthreads();
     if (threadIdx.x == 0) {
-        const unsigned prev = atomicAdd(p.counters + unit, 1u);
-        s_is_last = (prev == (unsigned)(p.splits - 1));
+        float m = -INFINITY;
+        for (int w = 0; w < kMergeWarps; ++w) m = fmaxf(m, red[w][0]);
+        sM = m;
     }
     __syncthreads();
-    if (!s_is_last) return;
-    __threadfence();
-
-    // ---- last CTA of this (sequence, KV head): merge all splits -------------
-    float* stat = mbuf;   // [head][M, L, D]
-    const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride);
-    if (threadIdx.x < G) {
-        const int hh = threadIdx.x;
-        float M = -INFINITY;
-        for (int s = 0; s < p.splits; ++s)
-            M = fmaxf(M, __ldcg(base + (s * kMaxGroup + hh) * kPartialStride + kHeadDim));
-        float L = 0.f, Dn = 0.f;
-        if (M != -INFINITY)
-            for (int s = 0; s < p.splits; ++s) {
-                const float* ps = base + (s * kMaxGroup + hh) * kPartialStride;
-                const float ms = __ldcg(ps + kHeadDim);
-                if (ms == -INFINITY) continue;
-                const float sc = fast_exp2(ms - M);
-                L = fmaf(sc, __ldcg(ps + kHeadDim + 1), L);
-                Dn = fmaf(sc, __ldcg(ps + kHeadDim + 2), Dn);
-            }
-        stat[hh * 3 + 0] = M;
-        stat[hh * 3 + 1] = L;
-        stat[hh * 3 + 2] = Dn;
-        const size_t cell = (size_t)b * p.num_q_heads + (size_t)h * G + hh;
-        float raw = 0.f;
-        if (L > 0.f) {
-            const float D = Dn / L;                 // A - 1
-            raw = 0.5f * D * (D + 2.0f);            // (A^2 - 1) / 2, +inf on overflow
+    M = sM;
+    float acc = 0.f, L = 0.f, Dn = 0.f;
+    if (M != -INFINITY) {
+        for (int s = warp; s < p.splits; s += kMergeWarps) {
+            const float* ps = base + s * split_stride;
+            const float ms = __ldcg(ps + kHeadDim);
+            const float w = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
+            acc = fmaf(w, __ldcg(ps + 32 * chunk + lane), acc);
+            L = fmaf(w, __ldcg(ps + kHeadDim + 1), L);
+            Dn = fmaf(w, __ldcg(ps + kHeadDim + 2), Dn);
         }
-        p.meter_raw[cell] = raw;
-        p.meter[cell] = fminf(1.0f, raw);
     }
     __syncthreads();
-    for (int idx = threadIdx.x; idx < G * kHeadDim; idx += kThreads) {
-        const int hh = idx / kHeadDim, d = idx % kHeadDim;
-        const float M = stat[hh * 3], L = stat[hh * 3 + 1];
-        float v = 0.f;
-        if (L > 0.f) {
-            for (int s = 0; s < p.splits; ++s) {
-                const float* ps = base + (s * kMaxGroup + hh) * kPartialStride;
-                const float ms = __ldcg(ps + kHeadDim);
-                if (ms == -INFINITY) continue;
-                v = fmaf(fast_exp2(ms - M), __ldcg(ps + d), v);
-            }
-            v /= L;
-        }
-        p.out[((size_t)b * p.num_q_heads + (size_t)h * G + hh) * kHeadDim + d] = v;
+    red[warp][lane] = acc;
+    if (lane == 0) {
+        red[warp][32] = L;
+        red[warp][33] = Dn;
     }
-    if (threadIdx.x == 0) p.counters[unit] = 0u;   // ready for the next call
+    __syncthreads();
+    if (warp == 0) {
+        float a = 0.f, l = 0.f, dn = 0.f;
+#pragma unroll
+        for (int w = 0; w < kMergeWarps; ++w) {
+            a += red[w][lane];
+            l += red[w][32];
+            dn += red[w][33];
+        }
+        const size_t cell = (size_t)b * p.num_q_heads + hq;
+        p.out[cell * kHeadDim + 32 * chunk + lane] = l > 0.f ? a / l : 0.f;
+        if (chunk == 0 && lane == 0) {
+            float raw = 0.f;
+            if (l > 0.f) {
+                const float D = dn / l;                 // A - 1
+                raw = 0.5f * D * (D + 2.0f);            // (A^2 - 1) / 2, +inf on overflow
+            }
+            p.meter_raw[cell] = raw;
+            p.meter[cell] = fminf(1.0f, raw);
+        }
+    }
 }
 
 }  // namespace
@@ -532,22 +564,22 @@ __global__ void __launch_bounds__(kThreads, 3) decode_kernel(const __grid_consta
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms) {
     DecodePlan pl;
     const long units = (long)batch * num_kv_heads;
-    const long target = (long)num_sms * 3;   // resident CTAs
+    const long target = (long)num_sms * kMinBlocks;   // resident CTAs
     long pps = (max_pages * units + target - 1) / target;
-    pps = std::max<long>(pps, 8);
+    pps = std::max<long>(pps, 16);
     pps = std::min<long>(pps, std::max(max_pages, 1));
     pl.pages_per_split = (int)pps;
     pl.splits = (int)std::max<long>(1, (max_pages + pps - 1) / pps);
     auto align = [](size_t x) { return (x + 255) & ~(size_t)255; };
     pl.counters_off = 256;
-    pl.partials_off = align(pl.counters_off + sizeof(uint32_t) * units);
+    pl.partials_off = 256;
     pl.total = align(pl.partials_off + sizeof(float) * (size_t)units * pl.splits * kMaxGroup * kPartialStride);
     return pl;
 }
 
 template <int kScheme, int kBits>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
-    static bool configured = false;   // per process; attribute is per function
+    static bool configured = false;   // per process; the attribute is per function
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
@@ -556,7 +588,21 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     }
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
     decode_kernel<kScheme, kBits><<<grid, kThreads, kSmemBytes, stream>>>(p);
-    return cudaGetLastError();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    // merge as a programmatic dependent launch: its CTAs are scheduled while
+    // the decode grid drains and wait (griddepcontrol.wait) for all of it
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(kHeadDim / 32, p.num_q_heads, p.batch);
+    cfg.blockDim = dim3(32 * kMergeWarps);
+    cfg.dynamicSmemBytes = 0;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, merge_kernel, p);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
