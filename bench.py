@@ -168,23 +168,24 @@ class Setup:
         self.keep_q = torch.empty(L * B * Hq, dtype=torch.uint8, device="cuda")
         self.keep_kv = torch.empty(L * B * Hq // wl.group, dtype=torch.uint8, device="cuda")
         self.n_kept = torch.empty(2, dtype=torch.int32, device="cuda")
-        # events recorded inside the captured graph must be "external" records
-        self.ev = [(_graph_event(), _graph_event()) for _ in range(L)]
         self.tau = wl.taus[0]
 
-    def step(self, timed_events=True):
+    def decode(self, layer):
+        self.wc.metered_decode_attention(self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer],
+                                         self.ws, out=self.out[layer], meter=self.meter[layer],
+                                         meter_raw=self.raw[layer])
+
+    def step(self):
         wc, wl = self.wc, self.wl
         for layer in range(wl.n_layers):
             wc.kv_quantize_witness(self.desc, layer, self.k_new[layer], self.v_new[layer], self.new_slots,
                                    self.caches[layer])
-            if timed_events:
-                self.ev[layer][0].record()
-            wc.metered_decode_attention(self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer],
-                                        self.ws, out=self.out[layer], meter=self.meter[layer],
-                                        meter_raw=self.raw[layer])
-            if timed_events:
-                self.ev[layer][1].record()
+            self.decode(layer)
         wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
+
+    def decode_all(self):
+        for layer in range(self.wl.n_layers):
+            self.decode(layer)
 
     def launches_per_step(self):
         # per layer: write kernel, decode kernel, merge kernel; then one gate
@@ -192,13 +193,6 @@ class Setup:
 
     def decode_bytes_per_launch(self):
         return sum(self.wl.ctx_lens) * self.wl.n_kv_heads * BYTES_PER_TOKEN_HEAD[self.wl.scheme]
-
-
-def _graph_event():
-    try:
-        return torch.cuda.Event(enable_timing=True, external=True)
-    except TypeError:
-        return torch.cuda.Event(enable_timing=True)
 
 
 def capture(fn):
@@ -236,9 +230,21 @@ def run_ours(args, rank, world, local):
     barrier(world)
     ms = t0.elapsed_time(t1) / args.steps
     ms = max_over_ranks(ms, world)
-    dec_ms = [a.elapsed_time(b) for a, b in st.ev]            # last replay, per layer
-    dec_avg_ms = sum(dec_ms) / len(dec_ms)
-    st.wc.read_status(st.ws)
+    status = st.wc.read_status(st.ws)
+
+    # ---- the dominant call alone: all layers' metered decode back to back ----
+    # (events only at the ends of the replayed graph, so they do not split it)
+    dgraph = capture(st.decode_all)
+    for _ in range(args.warmup):
+        dgraph.replay()
+    torch.cuda.synchronize()
+    d0, d1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    d0.record()
+    for _ in range(args.steps):
+        dgraph.replay()
+    d1.record()
+    torch.cuda.synchronize()
+    dec_avg_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
 
     kv_tokens_step = wl.kv_tokens
     value = kv_tokens_step * world / (ms / 1e3)
@@ -285,6 +291,7 @@ def run_ours(args, rank, world, local):
                           "bytes_per_token_head": WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme]},
         "gate": coverage,
         "gpu_launches": st.launches_per_step() * args.steps,
+        "device_status": status,
         "clocks": clk.summary(),
         "e2e": e2e,
     }
@@ -316,7 +323,7 @@ def run_e2e(st, args, world):
         for layer in range(wl.n_layers):
             st.k_new[layer].copy_(dev_k[layer], non_blocking=True)
             st.v_new[layer].copy_(dev_v[layer], non_blocking=True)
-        st.step(timed_events=False)
+        st.step()
         out_h.copy_(st.out, non_blocking=True)
         raw_h.copy_(st.raw, non_blocking=True)
         meter_h.copy_(st.meter, non_blocking=True)

@@ -34,7 +34,7 @@ constexpr int kStages = 3;
 constexpr int kMinBlocks = 2;            // two CTAs (16 warps) per SM
 constexpr int kStageBytes = 4416;   // K codes | V codes | K scale | V scale | witness
 constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
-constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8 + 16;
+constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8 + kMaxGroup * kHeadDim * 2;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;  // log2(e)/sqrt(128)
 
@@ -84,6 +84,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 
     uint8_t* my_stages = smem + warp * kStages * kStageBytes;
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageBytes) + warp * kStages;
+    if (lane == 0)
+        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
+    fence_barrier_init();
+    grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
     int ctx = __ldg(p.ctx_lens + b);
     if (ctx < 0 || ctx > p.max_pages * kPage) {
@@ -98,9 +102,6 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
 
     // ---- per-warp stage ring -------------------------------------------------
-    if (lane == 0)
-        for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
-    fence_barrier_init();
     __syncwarp();
 
     auto issue = [&](int k) {
@@ -128,15 +129,21 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 
     // ---- query fragments, band norms ------------------------------------------
     const bool row_valid = g < G;
-    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
-    {
-        const uint4* qsrc = reinterpret_cast<const uint4*>(
-            p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+    // q of the CTA's G heads, fp16 [kMaxGroup][128], after the stage rings
+    uint32_t* q_sm = reinterpret_cast<uint32_t*>(smem + kWarps * kStages * kStageBytes + kWarps * kStages * 8);
+    for (int i = threadIdx.x; i < kMaxGroup * kHeadDim / 8; i += kThreads) {
+        const int hh = i / (kHeadDim / 8), col = i % (kHeadDim / 8);
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (hh < G) v = __ldg(reinterpret_cast<const uint4*>(p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + hh) * kHeadDim) + col);
+        reinterpret_cast<uint4*>(q_sm)[i] = v;
+    }
+    __syncthreads();
+    const uint4* my_q = reinterpret_cast<const uint4*>(q_sm + g * (kHeadDim / 2) + 16 * c);   // head g, ch 32c..
+    uint32_t qw[16];
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
-            qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
-        }
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = my_q[i];
+        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
     }
     float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
@@ -169,8 +176,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         a_hi = pack_h2(__half2float(h0), __half2float(h1));
         a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
     }
-    // q . (code - xi) = q . (code + 1152) - q . h' + (kappa - 1152) sum(q)
-    const float zoff = kInt8 ? (DitherConst<kBits == 10 ? 10 : 8>::kappa - 1152.0f) * qsum : 0.f;
+    // q . (code - xi) = q . code - q . h' + kappa sum(q)
+    const float zoff = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa * qsum : 0.f;
 
     // ---- running state -----------------------------------------------------------
     // Log2-domain softmax reference m_run, moved lazily: only when a page's max
@@ -209,6 +216,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             for (int nt = 0; nt < 2; ++nt)
 #pragma unroll
                 for (int e = 0; e < 4; ++e) dc[nt][e] = dd[nt][e] = 0.f;
+            uint32_t qf[16];   // reloaded per page: keeps 16 registers free across the loop
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const uint4 v = my_q[i];
+                qf[4 * i] = v.x; qf[4 * i + 1] = v.y; qf[4 * i + 2] = v.z; qf[4 * i + 3] = v.w;
+            }
             // codes first, then the dither: their operands are never live together
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {                 // channels 32c + 16gp .. +15
@@ -219,13 +232,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const int ks = 4 * gp + kk;              // channels 32c + 4ks .. +3
-                    const uint32_t A[4] = {qw[2 * ks], 0u, qw[2 * ks + 1], 0u};
+                    const uint32_t A[4] = {qf[2 * ks], 0u, qf[2 * ks + 1], 0u};
 #pragma unroll
                     for (int nt = 0; nt < 2; ++nt) {
                         const uint32_t w = word_of(kq[nt], kk);
                         if constexpr (kInt8) {
                             const uint32_t wx = w ^ 0x80808080u;
-                            mma16816(dc[nt], A, s8x2_biased(wx, kSel01), s8x2_biased(wx, kSel23));
+                            mma16816(dc[nt], A, s8x2_to_h2(wx, kSel01), s8x2_to_h2(wx, kSel23));
                         } else {
                             mma16816(dc[nt], A, e4m3x2_to_h2(w), e4m3x2_to_h2(w >> 16));
                         }
@@ -234,17 +247,24 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             }
             if constexpr (kInt8) {
                 constexpr int kCalls = (kBits == 10) ? 4 : 2;     // Philox calls per token
+                constexpr int kBatch = (kBits == 10) ? 2 : 2;     // calls per token in flight
 #pragma unroll
-                for (int gi = 0; gi < kCalls; ++gi) {
-                    uint4 dk[2];
+                for (int g0 = 0; g0 < kCalls; g0 += kBatch) {
+                  uint4 dkb[kBatch][2];
+#pragma unroll
+                  for (int bi = 0; bi < kBatch; ++bi)
 #pragma unroll
                     for (int nt = 0; nt < 2; ++nt)
-                        dk[nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kCalls * c + gi), 0u, p.keys);
+                        dkb[bi][nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kCalls * c + g0 + bi), 0u, p.keys);
+#pragma unroll
+                  for (int bi = 0; bi < kBatch; ++bi) {
+                    const int gi = g0 + bi;
+                    const uint4* dk = dkb[bi];
                     constexpr int kSteps = 8 / kCalls;            // k-steps covered by one call
 #pragma unroll
                     for (int kk = 0; kk < kSteps; ++kk) {
                         const int ks = kSteps * gi + kk;
-                        const uint32_t A[4] = {qw[2 * ks], 0u, qw[2 * ks + 1], 0u};
+                        const uint32_t A[4] = {qf[2 * ks], 0u, qf[2 * ks + 1], 0u};
 #pragma unroll
                         for (int nt = 0; nt < 2; ++nt) {
                             uint32_t h0, h1;
@@ -259,6 +279,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                             mma16816(dd[nt], A, h0, h1);
                         }
                     }
+                  }
                 }
             }
 
@@ -469,20 +490,26 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     __syncthreads();
     const size_t unit = (size_t)b * p.num_kv_heads + h;
     float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
+    float* wts = reinterpret_cast<float*>(smem) + kWarps * kMaxGroup * kPartialStride;   // [head][warp]
+    if (threadIdx.x < kMaxGroup) {
+        const int hh = threadIdx.x;
+        float M = -INFINITY;
+        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim]);
+        for (int w = 0; w < kWarps; ++w) {
+            const float mw = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
+            wts[hh * (kWarps + 1) + w] = (mw == -INFINITY) ? 0.f : fast_exp2(mw - M);
+        }
+        wts[hh * (kWarps + 1) + kWarps] = M;
+    }
+    __syncthreads();
     for (int idx = threadIdx.x; idx < G * (kHeadDim + 3); idx += kThreads) {
         const int hh = idx / (kHeadDim + 3), col = idx % (kHeadDim + 3);
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim]);
-        float v = M;
+        const float* wh = wts + hh * (kWarps + 1);
+        float v = wh[kWarps];   // M
         if (col != kHeadDim) {
             v = 0.f;
 #pragma unroll
-            for (int w = 0; w < kWarps; ++w) {
-                const float* wb = mbuf + (w * kMaxGroup + hh) * kPartialStride;
-                const float sc = (wb[kHeadDim] == -INFINITY) ? 0.f : fast_exp2(wb[kHeadDim] - M);
-                v = fmaf(sc, wb[col], v);
-            }
+            for (int w = 0; w < kWarps; ++w) v = fmaf(wh[w], mbuf[(w * kMaxGroup + hh) * kPartialStride + col], v);
         }
         part_out[hh * kPartialStride + col] = v;
     }
@@ -509,6 +536,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     __shared__ float sM;
 
     float M = -INFINITY;
+#pragma unroll 4
     for (int s = warp; s < p.splits; s += kMergeWarps) M = fmaxf(M, __ldcg(base + s * split_stride + kHeadDim));
     if (lane == 0) red[warp][0] = M;
     __syncthreads();
@@ -521,6 +549,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     M = sM;
     float acc = 0.f, L = 0.f, Dn = 0.f;
     if (M != -INFINITY) {
+#pragma unroll 4
         for (int s = warp; s < p.splits; s += kMergeWarps) {
             const float* ps = base + s * split_stride;
             const float ms = __ldcg(ps + kHeadDim);
@@ -587,22 +616,12 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
         configured = true;
     }
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    decode_kernel<kScheme, kBits><<<grid, kThreads, kSmemBytes, stream>>>(p);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits>, grid, dim3(kThreads), kSmemBytes, stream, p);
     if (e != cudaSuccess) return e;
-    // merge as a programmatic dependent launch: its CTAs are scheduled while
+    // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(kHeadDim / 32, p.num_q_heads, p.batch);
-    cfg.blockDim = dim3(32 * kMergeWarps);
-    cfg.dynamicSmemBytes = 0;
-    cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, merge_kernel, p);
+    return launch_pdl(merge_kernel, dim3(kHeadDim / 32, p.num_q_heads, p.batch), dim3(32 * kMergeWarps), 0,
+                      stream, p);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {

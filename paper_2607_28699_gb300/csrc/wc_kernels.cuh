@@ -54,6 +54,23 @@ struct DecodePlan {
 
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms);
 
+// Launch `kernel` on `stream` as a programmatic dependent of the preceding work.
+template <typename Kernel, typename Params>
+inline cudaError_t launch_pdl(Kernel kernel, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              const Params& p) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, p);
+}
+
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float tau, uint8_t* keep_q,

@@ -29,7 +29,9 @@ __device__ __forceinline__ int dither_code(float x, float s, float inv_s, float 
 }
 
 template <int kScheme, int kBits>
-__global__ void __launch_bounds__(128) write_kernel(WriteParams p) {
+__global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ WriteParams p) {
+    grid_dep_wait();      // inputs may come from the preceding kernel
+    grid_dep_launch();    // a dependent decode waits for this whole grid anyway
     const int lane = threadIdx.x & 31;
     const int unit = (blockIdx.x * 4 + (threadIdx.x >> 5)) * 2 + (lane >> 4);  // token*Hkv + h
     const int row = (lane >> 3) & 1;                                             // 0 = K, 1 = V
@@ -38,17 +40,17 @@ __global__ void __launch_bounds__(128) write_kernel(WriteParams p) {
     const int tok = live_unit ? unit / p.num_kv_heads : 0;
     const int h = live_unit ? unit % p.num_kv_heads : 0;
     const int slot = live_unit ? __ldg(p.slot_mapping + tok) : -1;
-    const bool bad = slot >= p.num_pages * kPage;
-    const bool active = live_unit && slot >= 0 && !bad;
-    if (live_unit && bad && sub == 0 && row == 0 && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_SLOT);
-
-    // ---- load 16 fp16 channels -------------------------------------------
+    // the row loads do not depend on the slot: issue them alongside its load
     const __half* src = (row == 0 ? p.k : p.v) + ((size_t)tok * p.num_kv_heads + h) * kHeadDim + sub * 16;
     uint4 raw[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-    if (active) {
+    if (live_unit) {
         raw[0] = __ldg(reinterpret_cast<const uint4*>(src));
         raw[1] = __ldg(reinterpret_cast<const uint4*>(src) + 1);
     }
+    const bool bad = slot >= p.num_pages * kPage;
+    const bool active = live_unit && slot >= 0 && !bad;
+    if (live_unit && bad && sub == 0 && row == 0 && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_SLOT);
+    if (!active) raw[0] = raw[1] = make_uint4(0, 0, 0, 0);
     float x[16];
     {
         const __half2* hv = reinterpret_cast<const __half2*>(raw);
@@ -170,12 +172,9 @@ cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_
     const int blocks = (units + 7) / 8;
     if (blocks == 0) return cudaSuccess;
     if (scheme == WC_SCHEME_FP8_E4M3)
-        write_kernel<WC_SCHEME_FP8_E4M3, 8><<<blocks, 128, 0, stream>>>(p);
-    else if (bits == 8)
-        write_kernel<WC_SCHEME_DITHER_INT8, 8><<<blocks, 128, 0, stream>>>(p);
-    else
-        write_kernel<WC_SCHEME_DITHER_INT8, 10><<<blocks, 128, 0, stream>>>(p);
-    return cudaGetLastError();
+        return launch_pdl(write_kernel<WC_SCHEME_FP8_E4M3, 8>, dim3(blocks), dim3(128), 0, stream, p);
+    if (bits == 8) return launch_pdl(write_kernel<WC_SCHEME_DITHER_INT8, 8>, dim3(blocks), dim3(128), 0, stream, p);
+    return launch_pdl(write_kernel<WC_SCHEME_DITHER_INT8, 10>, dim3(blocks), dim3(128), 0, stream, p);
 }
 
 }  // namespace wc
