@@ -18,7 +18,17 @@ def close(gpu, ref, rtol=RTOL, atol=ATOL):
     return ok
 
 
+def margin(gpu, ref, rtol=RTOL, atol=ATOL):
+    """Largest |gpu - ref| / (atol + rtol |ref|) over finite entries (1.0 = at tolerance)."""
+    g, r = np.asarray(gpu, np.float64), np.asarray(ref, np.float64)
+    fin = np.isfinite(g) & np.isfinite(r)
+    if not np.any(fin):
+        return 0.0
+    return float(np.max(np.abs(g[fin] - r[fin]) / (atol + rtol * np.abs(r[fin]))))
+
+
 def assert_close(gpu, ref, what, rtol=RTOL, atol=ATOL):
+    print(f"[margin] {what}: {margin(gpu, ref, rtol, atol):.3f}")
     ok = close(gpu, ref, rtol, atol)
     if not np.all(ok):
         g, r = np.asarray(gpu, np.float64), np.asarray(ref, np.float64)
