@@ -37,6 +37,22 @@ WRITE_BYTES_PER_TOKEN_HEAD = {0: 512 + 276, 1: 512 + 272}
 METRIC = "metered decode KV tokens/s & HBM GB/s vs 8 TB/s; witness-write GB/s"
 
 
+def _traffic(workload):
+    """DRAM bytes per decode launch from the committed ncu summary, if the
+    kernel source is unchanged since the capture; else None."""
+    import hashlib
+    try:
+        src = open(os.path.join(ROOT, "paper_2607_28699_gb300", "csrc", "decode_kernel.cu"), "rb").read()
+        sha = hashlib.sha256(src).hexdigest()[:16]
+        for line in open(os.path.join(ROOT, "profiles", "traffic.txt")):
+            f = line.split()
+            if len(f) == 4 and f[0] == "decode_kernel" and f[1] == sha and f[2] == workload:
+                return int(f[3])
+    except OSError:
+        pass
+    return None
+
+
 def _peaks():
     try:
         return json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
@@ -283,7 +299,7 @@ def run_ours(args, rank, world, local):
         "decode_call_ms": dec_avg_ms,
         "roofline": {"kernel": "decode_kernel + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                     "frac": achieved / peak, "traffic": None,
+                     "frac": achieved / peak, "traffic": _traffic(wl.name),
                      "frac_of_nominal_8tbs": achieved / 8000.0,
                      "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peaks else "fallback 6.8 TB/s",
                      "algorithmic_bytes_per_launch": algo_bytes},
