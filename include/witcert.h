@@ -167,6 +167,38 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer,
                                       void* stream);
 
 /*
+ * Allocation-free metered decode.  The paper has no counterpart: this is a
+ * deployment convenience for callers that cannot allocate device memory at
+ * decode time (a runtime that pre-plans every buffer, code running inside an
+ * allocator's own hooks, a process under a fixed memory budget) and so cannot
+ * provide the workspace wc_metered_decode_attention needs.
+ *
+ * Same computation, arguments and outputs as wc_metered_decode_attention,
+ * without the workspace.  Its scratch is one fixed 4 MiB device array built
+ * into the library; every GPU that loads the library keeps it until the
+ * process exits.  The call never allocates or frees memory.
+ *   dev_status  optional device uint32 that collects WC_DEV_* bits (OR); when
+ *               NULL the bits go to a word inside the built-in scratch.
+ * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
+ * more scratch than 4 MiB (about 990 (sequence, KV head, split) partial
+ * results; the split count follows wc_workspace_size's plan).
+ * The first call on each device looks up the scratch address and clears its
+ * status word (a synchronous cudaMemset); make that first call before any
+ * stream capture.  All calls share the one scratch array and it keeps the
+ * last call's contents: calls that can overlap on the GPU (different streams,
+ * or several host threads) race and must be ordered by the caller.
+ */
+wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t layer,
+                                              const void* q, const int32_t* block_table,
+                                              int32_t max_pages, const int32_t* ctx_lens,
+                                              int32_t batch,
+                                              const void* k_codes, const void* v_codes,
+                                              const void* k_scale, const void* v_scale,
+                                              const void* k_witness,
+                                              float* out, float* meter, float* meter_raw,
+                                              uint32_t* dev_status, void* stream);
+
+/*
  * Gate (§6 meter-loop box; certified tau < 1 vs risk-ranked tau >= 1, §4.3).
  *
  * keep_q[i] = (meter_raw[i] <= tau) in fp32 (equality keeps the compressed

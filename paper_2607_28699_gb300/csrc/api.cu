@@ -2,6 +2,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <string>
 
 #include "wc_kernels.cuh"
@@ -210,3 +211,105 @@ wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word, uint32
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of the metered decode call.
+//
+// Some callers cannot allocate device memory when they call the decode: code
+// running where cudaMalloc is forbidden or unsafe (inside a custom allocator's
+// hooks, under a memory budget that must not move, or from a runtime that
+// pre-plans every buffer and hands the library only its inputs and outputs).
+// For them the scratch the decode needs (per-split partial results) lives in
+// one fixed device array compiled into this library.  Every GPU that loads the
+// library holds this array until the process exits.
+// ---------------------------------------------------------------------------
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;   // 4 MiB per device
+constexpr int kNoAllocMaxDevices = 64;
+
+// File-scope device scratch.  In host code this name is only a stand-in for
+// the device array, never a device address: the address is looked up once
+// per device with cudaGetSymbolAddress (below) and passed to the kernels.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+
+// Address of the scratch on the current device; looked up (and its status
+// word cleared) the first time a device is seen.
+wc_status noalloc_scratch(void** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(WC_ERR_UNSUPPORTED, "device index %d too large", dev);
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void* ptr = nullptr;
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the decode scratch");
+        e = cudaMemset(ptr, 0, 256);   // the status word must start at zero
+        if (e != cudaSuccess) return cuda_fail(e, "clearing the decode scratch status word");
+        g_noalloc_ptr[dev] = ptr;
+    }
+    *out = g_noalloc_ptr[dev];
+    return WC_OK;
+}
+
+}  // namespace
+
+extern "C" wc_status wc_metered_decode_attention_noalloc(
+    const wc_cache_desc* desc, int32_t layer, const void* q, const int32_t* block_table, int32_t max_pages,
+    const int32_t* ctx_lens, int32_t batch, const void* k_codes, const void* v_codes, const void* k_scale,
+    const void* v_scale, const void* k_witness, float* out, float* meter, float* meter_raw, uint32_t* dev_status,
+    void* stream) {
+    if (wc_status st = check_desc(desc)) return st;
+    if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
+    if (batch < 0 || batch > 65535) return fail(WC_ERR_INVALID_ARG, "batch must be in [0, 65535] (got %d)", batch);
+    if (max_pages < 1) return fail(WC_ERR_INVALID_ARG, "max_pages must be positive (got %d)", max_pages);
+    if ((long long)max_pages * wc::kPage > 0x7FFFFFFFLL) return fail(WC_ERR_UNSUPPORTED, "max_pages too large");
+    if (batch == 0) return WC_OK;
+    if (!q || !block_table || !ctx_lens || !out || !meter || !meter_raw)
+        return fail(WC_ERR_INVALID_ARG, "q, block_table, ctx_lens, out, meter, meter_raw must not be NULL");
+    if (!aligned16(q)) return fail(WC_ERR_INVALID_ARG, "q must be 16-byte aligned");
+    if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
+    int sms = 0;
+    if (current_sm_count(&sms) != 0) return fail(WC_ERR_CUDA, "cannot query the current device");
+    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms);
+    if (pl.total > kNoAllocScratchBytes)
+        return fail(WC_ERR_UNSUPPORTED,
+                    "this decode needs %zu bytes of scratch but the built-in scratch holds %zu; "
+                    "use wc_metered_decode_attention with a caller workspace",
+                    pl.total, kNoAllocScratchBytes);
+    void* scratch = nullptr;
+    if (wc_status st = noalloc_scratch(&scratch)) return st;
+    uint8_t* ws = static_cast<uint8_t*>(scratch);
+    wc::DecodeParams p;
+    p.q = static_cast<const __half*>(q);
+    p.block_table = block_table;
+    p.ctx_lens = ctx_lens;
+    p.k_codes = static_cast<const uint8_t*>(k_codes);
+    p.v_codes = static_cast<const uint8_t*>(v_codes);
+    p.k_scale = static_cast<const __half*>(k_scale);
+    p.v_scale = static_cast<const __half*>(v_scale);
+    p.k_witness = static_cast<const __half*>(k_witness);
+    p.out = out;
+    p.meter = meter;
+    p.meter_raw = meter_raw;
+    p.status = dev_status ? dev_status : reinterpret_cast<uint32_t*>(ws);
+    p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
+    p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
+    p.batch = batch;
+    p.max_pages = max_pages;
+    p.num_q_heads = desc->num_q_heads;
+    p.num_kv_heads = desc->num_kv_heads;
+    p.group = desc->num_q_heads / desc->num_kv_heads;
+    p.num_pages = desc->num_pages;
+    p.layer = layer;
+    p.rope_layout = desc->rope_layout;
+    p.splits = pl.splits;
+    p.pages_per_split = pl.pages_per_split;
+    p.keys = wc::make_philox_keys(desc->seed);
+    cudaError_t e = wc::launch_decode(p, desc->scheme, desc->dither_bits, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "decode kernel launch");
+}
