@@ -6,19 +6,19 @@
 // merged across context splits under log-sum-exp weights (A is a p~-weighted
 // mean, so it merges exactly like the output; §6.2.2).
 //
-// Grid (splits, Hkv, batch); 4 warps per CTA.  Each warp owns a 4-stage ring
-// of page buffers in shared memory filled by bulk asynchronous copies
-// (cp.async.bulk + mbarrier) that its lane 0 issues ahead of use; a page is
-// 16 tokens of one KV head (2 KiB K codes, 2 KiB V codes, scales, witness).
+// Grid (splits, Hkv, batch); 8 warps per CTA, two CTAs per SM.  Each warp owns
+// a 3-stage ring of page buffers in shared memory filled by bulk asynchronous
+// copies (cp.async.bulk + mbarrier) that its lane 0 issues ahead of use; a
+// page is 16 tokens of one KV head (2 KiB K codes, 2 KiB V codes, scales,
+// witness).  Warps run independently until the CTA's closing merge.
 //
-// Per page a warp computes, with mma.m16n8k16 (fp16 in, fp32 accumulate):
-//   QK:  D[head][token] = q . code - q . h'   (A = q, B = codes / dither),
-//   PV:  acc[dim][head] += code^T P - h'^T P (A = V codes / dither, B = P),
-// and the bound C[head][token] = a[head][band] . W[token][band] with
-// mma.m16n8k8 (a split into two fp16 terms).  Integer codes and the dither
-// (h' = 4 + j/256 for 8-bit, 1 + j/1024 for 10-bit; xi = h' - kappa) are
-// exact fp16 operands, so code - xi = code - h' + kappa is carried exactly
-// until the fp32 accumulators.
+// Per page a warp computes, on mma.sync (fp16 in, fp32 accumulate):
+//   QK:    S[token][head]  = code . q - h' . q                m16n8k16, A = codes / dither
+//   bound: C[token][head]  = W[token][band] . a[band][head]    m16n8k8, a = ||q_b||/sqrt(d) (hi + lo)
+//   PV:    acc[dim][head] += V^T P^T - H^T P^T                 m16n8k16, B = P^T (hi + lo, movmatrix)
+// Integer codes and the dither enter the tensor cores as exact fp16 values
+// (h' = 4 + j/256 for 8-bit, 1 + j/1024 for 10-bit dither; xi = h' - kappa),
+// so code - xi = code - h' + kappa is carried exactly to the fp32 accumulators.
 #include <algorithm>
 #include <climits>
 
@@ -32,11 +32,12 @@ constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kStages = 3;
 constexpr int kMinBlocks = 2;            // two CTAs (16 warps) per SM
-constexpr int kStageBytes = 4416;   // K codes | V codes | K scale | V scale | witness
+constexpr int kStageBytes = 4416;        // K codes | V codes | K scale | V scale | witness
 constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
-constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8 + kMaxGroup * kHeadDim * 2;
+constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8;
 constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;  // log2(e)/sqrt(128)
+constexpr float kRsd = 0.08838834764831845f;                      // 1/sqrt(128)
+constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;
 
 constexpr uint32_t kSel01 = 0x4140u, kSel23 = 0x4342u;   // [x0,K,x1,K], [x2,K,x3,K]
 
@@ -55,12 +56,6 @@ struct DitherConst<10> {  // xi = (j + 1/2)/1024 - 1/2 = h' - kappa, h' = 1 + j/
     static constexpr float kappa = 1.49951171875f;
 };
 
-// Two int8 codes as the fp16 pair 1152 + code (exact): (code ^ 0x80) in the
-// low mantissa byte of 1024.0.  The constant 1152 is removed once per logit.
-__device__ __forceinline__ uint32_t s8x2_biased(uint32_t w_xor80, uint32_t sel) {
-    return prmt(w_xor80, 0x64646464u, sel);
-}
-
 // h' pair (fp16) for two 8-bit dithers: bytes of x at the selector.
 __device__ __forceinline__ uint32_t h8(uint32_t x, uint32_t sel) { return prmt(x, 0x44444444u, sel); }
 // h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
@@ -71,6 +66,13 @@ __device__ __forceinline__ float pow2(int n) { return __int_as_float((127 + n) <
 
 __device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
     return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
+}
+
+// Transpose of an 8x8 b16 matrix held in the mma fragment layout.
+__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
+    uint32_t y;
+    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
+    return y;
 }
 
 template <int kScheme, int kBits>
@@ -89,24 +91,40 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     fence_barrier_init();
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
+    // Independent loads first: context length, this warp's first page-table
+    // entries and the query fragments do not depend on one another.
+    const int p0 = split * p.pages_per_split;
+    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+    const int lim = min(p0 + p.pages_per_split, p.max_pages);
+    int ring[kStages];   // physical pages of this warp's next kStages pages
+#pragma unroll
+    for (int k = 0; k < kStages; ++k) {
+        const int lp = p0 + warp + kWarps * k;
+        ring[k] = lp < lim ? __ldg(bt_row + lp) : -1;
+    }
     int ctx = __ldg(p.ctx_lens + b);
+    const bool row_valid = g < G;
+    const uint4* qsrc = reinterpret_cast<const uint4*>(
+        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
+        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+    }
+
     if (ctx < 0 || ctx > p.max_pages * kPage) {
         if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
         ctx = max(0, min(ctx, p.max_pages * kPage));
     }
     const int npages = (ctx + kPage - 1) / kPage;
-    const int p0 = split * p.pages_per_split;
     const int p1 = min(p0 + p.pages_per_split, npages);
     const int n_my = (p1 - p0 - warp > 0) ? (p1 - p0 - warp + kWarps - 1) / kWarps : 0;
-    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
     const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
 
-    // ---- per-warp stage ring -------------------------------------------------
-    __syncwarp();
-
-    auto issue = [&](int k) {
+    // ---- per-warp stage ring --------------------------------------------------
+    auto issue = [&](int k, int phys) {
         if (k >= n_my || lane != 0) return;
-        const int phys = __ldg(bt_row + p0 + warp + kWarps * k);
         uint64_t* bar = &bars[k % kStages];
         if (phys < 0 || phys >= p.num_pages) {
             atomicOr(p.status, WC_DEV_BAD_PAGE);
@@ -125,26 +143,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         }
         bulk_g2s(st + kOffW, p.k_witness + ph * (kPage * kBands), 256, bar);
     };
-    for (int k = 0; k < kStages; ++k) issue(k);
-
-    // ---- query fragments, band norms ------------------------------------------
-    const bool row_valid = g < G;
-    // q of the CTA's G heads, fp16 [kMaxGroup][128], after the stage rings
-    uint32_t* q_sm = reinterpret_cast<uint32_t*>(smem + kWarps * kStages * kStageBytes + kWarps * kStages * 8);
-    for (int i = threadIdx.x; i < kMaxGroup * kHeadDim / 8; i += kThreads) {
-        const int hh = i / (kHeadDim / 8), col = i % (kHeadDim / 8);
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (hh < G) v = __ldg(reinterpret_cast<const uint4*>(p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + hh) * kHeadDim) + col);
-        reinterpret_cast<uint4*>(q_sm)[i] = v;
-    }
-    __syncthreads();
-    const uint4* my_q = reinterpret_cast<const uint4*>(q_sm + g * (kHeadDim / 2) + 16 * c);   // head g, ch 32c..
-    uint32_t qw[16];
+    __syncwarp();
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 v = my_q[i];
-        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
-    }
+    for (int k = 0; k < kStages; ++k) issue(k, ring[k]);
+
+    // ---- band norms and the bound operand ----------------------------------------
     float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -169,21 +172,23 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         band_a = part[0] + part[1];   // dims 32c .. 32c+15 = band 2c
         band_b = part[2] + part[3];
     }
-    uint32_t a_hi = 0, a_lo = 0;   // bound A fragment, rows g (rows g+8 are zero)
+    uint32_t a_hi = 0, a_lo = 0;   // B operand of the bound: a[head g][bands 2c, 2c+1]
     if (row_valid) {
-        const float x0 = sqrtf(band_a) * 0.08838834764831845f, x1 = sqrtf(band_b) * 0.08838834764831845f;
+        const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
         const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
         a_hi = pack_h2(__half2float(h0), __half2float(h1));
         a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
     }
-    // q . (code - xi) = q . code - q . h' + kappa sum(q)
-    const float zoff = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa * qsum : 0.f;
+    // this thread's softmax heads are 2c and 2c+1: kappa * sum(q) for each
+    constexpr float kKappa = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
+    const float zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
+    const float zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
 
-    // ---- running state -----------------------------------------------------------
-    // Log2-domain softmax reference m_run, moved lazily: only when a page's max
+    // ---- running state (heads 2c, 2c+1) ----------------------------------------------
+    // Log2-domain softmax reference, moved lazily: only when a page's max
     // exceeds it by more than 8 (P may reach 2^8 in between).
-    float m_run = -INFINITY;
-    float l_part = 0.f, d_part = 0.f, spv_part = 0.f;
+    float m_run[2] = {-INFINITY, -INFINITY};
+    float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
@@ -191,12 +196,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     int lam_exp = kInt8 ? INT_MIN : 6;
     bool failed = false;
     int consumed = 0;
-    int phys_next = n_my > 0 ? __ldg(bt_row + p0 + warp) : 0;
 
     for (int k = 0; k < n_my; ++k) {
         const int lp = p0 + warp + kWarps * k;
-        const int phys = phys_next;
-        if (k + 1 < n_my) phys_next = __ldg(bt_row + lp + kWarps);
+        const int phys = ring[0];
+        // page-table entry for the page issued at the end of this iteration
+        const int phys_issue = (k + kStages < n_my) ? __ldg(bt_row + lp + kWarps * kStages) : -1;
         const bool page_ok = phys >= 0 && phys < p.num_pages;
         const bool landed = mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
         if (!__all_sync(0xffffffffu, landed)) {   // warp-uniform decision
@@ -210,142 +215,120 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             const uint32_t slot0 = (uint32_t)phys * kPage;
             const int nvalid = min(kPage, ctx - lp * kPage);
 
-            // ---------------- QK: D[head][token] ------------------------------
-            float dc[2][4], dd[2][4];
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) dc[nt][e] = dd[nt][e] = 0.f;
-            uint32_t qf[16];   // reloaded per page: keeps 16 registers free across the loop
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint4 v = my_q[i];
-                qf[4 * i] = v.x; qf[4 * i + 1] = v.y; qf[4 * i + 2] = v.z; qf[4 * i + 3] = v.w;
-            }
-            // codes first, then the dither: their operands are never live together
+            // ---------------- QK: S[token][head] --------------------------------
+            // rows g and g+8 are tokens g and g+8; d*[0..3] =
+            // (tok g, head 2c), (tok g, 2c+1), (tok g+8, 2c), (tok g+8, 2c+1)
+            float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {                 // channels 32c + 16gp .. +15
-                uint4 kq[2];
-#pragma unroll
-                for (int nt = 0; nt < 2; ++nt)
-                    kq[nt] = *reinterpret_cast<const uint4*>(st + (8 * nt + g) * kHeadDim + 32 * c + 16 * gp);
+                const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + 32 * c + 16 * gp);
+                const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + 32 * c + 16 * gp);
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const int ks = 4 * gp + kk;              // channels 32c + 4ks .. +3
-                    const uint32_t A[4] = {qf[2 * ks], 0u, qf[2 * ks + 1], 0u};
-#pragma unroll
-                    for (int nt = 0; nt < 2; ++nt) {
-                        const uint32_t w = word_of(kq[nt], kk);
-                        if constexpr (kInt8) {
-                            const uint32_t wx = w ^ 0x80808080u;
-                            mma16816(dc[nt], A, s8x2_to_h2(wx, kSel01), s8x2_to_h2(wx, kSel23));
-                        } else {
-                            mma16816(dc[nt], A, e4m3x2_to_h2(w), e4m3x2_to_h2(w >> 16));
-                        }
+                    const uint32_t wa = word_of(ka, kk), wb = word_of(kb, kk);
+                    uint32_t A[4];
+                    if constexpr (kInt8) {
+                        const uint32_t xa = wa ^ 0x80808080u, xb = wb ^ 0x80808080u;
+                        A[0] = s8x2_to_h2(xa, kSel01);
+                        A[1] = s8x2_to_h2(xb, kSel01);
+                        A[2] = s8x2_to_h2(xa, kSel23);
+                        A[3] = s8x2_to_h2(xb, kSel23);
+                    } else {
+                        A[0] = e4m3x2_to_h2(wa);
+                        A[1] = e4m3x2_to_h2(wb);
+                        A[2] = e4m3x2_to_h2(wa >> 16);
+                        A[3] = e4m3x2_to_h2(wb >> 16);
                     }
+                    mma16816(dc, A, qw[2 * ks], qw[2 * ks + 1]);
                 }
             }
             if constexpr (kInt8) {
                 constexpr int kCalls = (kBits == 10) ? 4 : 2;     // Philox calls per token
-                constexpr int kBatch = (kBits == 10) ? 2 : 2;     // calls per token in flight
+                constexpr int kSteps = 8 / kCalls;                // k-steps covered by one call
 #pragma unroll
-                for (int g0 = 0; g0 < kCalls; g0 += kBatch) {
-                  uint4 dkb[kBatch][2];
-#pragma unroll
-                  for (int bi = 0; bi < kBatch; ++bi)
-#pragma unroll
-                    for (int nt = 0; nt < 2; ++nt)
-                        dkb[bi][nt] = philox(slot0 + 8 * nt + g, c1, (uint32_t)(kCalls * c + g0 + bi), 0u, p.keys);
-#pragma unroll
-                  for (int bi = 0; bi < kBatch; ++bi) {
-                    const int gi = g0 + bi;
-                    const uint4* dk = dkb[bi];
-                    constexpr int kSteps = 8 / kCalls;            // k-steps covered by one call
+                for (int gi = 0; gi < kCalls; ++gi) {
+                    const uint4 da = philox(slot0 + g, c1, (uint32_t)(kCalls * c + gi), 0u, p.keys);
+                    const uint4 db = philox(slot0 + g + 8, c1, (uint32_t)(kCalls * c + gi), 0u, p.keys);
 #pragma unroll
                     for (int kk = 0; kk < kSteps; ++kk) {
                         const int ks = kSteps * gi + kk;
-                        const uint32_t A[4] = {qf[2 * ks], 0u, qf[2 * ks + 1], 0u};
-#pragma unroll
-                        for (int nt = 0; nt < 2; ++nt) {
-                            uint32_t h0, h1;
-                            if constexpr (kBits == 8) {
-                                const uint32_t dw = word_of(dk[nt], kk);
-                                h0 = h8(dw, kSel01);
-                                h1 = h8(dw, kSel23);
-                            } else {
-                                h0 = h10(word_of(dk[nt], 2 * kk));
-                                h1 = h10(word_of(dk[nt], 2 * kk + 1));
-                            }
-                            mma16816(dd[nt], A, h0, h1);
+                        uint32_t A[4];
+                        if constexpr (kBits == 8) {
+                            const uint32_t xa = word_of(da, kk), xb = word_of(db, kk);
+                            A[0] = h8(xa, kSel01);
+                            A[1] = h8(xb, kSel01);
+                            A[2] = h8(xa, kSel23);
+                            A[3] = h8(xb, kSel23);
+                        } else {
+                            A[0] = h10(word_of(da, 2 * kk));
+                            A[1] = h10(word_of(db, 2 * kk));
+                            A[2] = h10(word_of(da, 2 * kk + 1));
+                            A[3] = h10(word_of(db, 2 * kk + 1));
                         }
+                        mma16816(dd, A, qw[2 * ks], qw[2 * ks + 1]);
                     }
-                  }
                 }
             }
 
-            // ---------------- logits, bound, softmax --------------------------
-            float y[2][2], cb[2][2], sv[2][2];
-#pragma unroll
-            for (int nt = 0; nt < 2; ++nt) {
-                float db[4] = {0.f, 0.f, 0.f, 0.f};
-                const uint32_t wreg = *reinterpret_cast<const uint32_t*>(
-                    st + kOffW + ((8 * nt + g) * kBands + 2 * c) * 2);
-                mma1688(db, a_hi, 0u, wreg);
-                mma1688(db, a_lo, 0u, wreg);
-                float sk0 = 1.f, sk1 = 1.f;
-                if constexpr (kInt8) {
-                    const float2 sk = __half22float2(
-                        *reinterpret_cast<const __half2*>(st + kOffKs + (8 * nt + 2 * c) * 2));
-                    const float2 vv = __half22float2(
-                        *reinterpret_cast<const __half2*>(st + kOffVs + (8 * nt + 2 * c) * 2));
-                    sk0 = sk.x; sk1 = sk.y;
-                    sv[nt][0] = vv.x; sv[nt][1] = vv.y;
-                } else {
-                    sv[nt][0] = sv[nt][1] = 1.f;
-                }
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const int t = 8 * nt + 2 * c + e;
-                    const float raw = kInt8 ? (dc[nt][e] - dd[nt][e] + zoff) : dc[nt][e];
-                    const bool ok = t < nvalid;
-                    y[nt][e] = ok ? raw * ((e ? sk1 : sk0) * kRsdLog2e) : -INFINITY;
-                    cb[nt][e] = ok ? db[e] : 0.f;   // tail slots may hold any bits
-                    if (!ok) sv[nt][e] = 0.f;
-                }
+            // ---------------- logits, bound, softmax ------------------------------
+            float cb[4] = {0.f, 0.f, 0.f, 0.f};
+            {
+                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kOffW + (g * kBands + 2 * c) * 2);
+                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kOffW + ((g + 8) * kBands + 2 * c) * 2);
+                mma1688(cb, wa, wb, a_hi);
+                mma1688(cb, wa, wb, a_lo);
             }
-            float mx = fmaxf(fmaxf(y[0][0], y[0][1]), fmaxf(y[1][0], y[1][1]));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 1));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, 2));
-            const bool move = mx > m_run + 8.0f;
-            if (__any_sync(0xffffffffu, move)) {
-                const float alpha = move ? (m_run == -INFINITY ? 0.f : fast_exp2(m_run - mx)) : 1.f;
-                if (move) m_run = mx;
-                l_part *= alpha;
-                d_part *= alpha;
-                spv_part *= alpha;
-                const float a0 = __shfl_sync(0xffffffffu, alpha, 8 * c);      // head 2c
-                const float a1 = __shfl_sync(0xffffffffu, alpha, 8 * c + 4);  // head 2c+1
+            float sk[2] = {1.f, 1.f}, sv[2] = {1.f, 1.f};   // tokens g, g+8
+            if constexpr (kInt8) {
+                const __half* ks = reinterpret_cast<const __half*>(st + kOffKs);
+                const __half* vs = reinterpret_cast<const __half*>(st + kOffVs);
+                sk[0] = __half2float(ks[g]); sk[1] = __half2float(ks[g + 8]);
+                sv[0] = __half2float(vs[g]); sv[1] = __half2float(vs[g + 8]);
+            }
+            float y[4], P[4];
+            const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = i >> 1, e = i & 1;
+                const bool ok = r ? ok1 : ok0;
+                const float raw = kInt8 ? (dc[i] - dd[i] + (e ? zoff1 : zoff0)) : dc[i];
+                y[i] = ok ? raw * (sk[r] * kRsdLog2e) : -INFINITY;
+                if (!ok) cb[i] = 0.f;                 // tail slots may hold any bits
+            }
+            if (!ok0) sv[0] = 0.f;
+            if (!ok1) sv[1] = 0.f;
+            float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+#pragma unroll
+            for (int o = 4; o < 32; o <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+            }
+            const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
+            if (__any_sync(0xffffffffu, mv0 || mv1)) {
+                const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
+                const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
+                if (mv0) m_run[0] = mx0;
+                if (mv1) m_run[1] = mx1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
                     acc[mt][1] *= a1; acc[mt][3] *= a1;
                 }
             }
-            float P[2][2];
-            float smax = 0.f;
 #pragma unroll
-            for (int nt = 0; nt < 2; ++nt)
-#pragma unroll
-                for (int e = 0; e < 2; ++e) {
-                    const float pe = fast_exp2(y[nt][e] - m_run);    // 0 for masked tokens
-                    l_part += pe;
-                    d_part = fmaf(pe, fast_exp2(cb[nt][e] * kLog2e) - 1.f, d_part);
-                    const float pv = pe * sv[nt][e];
-                    spv_part += pv;
-                    P[nt][e] = pv;
-                    smax = fmaxf(smax, sv[nt][e]);
-                }
+            for (int i = 0; i < 4; ++i) {
+                const int r = i >> 1, e = i & 1;
+                const float pe = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
+                l_part[e] += pe;
+                d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                P[i] = pe * sv[r];
+                spv_part[e] += P[i];
+            }
             if constexpr (kInt8) {
+                const float smax = fmaxf(sv[0], sv[1]);
                 const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
                 if (wmax > 0.f) {
                     const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
@@ -362,22 +345,25 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                     }
                 }
             }
-            const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
-            // B = P^T as a sum of two fp16 terms (hi + lo): the output is a
-            // sum with heavy cancellation, so one fp16 rounding of P is not
-            // accurate enough.  Tokens 2c, 2c+1 (b*0) and 8+2c, 9+2c (b*1).
+            // B = P^T for PV as two fp16 terms (hi + lo): the output is a sum with
+            // heavy cancellation, one fp16 rounding of P is not accurate enough.
+            // Packed as 8x8 blocks [token][head] (tokens 0-7 and 8-15) and
+            // transposed with movmatrix into (P[tok 2c][head g], P[tok 2c+1][head g]).
             uint32_t bp0, bp1, bl0, bl1;
             {
-                const float x00 = P[0][0] * lam, x01 = P[0][1] * lam, x10 = P[1][0] * lam, x11 = P[1][1] * lam;
-                bp0 = pack_h2(x00, x01);
-                bp1 = pack_h2(x10, x11);
-                const float2 r0 = __half22float2(*reinterpret_cast<const __half2*>(&bp0));
-                const float2 r1 = __half22float2(*reinterpret_cast<const __half2*>(&bp1));
-                bl0 = pack_h2(x00 - r0.x, x01 - r0.y);
-                bl1 = pack_h2(x10 - r1.x, x11 - r1.y);
+                const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
+                const float x0 = P[0] * lam, x1 = P[1] * lam, x2 = P[2] * lam, x3 = P[3] * lam;
+                const uint32_t h01 = pack_h2(x0, x1), h23 = pack_h2(x2, x3);
+                const float2 r01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
+                const float2 r23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
+                const uint32_t l01 = pack_h2(x0 - r01.x, x1 - r01.y), l23 = pack_h2(x2 - r23.x, x3 - r23.y);
+                bp0 = movmatrix_t(h01);
+                bp1 = movmatrix_t(h23);
+                bl0 = movmatrix_t(l01);
+                bl1 = movmatrix_t(l23);
             }
 
-            // ---------------- PV: acc[dim][head] ------------------------------
+            // ---------------- PV: acc[dim][head] ------------------------------------
             const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
             uint4 vq[4];
 #pragma unroll
@@ -450,7 +436,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             }
         }
         __syncwarp();
-        issue(k + kStages);
+        issue(k + kStages, phys_issue);
+#pragma unroll
+        for (int i = 0; i + 1 < kStages; ++i) ring[i] = ring[i + 1];
+        ring[kStages - 1] = phys_issue;
     }
     if (failed) {
         // let copies still in flight land before the CTA's smem is released
@@ -458,74 +447,95 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             (void)mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
     }
 
-    // ---- warp partials -> shared, merge the warps of this CTA ----------------------
+    // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
 #pragma unroll
-    for (int o = 1; o < 4; o <<= 1) {
-        l_part += __shfl_xor_sync(0xffffffffu, l_part, o);
-        d_part += __shfl_xor_sync(0xffffffffu, d_part, o);
-        spv_part += __shfl_xor_sync(0xffffffffu, spv_part, o);
-    }
+    for (int o = 4; o < 32; o <<= 1)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
+            d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+            spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
+        }
     const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
     const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
-    const float spv0 = __shfl_sync(0xffffffffu, spv_part, 8 * c);
-    const float spv1 = __shfl_sync(0xffffffffu, spv_part, 8 * c + 4);
+
+    // ---- CTA merge: warps -> shared, one partial per CTA -----------------------------
     __syncthreads();   // stage buffers are reused below
     float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
     {
         float* wb = mbuf + warp * kMaxGroup * kPartialStride;
 #pragma unroll
-        for (int mt = 0; mt < 8; ++mt) {
-            const int d0 = 16 * g + 2 * mt;
-            wb[(2 * c) * kPartialStride + d0] = fmaf(acc[mt][0], inv_lam, kap * spv0);
-            wb[(2 * c + 1) * kPartialStride + d0] = fmaf(acc[mt][1], inv_lam, kap * spv1);
-            wb[(2 * c) * kPartialStride + d0 + 1] = fmaf(acc[mt][2], inv_lam, kap * spv0);
-            wb[(2 * c + 1) * kPartialStride + d0 + 1] = fmaf(acc[mt][3], inv_lam, kap * spv1);
-        }
-        if (c == 0) {
-            wb[g * kPartialStride + kHeadDim + 0] = m_run;
-            wb[g * kPartialStride + kHeadDim + 1] = l_part;
-            wb[g * kPartialStride + kHeadDim + 2] = d_part;
+        for (int e = 0; e < 2; ++e) {
+            float* row = wb + (2 * c + e) * kPartialStride + 16 * g;   // dims 16g .. 16g+15
+            const float add = kap * spv_part[e];
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                float4 v;
+                v.x = fmaf(acc[2 * q4][e], inv_lam, add);
+                v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
+                v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
+                v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
+                *reinterpret_cast<float4*>(row + 4 * q4) = v;
+            }
+            if (g == 0) {
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+            }
         }
     }
     __syncthreads();
     const size_t unit = (size_t)b * p.num_kv_heads + h;
     float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
-    float* wts = reinterpret_cast<float*>(smem) + kWarps * kMaxGroup * kPartialStride;   // [head][warp]
-    if (threadIdx.x < kMaxGroup) {
-        const int hh = threadIdx.x;
+    // thread -> (head, 4-dim chunk); chunk 32 carries (M, l, D)
+    for (int idx = threadIdx.x; idx < G * 33; idx += kThreads) {
+        const int hh = idx / 33, ch = idx % 33;
+        float mw[kWarps];
         float M = -INFINITY;
-        for (int w = 0; w < kWarps; ++w) M = fmaxf(M, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim]);
-        for (int w = 0; w < kWarps; ++w) {
-            const float mw = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
-            wts[hh * (kWarps + 1) + w] = (mw == -INFINITY) ? 0.f : fast_exp2(mw - M);
-        }
-        wts[hh * (kWarps + 1) + kWarps] = M;
-    }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < G * (kHeadDim + 3); idx += kThreads) {
-        const int hh = idx / (kHeadDim + 3), col = idx % (kHeadDim + 3);
-        const float* wh = wts + hh * (kWarps + 1);
-        float v = wh[kWarps];   // M
-        if (col != kHeadDim) {
-            v = 0.f;
 #pragma unroll
-            for (int w = 0; w < kWarps; ++w) v = fmaf(wh[w], mbuf[(w * kMaxGroup + hh) * kPartialStride + col], v);
+        for (int w = 0; w < kWarps; ++w) {
+            mw[w] = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
+            M = fmaxf(M, mw[w]);
         }
-        part_out[hh * kPartialStride + col] = v;
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int col = (ch < 32) ? 4 * ch : kHeadDim + 1;   // chunk 32: l, D
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            if (mw[w] == -INFINITY) continue;   // a warp without pages: its values are not read
+            const float wt = fast_exp2(mw[w] - M);
+            const float* src = mbuf + (w * kMaxGroup + hh) * kPartialStride + col;
+            if (ch < 32) {
+                const float4 v = *reinterpret_cast<const float4*>(src);
+                s.x = fmaf(wt, v.x, s.x); s.y = fmaf(wt, v.y, s.y);
+                s.z = fmaf(wt, v.z, s.z); s.w = fmaf(wt, v.w, s.w);
+            } else {
+                s.x = fmaf(wt, src[0], s.x);   // l
+                s.y = fmaf(wt, src[1], s.y);   // D
+            }
+        }
+        float* dst = part_out + hh * kPartialStride;
+        if (ch < 32) {
+            *reinterpret_cast<float4*>(dst + 4 * ch) = s;
+        } else {
+            dst[kHeadDim] = M;
+            dst[kHeadDim + 1] = s.x;
+            dst[kHeadDim + 2] = s.y;
+        }
     }
     // the merge kernel (launched as a programmatic dependent) may start now;
     // it waits for this whole grid before reading the partials
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    grid_dep_launch();
 }
 
 // Merge of the per-split partials of one (sequence, query head), 32 output
 // dims per CTA: out = sum_s w_s acc_s / sum_s w_s l_s with w_s = 2^(m_s - M),
 // D = sum_s w_s D_s / sum_s w_s l_s, meter_raw = D (D + 2) / 2 (§6.2.2: the
-// meter accumulator merges under the same LSE weights as the output).
+// meter accumulator merges under the same LSE weights as the output).  Each
+// warp folds its splits with a running maximum in one pass.
 constexpr int kMergeWarps = 8;
 
 __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_constant__ DecodeParams p) {
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    grid_dep_wait();
     const int chunk = blockIdx.x, hq = blockIdx.y, b = blockIdx.z;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int h = hq / p.group, hh = hq % p.group;
@@ -533,46 +543,65 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride) + hh * kPartialStride;
     const size_t split_stride = kMaxGroup * kPartialStride;
     __shared__ float red[kMergeWarps][36];
-    __shared__ float sM;
 
-    float M = -INFINITY;
-#pragma unroll 4
-    for (int s = warp; s < p.splits; s += kMergeWarps) M = fmaxf(M, __ldcg(base + s * split_stride + kHeadDim));
-    if (lane == 0) red[warp][0] = M;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        float m = -INFINITY;
-        for (int w = 0; w < kMergeWarps; ++w) m = fmaxf(m, red[w][0]);
-        sM = m;
-    }
-    __syncthreads();
-    M = sM;
-    float acc = 0.f, L = 0.f, Dn = 0.f;
-    if (M != -INFINITY) {
-#pragma unroll 4
-        for (int s = warp; s < p.splits; s += kMergeWarps) {
-            const float* ps = base + s * split_stride;
-            const float ms = __ldcg(ps + kHeadDim);
-            const float w = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
-            acc = fmaf(w, __ldcg(ps + 32 * chunk + lane), acc);
-            L = fmaf(w, __ldcg(ps + kHeadDim + 1), L);
-            Dn = fmaf(w, __ldcg(ps + kHeadDim + 2), Dn);
+    // all of this warp's split rows of a round are loaded before any is
+    // combined, so the loads overlap (one memory latency per round, not per split)
+    constexpr int kMaxRows = 16;   // rows per warp and round
+    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f;
+    for (int s0 = warp; s0 < p.splits; s0 += kMergeWarps * kMaxRows) {
+        float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows];
+#pragma unroll
+        for (int i = 0; i < kMaxRows; ++i) {
+            const int s = s0 + i * kMergeWarps;
+            ms[i] = -INFINITY;
+            v[i] = ls[i] = ds[i] = 0.f;
+            if (s < p.splits) {
+                const float* ps = base + s * split_stride;
+                ms[i] = __ldcg(ps + kHeadDim);
+                v[i] = __ldcg(ps + 32 * chunk + lane);
+                ls[i] = __ldcg(ps + kHeadDim + 1);
+                ds[i] = __ldcg(ps + kHeadDim + 2);
+            }
+        }
+        float Mr = M;
+#pragma unroll
+        for (int i = 0; i < kMaxRows; ++i) Mr = fmaxf(Mr, ms[i]);
+        if (Mr == -INFINITY) continue;
+        if (Mr > M) {   // move the running sums to the new reference
+            const float f = (M == -INFINITY) ? 0.f : fast_exp2(M - Mr);
+            acc *= f; L *= f; Dn *= f;
+            M = Mr;
+        }
+#pragma unroll
+        for (int i = 0; i < kMaxRows; ++i) {
+            if (ms[i] == -INFINITY) continue;          // empty split: values not read
+            const float w = fast_exp2(ms[i] - M);
+            acc = fmaf(w, v[i], acc);
+            L = fmaf(w, ls[i], L);
+            Dn = fmaf(w, ds[i], Dn);
         }
     }
-    __syncthreads();
     red[warp][lane] = acc;
     if (lane == 0) {
-        red[warp][32] = L;
-        red[warp][33] = Dn;
+        red[warp][32] = M;
+        red[warp][33] = L;
+        red[warp][34] = Dn;
     }
     __syncthreads();
     if (warp == 0) {
-        float a = 0.f, l = 0.f, dn = 0.f;
+        float Mt = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < kMergeWarps; ++w) {
-            a += red[w][lane];
-            l += red[w][32];
-            dn += red[w][33];
+        for (int w = 0; w < kMergeWarps; ++w) Mt = fmaxf(Mt, red[w][32]);
+        float a = 0.f, l = 0.f, dn = 0.f;
+        if (Mt != -INFINITY) {
+#pragma unroll
+            for (int w = 0; w < kMergeWarps; ++w) {
+                if (red[w][32] == -INFINITY) continue;
+                const float f = fast_exp2(red[w][32] - Mt);
+                a = fmaf(f, red[w][lane], a);
+                l = fmaf(f, red[w][33], l);
+                dn = fmaf(f, red[w][34], dn);
+            }
         }
         const size_t cell = (size_t)b * p.num_q_heads + hq;
         p.out[cell * kHeadDim + 32 * chunk + lane] = l > 0.f ? a / l : 0.f;
@@ -608,10 +637,18 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms) 
 
 template <int kScheme, int kBits>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
-    static bool configured = false;   // per process; the attribute is per function
+    static bool configured = false;   // per process; the attributes are per function
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
+        if (e != cudaSuccess) return e;
+        // the library's kernels all prefer the largest shared-memory carveout,
+        // so consecutive launches do not reconfigure the L1 / shared split
+        e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
     }

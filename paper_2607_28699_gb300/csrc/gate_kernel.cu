@@ -51,6 +51,13 @@ __global__ void __launch_bounds__(kGateThreads) gate_kernel(const float* __restr
 
 cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float tau, uint8_t* keep_q,
                         uint8_t* keep_kv, int32_t* n_kept, cudaStream_t stream) {
+    static bool configured = false;   // same carveout as the decode kernels
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(gate_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                             (int)cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
     gate_kernel<<<1, kGateThreads, 0, stream>>>(meter_raw, n_cells, group, tau, keep_q, keep_kv, n_kept);
     return cudaGetLastError();
 }

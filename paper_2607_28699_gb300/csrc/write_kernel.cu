@@ -171,6 +171,18 @@ cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_
     const int units = p.n_tok * p.num_kv_heads;
     const int blocks = (units + 7) / 8;
     if (blocks == 0) return cudaSuccess;
+    static bool configured = false;   // same carveout as the decode kernels: no L1/shared reconfiguration
+    if (!configured) {
+        const void* fns[3] = {(const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10>};
+        for (const void* f : fns) {
+            cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                                 (int)cudaSharedmemCarveoutMaxShared);
+            if (e != cudaSuccess) return e;
+        }
+        configured = true;
+    }
     if (scheme == WC_SCHEME_FP8_E4M3)
         return launch_pdl(write_kernel<WC_SCHEME_FP8_E4M3, 8>, dim3(blocks), dim3(128), 0, stream, p);
     if (bits == 8) return launch_pdl(write_kernel<WC_SCHEME_DITHER_INT8, 8>, dim3(blocks), dim3(128), 0, stream, p);
