@@ -159,22 +159,29 @@ class Setup:
         last = np.cumsum(wl.ctx_lens) - 1                       # index of each sequence's newest token
         self.new_slots = self.sm[torch.from_numpy(last).cuda()].contiguous()
         self.caches, self.k_new, self.v_new = [], [], []
-        self.prefill_write_s = 0.0
-        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         for layer in range(wl.n_layers):
             k, v = W.layer_kv(wl, layer, device="cuda")
             cache = wc.LayerCache.empty(self.desc)
-            torch.cuda.synchronize()
-            s.record()
-            wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, cache)
-            e.record()
-            e.synchronize()
-            self.prefill_write_s += s.elapsed_time(e) / 1e3
+            wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, cache)   # prefill write
             self.caches.append(cache)
             li = torch.from_numpy(last).cuda()
             self.k_new.append(k[li].contiguous())
             self.v_new.append(v[li].contiguous())
-            del k, v
+            if layer + 1 < wl.n_layers:
+                del k, v
+        # write-path throughput: the last layer's whole prefill, rewritten
+        # (same inputs, same slots) by warm, back-to-back calls
+        reps = 10
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.caches[-1])
+        torch.cuda.synchronize()
+        s.record()
+        for _ in range(reps):
+            wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.caches[-1])
+        e.record()
+        e.synchronize()
+        self.write_call_s = s.elapsed_time(e) / 1e3 / reps
+        del k, v
         self.q = torch.stack([W.layer_queries(wl, layer, device="cuda") for layer in range(wl.n_layers)])
         self.ws = wc.Workspace(self.desc, wl.batch, wl.max_pages)
         L, B, Hq = wl.n_layers, wl.batch, wl.n_q_heads
@@ -273,9 +280,9 @@ def run_ours(args, rank, world, local):
     # ---- end-to-end: host buffers, copies inside the timed region --------
     e2e = run_e2e(st, args, world)
 
-    # ---- write path: full prefill write of the cache ---------------------
-    write_th = sum(wl.ctx_lens) * wl.n_layers * wl.n_kv_heads
-    write_gbs = write_th * WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme] / st.prefill_write_s / 1e9
+    # ---- write path: one layer's full prefill (all sequences, all KV heads) ----
+    write_th = sum(wl.ctx_lens) * wl.n_kv_heads
+    write_gbs = write_th * WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme] / st.write_call_s / 1e9
 
     # ---- gate summary ---------------------------------------------------------
     kept = st.n_kept.cpu().tolist()
@@ -303,8 +310,10 @@ def run_ours(args, rank, world, local):
                      "frac_of_nominal_8tbs": achieved / 8000.0,
                      "peak_source": "MEASURED_PEAKS.json hbm_gbs (measured copy)" if peaks else "fallback 6.8 TB/s",
                      "algorithmic_bytes_per_launch": algo_bytes},
-        "witness_write": {"gbs": write_gbs, "token_heads_per_s": write_th / st.prefill_write_s,
-                          "bytes_per_token_head": WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme]},
+        "witness_write": {"gbs": write_gbs, "token_heads_per_s": write_th / st.write_call_s,
+                          "ms_per_layer_prefill": st.write_call_s * 1e3, "token_heads_per_call": write_th,
+                          "bytes_per_token_head": WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme],
+                          "frac_of_peak": write_gbs / (_peaks() or {}).get("hbm_gbs", 6800.0)},
         "gate": coverage,
         "gpu_launches": st.launches_per_step() * args.steps,
         "device_status": status,

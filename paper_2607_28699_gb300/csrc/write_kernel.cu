@@ -12,20 +12,25 @@ namespace wc {
 
 namespace {
 
-// round-half-even of the exact real x/s + xi, clamped to [-127, 127].
-// k0 from an fp32 estimate is within 1 of the answer whenever |x/s| < 2^21;
-// the FMA residuals x - s*(k0 +- 1/2 - xi) have exactly the sign of the
-// exact value (k0 +- 1/2 - xi is exact in fp32), which settles the rounding.
-__device__ __forceinline__ int dither_code(float x, float s, float inv_s, float xi) {
-    const float est = fmaf(x, inv_s, xi);
-    if (!(fabsf(est) < 200.0f)) return est > 0.0f ? 127 : -127;
-    float k = rintf(est);
+// Quantizer: code = round-half-even of the exact real x/s + xi, clamped to
+// [-127, 127].  The fp32 estimate est = fma(x, 1/s, xi) is within 3e-5 of the
+// exact value whenever |est| < 200 (1/s and the product each carry at most
+// 2^-24 relative error), so rint(est) is exact unless est lies within 1e-4 of
+// a half-integer (about 2 elements in 10^4).  Those are re-decided exactly in
+// a separate pass: the FMA residual x - s*(k +- 1/2 - xi) has exactly the
+// sign of the exact value, because k +- 1/2 - xi is exact in fp32.
+__device__ __forceinline__ float exact_round(float x, float s, float xi, float k) {
     const float up = fmaf(-s, k + 0.5f - xi, x);   // sign of x/s + xi - (k + 1/2)
     const float dn = fmaf(-s, k - 0.5f - xi, x);   // sign of x/s + xi - (k - 1/2)
-    const bool k_odd = (((int)k) & 1) != 0;
+    const bool k_odd = (__float_as_uint(k + 12582912.0f) & 1u) != 0u;
     if (up > 0.0f || (up == 0.0f && k_odd)) k += 1.0f;
     else if (dn < 0.0f || (dn == 0.0f && k_odd)) k -= 1.0f;
-    return max(-127, min(127, (int)k));
+    return fminf(127.0f, fmaxf(-127.0f, k));
+}
+
+// Low byte of the integer held (exactly) in float k, |k| < 2^22: two's complement.
+__device__ __forceinline__ uint32_t code_byte(float k) {
+    return __float_as_uint(k + 12582912.0f) & 0xFFu;    // 1.5 * 2^23 bias
 }
 
 template <int kScheme, int kBits>
@@ -76,40 +81,57 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
         s = __half2float(sh);
         const float inv_s = s > 0.0f ? __frcp_rn(s) : 0.0f;
 
-        // dither integers j for channels 16*sub .. 16*sub + 15
-        uint32_t jw[8];  // 16-bit lanes: j of channel (2i, 2i+1) in (lo, hi)
+        // dither words for channels 16*sub .. 16*sub + 15
         const uint32_t slot_u = (uint32_t)max(slot, 0);
         const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
+        uint32_t dw[8];
         if constexpr (kBits == 8) {
             const uint4 w = philox(slot_u, c1, (uint32_t)sub, (uint32_t)row, p.keys);
-            const uint32_t ww[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                jw[2 * i] = prmt(ww[i], 0u, 0x4140u);      // bytes 0,1 -> 16-bit lanes
-                jw[2 * i + 1] = prmt(ww[i], 0u, 0x4342u);  // bytes 2,3
-            }
+            dw[0] = w.x; dw[1] = w.y; dw[2] = w.z; dw[3] = w.w;
         } else {
 #pragma unroll
-            for (int g = 0; g < 2; ++g) {
-                const uint4 w = philox(slot_u, c1, (uint32_t)(2 * sub + g), (uint32_t)row, p.keys);
-                jw[4 * g + 0] = w.x & 0x03FF03FFu;
-                jw[4 * g + 1] = w.y & 0x03FF03FFu;
-                jw[4 * g + 2] = w.z & 0x03FF03FFu;
-                jw[4 * g + 3] = w.w & 0x03FF03FFu;
+            for (int gi = 0; gi < 2; ++gi) {
+                const uint4 w = philox(slot_u, c1, (uint32_t)(2 * sub + gi), (uint32_t)row, p.keys);
+                dw[4 * gi + 0] = w.x; dw[4 * gi + 1] = w.y; dw[4 * gi + 2] = w.z; dw[4 * gi + 3] = w.w;
             }
         }
-        constexpr float kInvN = 1.0f / (float)(1 << kBits);
+        uint32_t cb[16];
+        float xis[16], ks[16];
+        uint32_t near_tie = 0u;
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-            const uint32_t j = (jw[i >> 1] >> (16 * (i & 1))) & 0xFFFFu;
-            const float xi = ((float)j + 0.5f) * kInvN - 0.5f;   // exact
-            int k = 0;
-            if (s > 0.0f) k = dither_code(x[i], s, inv_s, xi);
-            r[i] = fmaf(s, (float)k - xi, -x[i]);                // x^ - x, one rounding
-            const uint32_t b = (uint32_t)(k & 0xFF);
-            if ((i & 3) == 0) codes[i >> 2] = b;
-            else codes[i >> 2] |= b << (8 * (i & 3));
+            // xi = (j + 1/2)/N - 1/2 built exactly from the bits of j:
+            // (1 + j/N) - (1 + (N-1)/(2N))
+            uint32_t mant;
+            if constexpr (kBits == 8) {
+                const int sh = 8 * (i & 3);              // byte i%4 of word i/4
+                mant = ((dw[i >> 2] >> sh) & 0xFFu) << 15;
+            } else {
+                const int sh = 16 * (i & 1);             // field i%2 of word i/2
+                mant = ((dw[i >> 1] >> sh) & 0x3FFu) << 13;
+            }
+            constexpr float kOff = 1.0f + (float)((1 << kBits) - 1) / (float)(2 << kBits);
+            const float xi = __uint_as_float(0x3F800000u | mant) - kOff;   // exact
+            const float est = fmaf(x[i], inv_s, xi);
+            const float kr = rintf(est);
+            if (fabsf(est - kr) > 0.4999f && fabsf(est) < 200.0f) near_tie |= 1u << i;
+            xis[i] = xi;
+            ks[i] = fminf(127.0f, fmaxf(-127.0f, kr));    // s = 0 gives x = 0, est = xi, k = 0
         }
+        if (__any_sync(0xffffffffu, near_tie != 0u)) {
+#pragma unroll
+            for (int i = 0; i < 16; ++i)
+                if (near_tie & (1u << i)) ks[i] = exact_round(x[i], s, xis[i], rintf(fmaf(x[i], inv_s, xis[i])));
+        }
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            r[i] = fmaf(s, ks[i] - xis[i], -x[i]);        // x^ - x, one rounding
+            cb[i] = code_byte(ks[i]);
+        }
+#pragma unroll
+        for (int i = 0; i < 4; ++i)
+            codes[i] = prmt(prmt(cb[4 * i], cb[4 * i + 1], 0x0040u), prmt(cb[4 * i + 2], cb[4 * i + 3], 0x0040u),
+                            0x5410u);
     } else {
         const uint32_t* hw = reinterpret_cast<const uint32_t*>(raw);
 #pragma unroll
