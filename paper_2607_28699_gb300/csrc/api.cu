@@ -127,7 +127,7 @@ size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_p
         fail(WC_ERR_CUDA, "no current CUDA device to size the workspace for");
         return 0;
     }
-    return wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms).total;
+    return wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms, desc->scheme, desc->dither_bits).total;
 }
 
 wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, const void* q,
@@ -150,7 +150,7 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
     if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
     int sms = 0;
     if (current_sm_count(&sms) != 0) return fail(WC_ERR_CUDA, "cannot query the current device");
-    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms);
+    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms, desc->scheme, desc->dither_bits);
     if (workspace_bytes < pl.total)
         return fail(WC_ERR_WORKSPACE, "workspace has %zu bytes, needs %zu", workspace_bytes, pl.total);
     uint8_t* ws = static_cast<uint8_t*>(workspace);
@@ -275,7 +275,7 @@ extern "C" wc_status wc_metered_decode_attention_noalloc(
     if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
     int sms = 0;
     if (current_sm_count(&sms) != 0) return fail(WC_ERR_CUDA, "cannot query the current device");
-    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms);
+    const wc::DecodePlan pl = wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms, desc->scheme, desc->dither_bits);
     if (pl.total > kNoAllocScratchBytes)
         return fail(WC_ERR_UNSUPPORTED,
                     "this decode needs %zu bytes of scratch but the built-in scratch holds %zu; "

@@ -527,6 +527,423 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     grid_dep_launch();
 }
 
+// ---------------------------------------------------------------------------
+// Warp-specialized variant for the dithered INT8 cache with 8-bit dither.
+//
+// One CTA per SM with 8 consumer / 8 producer warp pairs.  Producer warp w
+// serves consumer warp w: it issues the bulk copies of the consumer's pages
+// and regenerates the page's dither in registers (Philox4x32-10), storing it
+// as byte tiles j[token][channel] laid out exactly like the code tiles, so the
+// consumer reads dither words with the same 16-byte shared loads as codes.
+// The consumer runs the attention, bound and meter math with no Philox on its
+// path.  Per stage: `full` completes when the copies have landed and the
+// dither is written (two arrivals + the copy bytes); `empty` when the consumer
+// has released the stage.  All waits are bounded.
+// ---------------------------------------------------------------------------
+constexpr int kWsPairs = 8;
+constexpr int kWsThreads = 64 * kWsPairs;
+constexpr int kWsStages = 3;
+constexpr int kWsOffKd = kStageBytes;                  // K dither bytes [16][128]
+constexpr int kWsOffVd = kStageBytes + 2048;           // V dither bytes [16][128]
+constexpr int kWsOffHdr = kStageBytes + 4096;          // physical page (or -1)
+constexpr int kWsStageBytes = kStageBytes + 4096 + 16;
+constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsPairs * kWsStages * 16;
+
+__device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
+}
+
+__global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ DecodeParams p) {
+    extern __shared__ __align__(128) uint8_t smem[];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const bool producer = warp >= kWsPairs;
+    const int pw = producer ? warp - kWsPairs : warp;     // pair index
+    const int g = lane >> 2, c = lane & 3;
+    const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    const int G = p.group;
+    constexpr float kKappa = DitherConst<8>::kappa;
+
+    uint8_t* stages = smem + pw * kWsStages * kWsStageBytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kWsPairs * kWsStages * kWsStageBytes) + pw * 2 * kWsStages;
+    uint64_t* empty = full + kWsStages;
+    if (producer && lane == 0)
+        for (int s = 0; s < kWsStages; ++s) {
+            mbar_init(&full[s], 2);
+            mbar_init(&empty[s], 1);
+        }
+    fence_barrier_init();
+    __syncthreads();   // every barrier is initialised before any warp waits on it
+    grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
+
+    int ctx = __ldg(p.ctx_lens + b);
+    if (ctx < 0 || ctx > p.max_pages * kPage) {
+        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+        ctx = max(0, min(ctx, p.max_pages * kPage));
+    }
+    const int npages = (ctx + kPage - 1) / kPage;
+    const int p0 = split * p.pages_per_split;
+    const int p1 = min(p0 + p.pages_per_split, npages);
+    const int n_my = (p1 - p0 - pw > 0) ? (p1 - p0 - pw + kWsPairs - 1) / kWsPairs : 0;
+    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+
+    if (producer) {
+        const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
+        const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+        int issued = 0;
+        int phys_next = n_my > 0 ? __ldg(bt_row + p0 + pw) : -1;
+        for (int k = 0; k < n_my; ++k) {
+            const int s = k % kWsStages;
+            if (k >= kWsStages) {
+                const bool freed = mbar_wait_bounded(&empty[s], (uint32_t)(((k / kWsStages) - 1) & 1));
+                if (!__all_sync(0xffffffffu, freed)) {
+                    if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+                    break;
+                }
+            }
+            const int phys = phys_next;
+            if (k + 1 < n_my) phys_next = __ldg(bt_row + p0 + pw + kWsPairs * (k + 1));
+            const bool ok = phys >= 0 && phys < p.num_pages;
+            uint8_t* st = stages + s * kWsStageBytes;
+            if (lane == 0) {
+                *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
+                if (ok) {
+                    const size_t ph = (size_t)phys * p.num_kv_heads + h;
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)kStageBytes);
+                    bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, &full[s]);
+                    bulk_g2s(st + kOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, &full[s]);
+                    bulk_g2s(st + kOffKs, p.k_scale + ph * kPage, 32, &full[s]);
+                    bulk_g2s(st + kOffVs, p.v_scale + ph * kPage, 32, &full[s]);
+                    bulk_g2s(st + kOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
+                } else {
+                    atomicOr(p.status, WC_DEV_BAD_PAGE);
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+                }
+            }
+            issued = k + 1;
+            if (ok) {
+                // dither bytes j[token][channel]: one Philox call covers 16
+                // channels of one token (channel i = byte i%4 of word i/4)
+                const uint32_t slot0 = (uint32_t)phys * kPage;
+                uint4 dk[4], dv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x channel groups 2c, 2c+1
+                    dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
+#pragma unroll
+                for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
+                    dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    *reinterpret_cast<uint4*>(st + kWsOffKd + (g + 8 * (i >> 1)) * kHeadDim + 32 * c + 16 * (i & 1)) =
+                        dk[i];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    *reinterpret_cast<uint4*>(st + kWsOffVd + tv[j] * kHeadDim + 16 * g) = dv[j];
+            }
+            __syncwarp();
+            if (lane == 0)   // second arrival: dither tiles and header are written
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+        }
+        // copies still in flight must land before the CTA's smem is released
+        for (int k = max(0, issued - kWsStages); k < issued; ++k)
+            (void)mbar_wait_bounded(&full[k % kWsStages], (uint32_t)((k / kWsStages) & 1));
+        return;
+    }
+
+    // ---------------------------- consumer warps ------------------------------------
+    const bool row_valid = g < G;
+    const uint4* qsrc = reinterpret_cast<const uint4*>(
+        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
+        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+    }
+    float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[i]));
+        qsum += f.x + f.y;
+        part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));
+    }
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
+    qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+    float band_a, band_b;
+    if (p.rope_layout == WC_ROPE_HALF) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) part[i] += __shfl_xor_sync(0xffffffffu, part[i], 2);
+        const int src = (lane & ~3) | (c >> 1);
+        float v[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) v[i] = __shfl_sync(0xffffffffu, part[i], src);
+        band_a = (c & 1) ? v[2] : v[0];
+        band_b = (c & 1) ? v[3] : v[1];
+    } else {
+        band_a = part[0] + part[1];
+        band_b = part[2] + part[3];
+    }
+    uint32_t a_hi = 0, a_lo = 0;
+    if (row_valid) {
+        const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
+        const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+        a_hi = pack_h2(__half2float(h0), __half2float(h1));
+        a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
+    }
+    const float zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
+    const float zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
+
+    float m_run[2] = {-INFINITY, -INFINITY};
+    float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
+    float acc[8][4];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+    int lam_exp = INT_MIN;
+    const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+
+    for (int k = 0; k < n_my; ++k) {
+        const int s = k % kWsStages;
+        const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kWsStages) & 1));
+        if (!__all_sync(0xffffffffu, landed)) {
+            if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+            break;
+        }
+        const uint8_t* st = stages + s * kWsStageBytes;
+        const int lp = p0 + pw + kWsPairs * k;
+        if (*reinterpret_cast<const int*>(st + kWsOffHdr) >= 0) {
+            const int nvalid = min(kPage, ctx - lp * kPage);
+
+            // ---------------- QK: S[token][head] --------------------------------
+            float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+            for (int gp = 0; gp < 2; ++gp) {
+                const int o = 32 * c + 16 * gp;
+                const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + o);
+                const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + o);
+                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + g * kHeadDim + o);
+                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + (g + 8) * kHeadDim + o);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) {
+                    const int ks = 4 * gp + kk;
+                    const uint32_t xa = word_of(ka, kk) ^ 0x80808080u, xb = word_of(kb, kk) ^ 0x80808080u;
+                    const uint32_t A[4] = {s8x2_to_h2(xa, kSel01), s8x2_to_h2(xb, kSel01), s8x2_to_h2(xa, kSel23),
+                                           s8x2_to_h2(xb, kSel23)};
+                    mma16816(dc, A, qw[2 * ks], qw[2 * ks + 1]);
+                    const uint32_t ya = word_of(ja, kk), yb = word_of(jb, kk);
+                    const uint32_t H[4] = {h8(ya, kSel01), h8(yb, kSel01), h8(ya, kSel23), h8(yb, kSel23)};
+                    mma16816(dd, H, qw[2 * ks], qw[2 * ks + 1]);
+                }
+            }
+
+            // ---------------- logits, bound, softmax ------------------------------
+            float cb[4] = {0.f, 0.f, 0.f, 0.f};
+            {
+                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kOffW + (g * kBands + 2 * c) * 2);
+                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kOffW + ((g + 8) * kBands + 2 * c) * 2);
+                mma1688(cb, wa, wb, a_hi);
+                mma1688(cb, wa, wb, a_lo);
+            }
+            const __half* ksc = reinterpret_cast<const __half*>(st + kOffKs);
+            const __half* vsc = reinterpret_cast<const __half*>(st + kOffVs);
+            float sk[2] = {__half2float(ksc[g]), __half2float(ksc[g + 8])};
+            float sv[2] = {__half2float(vsc[g]), __half2float(vsc[g + 8])};
+            float y[4], P[4];
+            const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = i >> 1, e = i & 1;
+                const bool okr = r ? ok1 : ok0;
+                const float raw = dc[i] - dd[i] + (e ? zoff1 : zoff0);
+                y[i] = okr ? raw * (sk[r] * kRsdLog2e) : -INFINITY;
+                if (!okr) cb[i] = 0.f;                 // tail slots may hold any bits
+            }
+            if (!ok0) sv[0] = 0.f;
+            if (!ok1) sv[1] = 0.f;
+            float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+#pragma unroll
+            for (int o = 4; o < 32; o <<= 1) {
+                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+            }
+            const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
+            if (__any_sync(0xffffffffu, mv0 || mv1)) {
+                const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
+                const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
+                if (mv0) m_run[0] = mx0;
+                if (mv1) m_run[1] = mx1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    acc[mt][0] *= a0; acc[mt][2] *= a0;
+                    acc[mt][1] *= a1; acc[mt][3] *= a1;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = i >> 1, e = i & 1;
+                const float pe = fast_exp2(y[i] - m_run[e]);
+                l_part[e] += pe;
+                d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                P[i] = pe * sv[r];
+                spv_part[e] += P[i];
+            }
+            {
+                const float smax = fmaxf(sv[0], sv[1]);
+                const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
+                if (wmax > 0.f) {
+                    const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
+                    const int want = 6 - e;
+                    if (lam_exp == INT_MIN) {
+                        lam_exp = want;
+                    } else if (want < lam_exp) {
+                        const float f = pow2(want - lam_exp);
+#pragma unroll
+                        for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+                            for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
+                        lam_exp = want;
+                    }
+                }
+            }
+            uint32_t bp0, bp1, bl0, bl1;
+            {
+                const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
+                const float x0 = P[0] * lam, x1 = P[1] * lam, x2 = P[2] * lam, x3 = P[3] * lam;
+                const uint32_t h01 = pack_h2(x0, x1), h23 = pack_h2(x2, x3);
+                const float2 r01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
+                const float2 r23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
+                const uint32_t l01 = pack_h2(x0 - r01.x, x1 - r01.y), l23 = pack_h2(x2 - r23.x, x3 - r23.y);
+                bp0 = movmatrix_t(h01);
+                bp1 = movmatrix_t(h23);
+                bl0 = movmatrix_t(l01);
+                bl1 = movmatrix_t(l23);
+            }
+
+            // ---------------- PV: acc[dim][head] ------------------------------------
+            {
+                uint4 vq[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    vq[j] = *reinterpret_cast<const uint4*>(st + kOffV + tv[j] * kHeadDim + 16 * g);
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int wi = mt >> 1, pos = 2 * (mt & 1);
+                    uint32_t A[4];
+#pragma unroll
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
+                                                word_of(vq[2 * pr + 1], wi) ^ 0x80808080u, sel_interleave(pos));
+                        A[2 * pr] = s8x2_to_h2(X, kSel01);
+                        A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
+                    }
+                    mma16816(acc[mt], A, bp0, bp1);
+                    mma16816(acc[mt], A, bl0, bl1);
+                }
+            }
+            {
+                const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
+                const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
+                uint4 dv[4];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + tv[j] * kHeadDim + 16 * g);
+#pragma unroll
+                for (int mt = 0; mt < 8; ++mt) {
+                    const int wi = mt >> 1, pos = 2 * (mt & 1);
+                    uint32_t H[4];
+#pragma unroll
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
+                                                sel_interleave(pos));
+                        H[2 * pr] = h8(Y, kSel01);
+                        H[2 * pr + 1] = h8(Y, kSel23);
+                    }
+                    mma16816(acc[mt], H, bn0, bn1);
+                    mma16816(acc[mt], H, bm0, bm1);
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0)   // release the stage to the producer
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&empty[s])) : "memory");
+    }
+
+    // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1)
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
+            d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+            spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
+        }
+    const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
+
+    // ---- CTA merge over the consumer warps: one partial per CTA ------------------------
+    consumer_sync();   // all consumers are done with their stages (reused below)
+    float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
+    {
+        float* wb = mbuf + pw * kMaxGroup * kPartialStride;
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            float* row = wb + (2 * c + e) * kPartialStride + 16 * g;
+            const float add = kKappa * spv_part[e];
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                float4 v;
+                v.x = fmaf(acc[2 * q4][e], inv_lam, add);
+                v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
+                v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
+                v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
+                *reinterpret_cast<float4*>(row + 4 * q4) = v;
+            }
+            if (g == 0) {
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+            }
+        }
+    }
+    consumer_sync();
+    const size_t unit = (size_t)b * p.num_kv_heads + h;
+    float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
+    for (int idx = threadIdx.x; idx < G * 33; idx += 32 * kWsPairs) {
+        const int hh = idx / 33, ch = idx % 33;
+        float mw[kWsPairs];
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < kWsPairs; ++w) {
+            mw[w] = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
+            M = fmaxf(M, mw[w]);
+        }
+        float4 s4 = make_float4(0.f, 0.f, 0.f, 0.f);
+        const int col = (ch < 32) ? 4 * ch : kHeadDim + 1;
+#pragma unroll
+        for (int w = 0; w < kWsPairs; ++w) {
+            if (mw[w] == -INFINITY) continue;   // a warp without pages: its values are not read
+            const float wt = fast_exp2(mw[w] - M);
+            const float* src = mbuf + (w * kMaxGroup + hh) * kPartialStride + col;
+            if (ch < 32) {
+                const float4 v = *reinterpret_cast<const float4*>(src);
+                s4.x = fmaf(wt, v.x, s4.x); s4.y = fmaf(wt, v.y, s4.y);
+                s4.z = fmaf(wt, v.z, s4.z); s4.w = fmaf(wt, v.w, s4.w);
+            } else {
+                s4.x = fmaf(wt, src[0], s4.x);
+                s4.y = fmaf(wt, src[1], s4.y);
+            }
+        }
+        float* dst = part_out + hh * kPartialStride;
+        if (ch < 32) {
+            *reinterpret_cast<float4*>(dst + 4 * ch) = s4;
+        } else {
+            dst[kHeadDim] = M;
+            dst[kHeadDim + 1] = s4.x;
+            dst[kHeadDim + 2] = s4.y;
+        }
+    }
+    grid_dep_launch();
+}
+
 // Merge of the per-split partials of one (sequence, query head), 32 output
 // dims per CTA: out = sum_s w_s acc_s / sum_s w_s l_s with w_s = 2^(m_s - M),
 // D = sum_s w_s D_s / sum_s w_s l_s, meter_raw = D (D + 2) / 2 (§6.2.2: the
@@ -619,10 +1036,12 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
 
 }  // namespace
 
-DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms) {
+static bool use_ws(int scheme, int bits) { return scheme == WC_SCHEME_DITHER_INT8 && bits == 8; }
+
+DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits) {
     DecodePlan pl;
     const long units = (long)batch * num_kv_heads;
-    const long target = (long)num_sms * kMinBlocks;   // resident CTAs
+    const long target = (long)num_sms * (use_ws(scheme, bits) ? 1 : kMinBlocks);   // resident CTAs
     long pps = (max_pages * units + target - 1) / target;
     pps = std::max<long>(pps, 16);
     pps = std::min<long>(pps, std::max(max_pages, 1));
@@ -661,10 +1080,31 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
                       stream, p);
 }
 
+static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             kWsSmemBytes);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(decode_ws_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 (int)cudaSharedmemCarveoutMaxShared);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    dim3 grid(p.splits, p.num_kv_heads, p.batch);
+    cudaError_t e = launch_pdl(decode_ws_kernel, grid, dim3(kWsThreads), kWsSmemBytes, stream, p);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(merge_kernel, dim3(kHeadDim / 32, p.num_q_heads, p.batch), dim3(32 * kMergeWarps), 0,
+                      stream, p);
+}
+
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.batch == 0) return cudaSuccess;
     if (scheme == WC_SCHEME_FP8_E4M3) return launch_one<WC_SCHEME_FP8_E4M3, 8>(p, stream);
-    if (bits == 8) return launch_one<WC_SCHEME_DITHER_INT8, 8>(p, stream);
+    if (use_ws(scheme, bits)) return launch_ws(p, stream);
     return launch_one<WC_SCHEME_DITHER_INT8, 10>(p, stream);
 }
 

@@ -52,7 +52,7 @@ struct DecodePlan {
     size_t counters_off, partials_off, total;
 };
 
-DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms);
+DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits);
 
 // Launch `kernel` on `stream` as a programmatic dependent of the preceding work.
 template <typename Kernel, typename Params>

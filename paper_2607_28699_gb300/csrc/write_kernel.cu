@@ -14,11 +14,12 @@ namespace {
 
 // Quantizer: code = round-half-even of the exact real x/s + xi, clamped to
 // [-127, 127].  The fp32 estimate est = fma(x, 1/s, xi) is within 3e-5 of the
-// exact value whenever |est| < 200 (1/s and the product each carry at most
-// 2^-24 relative error), so rint(est) is exact unless est lies within 1e-4 of
-// a half-integer (about 2 elements in 10^4).  Those are re-decided exactly in
-// a separate pass: the FMA residual x - s*(k +- 1/2 - xi) has exactly the
-// sign of the exact value, because k +- 1/2 - xi is exact in fp32.
+// exact value whenever |est| <= 127.5 (1/s and the product each carry at most
+// 2^-24 relative error), so its rounding is exact unless est lies within 1e-4
+// of a half-integer (about 2 elements in 10^4); beyond +-127 the clamp
+// decides.  Near-ties are re-decided exactly in a separate pass: the FMA
+// residual x - s*(k +- 1/2 - xi) has exactly the sign of the exact value,
+// because k +- 1/2 - xi is exact in fp32.
 __device__ __forceinline__ float exact_round(float x, float s, float xi, float k) {
     const float up = fmaf(-s, k + 0.5f - xi, x);   // sign of x/s + xi - (k + 1/2)
     const float dn = fmaf(-s, k - 0.5f - xi, x);   // sign of x/s + xi - (k - 1/2)
@@ -112,16 +113,18 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
             }
             constexpr float kOff = 1.0f + (float)((1 << kBits) - 1) / (float)(2 << kBits);
             const float xi = __uint_as_float(0x3F800000u | mant) - kOff;   // exact
-            const float est = fmaf(x[i], inv_s, xi);
-            const float kr = rintf(est);
-            if (fabsf(est - kr) > 0.4999f && fabsf(est) < 200.0f) near_tie |= 1u << i;
+            // clamp first (values beyond +-127 saturate), then round to nearest
+            // even with the 1.5 * 2^23 bias; s = 0 gives x = 0, est = xi, k = 0
+            const float est = fminf(127.0f, fmaxf(-127.0f, fmaf(x[i], inv_s, xi)));
+            const float kr = (est + 12582912.0f) - 12582912.0f;
+            if (fabsf(est - kr) > 0.4999f) near_tie |= 1u << i;
             xis[i] = xi;
-            ks[i] = fminf(127.0f, fmaxf(-127.0f, kr));    // s = 0 gives x = 0, est = xi, k = 0
+            ks[i] = kr;
         }
         if (__any_sync(0xffffffffu, near_tie != 0u)) {
 #pragma unroll
             for (int i = 0; i < 16; ++i)
-                if (near_tie & (1u << i)) ks[i] = exact_round(x[i], s, xis[i], rintf(fmaf(x[i], inv_s, xis[i])));
+                if (near_tie & (1u << i)) ks[i] = exact_round(x[i], s, xis[i], ks[i]);
         }
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
