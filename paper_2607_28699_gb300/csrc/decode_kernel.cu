@@ -549,6 +549,11 @@ constexpr int kWsOffHdr = kStageBytes + 4096;          // physical page (or -1)
 constexpr int kWsStageBytes = kStageBytes + 4096 + 16;
 constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsPairs * kWsStages * 16;
 
+// Byte offset of 16-byte chunk q of token row t in a dither tile.  The chunk
+// index is XOR-swizzled with the row so that the producer's stores and the
+// consumer's loads of one warp instruction fall in distinct shared-memory banks.
+__device__ __forceinline__ int dither_chunk(int t, int q) { return t * kHeadDim + 16 * (q ^ (t & 7)); }
+
 __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
 }
@@ -632,12 +637,13 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
                     dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
 #pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    *reinterpret_cast<uint4*>(st + kWsOffKd + (g + 8 * (i >> 1)) * kHeadDim + 32 * c + 16 * (i & 1)) =
-                        dk[i];
+                for (int i = 0; i < 4; ++i) {
+                    const int t = g + 8 * (i >> 1);
+                    *reinterpret_cast<uint4*>(st + kWsOffKd + dither_chunk(t, 2 * c + (i & 1))) = dk[i];
+                }
 #pragma unroll
                 for (int j = 0; j < 4; ++j)
-                    *reinterpret_cast<uint4*>(st + kWsOffVd + tv[j] * kHeadDim + 16 * g) = dv[j];
+                    *reinterpret_cast<uint4*>(st + kWsOffVd + dither_chunk(tv[j], g)) = dv[j];
             }
             __syncwarp();
             if (lane == 0)   // second arrival: dither tiles and header are written
@@ -719,8 +725,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const int o = 32 * c + 16 * gp;
                 const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + o);
                 const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + o);
-                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + g * kHeadDim + o);
-                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + (g + 8) * kHeadDim + o);
+                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + dither_chunk(g, 2 * c + gp));
+                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + dither_chunk(g + 8, 2 * c + gp));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const int ks = 4 * gp + kk;
@@ -846,7 +852,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 uint4 dv[4];
 #pragma unroll
                 for (int j = 0; j < 4; ++j)
-                    dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + tv[j] * kHeadDim + 16 * g);
+                    dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + dither_chunk(tv[j], g));
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     const int wi = mt >> 1, pos = 2 * (mt & 1);
