@@ -19,8 +19,12 @@
 // Integer codes and the dither enter the tensor cores as exact fp16 values
 // (h' = 4 + j/256 for 8-bit, 1 + j/1024 for 10-bit dither; xi = h' - kappa),
 // so code - xi = code - h' + kappa is carried exactly to the fp32 accumulators.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
 #include <algorithm>
 #include <climits>
+#include <mutex>
 
 #include "wc_kernels.cuh"
 
@@ -89,6 +93,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     if (lane == 0)
         for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
     fence_barrier_init();
+    // the dependent merge may be scheduled now: it waits for this whole grid
+    // (griddepcontrol.wait) and launches only once every CTA here has started
+    grid_dep_launch();
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
     // Independent loads first: context length, this warp's first page-table
@@ -522,44 +529,81 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             dst[kHeadDim + 2] = s.y;
         }
     }
-    // the merge kernel (launched as a programmatic dependent) may start now;
-    // it waits for this whole grid before reading the partials
-    grid_dep_launch();
 }
 
 // ---------------------------------------------------------------------------
 // Warp-specialized variant for the dithered INT8 cache with 8-bit dither.
 //
 // One CTA per SM with 8 consumer / 8 producer warp pairs.  Producer warp w
-// serves consumer warp w: it issues the bulk copies of the consumer's pages
-// and regenerates the page's dither in registers (Philox4x32-10), storing it
-// as byte tiles j[token][channel] laid out exactly like the code tiles, so the
-// consumer reads dither words with the same 16-byte shared loads as codes.
-// The consumer runs the attention, bound and meter math with no Philox on its
-// path.  Per stage: `full` completes when the copies have landed and the
-// dither is written (two arrivals + the copy bytes); `empty` when the consumer
-// has released the stage.  All waits are bounded.
+// serves consumer warp w through a 3-stage ring: it issues the page's copies
+// (K and V code tiles by tensor-map TMA with the 128-byte swizzle, scales and
+// witness by bulk copy) and regenerates the page's dither (Philox4x32-10) in
+// registers, storing it as byte tiles j[token][channel] under the same
+// swizzle, so the consumer reads dither words with the same conflict-free
+// 16-byte shared loads as codes.  The consumer runs the attention, bound and
+// meter math with no Philox on its path.  Per stage:
+// `full` completes when the copies have landed and the dither tiles are
+// written (two arrivals + the copy bytes); `empty` when the consumer has
+// released it.  All waits are bounded.
 // ---------------------------------------------------------------------------
 constexpr int kWsPairs = 8;
 constexpr int kWsThreads = 64 * kWsPairs;
 constexpr int kWsStages = 3;
-constexpr int kWsOffKd = kStageBytes;                  // K dither bytes [16][128]
-constexpr int kWsOffVd = kStageBytes + 2048;           // V dither bytes [16][128]
-constexpr int kWsOffHdr = kStageBytes + 4096;          // physical page (or -1)
-constexpr int kWsStageBytes = kStageBytes + 4096 + 16;
-constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsPairs * kWsStages * 16;
+constexpr int kWsOffK = 0;          // K codes [16][128], swizzled (1024-aligned)
+constexpr int kWsOffV = 2048;       // V codes [16][128], swizzled
+constexpr int kWsOffKd = 4096;      // K dither bytes [16][128], swizzled
+constexpr int kWsOffVd = 6144;      // V dither bytes [16][128], swizzled
+constexpr int kWsOffKs = 8192;      // K scales [16] fp16
+constexpr int kWsOffVs = 8224;      // V scales [16] fp16
+constexpr int kWsOffW = 8256;       // witness [16][8] fp16
+constexpr int kWsOffHdr = 8512;     // physical page (or -1)
+constexpr int kWsStageBytes = 9216;
+static_assert(kWsOffHdr + 16 <= kWsStageBytes && kWsStageBytes % 1024 == 0, "stage layout");
+constexpr int kWsBarBytes = kWsPairs * kWsStages * 2 * 8;
+constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsBarBytes + 1024;   // + alignment slack
+static_assert(kWsSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
+static_assert(kWsPairs * kMaxGroup * kPartialStride * 4 <= kWsPairs * kWsStages * kWsStageBytes, "merge buffer");
 
-// Byte offset of 16-byte chunk q of token row t in a dither tile.  The chunk
-// index is XOR-swizzled with the row so that the producer's stores and the
-// consumer's loads of one warp instruction fall in distinct shared-memory banks.
-__device__ __forceinline__ int dither_chunk(int t, int q) { return t * kHeadDim + 16 * (q ^ (t & 7)); }
+struct WsParams {
+    CUtensorMap k_map;   // k_codes as [num_pages * Hkv][16][128] bytes, box = one page of one head
+    CUtensorMap v_map;
+    DecodeParams p;
+};
+
+// Byte offset of 16-byte chunk q of token row t in a tile written with the
+// 128-byte swizzle (tile 1024-byte aligned): chunk q of row t sits at chunk
+// q ^ (t & 7), so the 8 rows a warp touches per instruction hit distinct banks.
+__device__ __forceinline__ int swz(int t, int q) { return t * kHeadDim + 16 * (q ^ (t & 7)); }
+
+__device__ __forceinline__ void tma_page(void* dst, const CUtensorMap* map, int z, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(z), "r"(smem_addr(bar))
+        : "memory");
+}
 
 __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
 }
 
-__global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ DecodeParams p) {
-    extern __shared__ __align__(128) uint8_t smem[];
+// q fragment of the B operand (head g, channels 32c + 2i, +1 in word i).
+__device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h, int G, int g, int c,
+                                            uint32_t (&qw)[16]) {
+    const bool row_valid = g < G;
+    const uint4* qsrc = reinterpret_cast<const uint4*>(
+        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
+        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+    }
+}
+
+__global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
+    const DecodeParams& p = wp.p;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const bool producer = warp >= kWsPairs;
     const int pw = producer ? warp - kWsPairs : warp;     // pair index
@@ -578,24 +622,30 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         }
     fence_barrier_init();
     __syncthreads();   // every barrier is initialised before any warp waits on it
+    // the dependent merge may be scheduled now: it waits for this whole grid
+    // (griddepcontrol.wait), and it launches only once every CTA of this grid
+    // has started, so its CTAs never hold resources this grid still needs
+    grid_dep_launch();
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
+    const int p0 = split * p.pages_per_split;
+    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+    // this pair's first page-table entry, loaded alongside the context length
+    // (in bounds whatever the length; used only if the pair has pages)
+    int phys_next = (producer && p.max_pages > 0) ? __ldg(bt_row + min(p0 + pw, p.max_pages - 1)) : -1;
     int ctx = __ldg(p.ctx_lens + b);
     if (ctx < 0 || ctx > p.max_pages * kPage) {
         if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
         ctx = max(0, min(ctx, p.max_pages * kPage));
     }
     const int npages = (ctx + kPage - 1) / kPage;
-    const int p0 = split * p.pages_per_split;
     const int p1 = min(p0 + p.pages_per_split, npages);
     const int n_my = (p1 - p0 - pw > 0) ? (p1 - p0 - pw + kWsPairs - 1) / kWsPairs : 0;
-    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
 
     if (producer) {
         const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
         const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
         int issued = 0;
-        int phys_next = n_my > 0 ? __ldg(bt_row + p0 + pw) : -1;
         for (int k = 0; k < n_my; ++k) {
             const int s = k % kWsStages;
             if (k >= kWsStages) {
@@ -612,13 +662,14 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             if (lane == 0) {
                 *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
                 if (ok) {
-                    const size_t ph = (size_t)phys * p.num_kv_heads + h;
+                    const int z = phys * p.num_kv_heads + h;
+                    const size_t ph = (size_t)z;
                     mbar_arrive_expect_tx(&full[s], (uint32_t)kStageBytes);
-                    bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, &full[s]);
-                    bulk_g2s(st + kOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, &full[s]);
-                    bulk_g2s(st + kOffKs, p.k_scale + ph * kPage, 32, &full[s]);
-                    bulk_g2s(st + kOffVs, p.v_scale + ph * kPage, 32, &full[s]);
-                    bulk_g2s(st + kOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
+                    tma_page(st + kWsOffK, &wp.k_map, z, &full[s]);
+                    tma_page(st + kWsOffV, &wp.v_map, z, &full[s]);
+                    bulk_g2s(st + kWsOffKs, p.k_scale + ph * kPage, 32, &full[s]);
+                    bulk_g2s(st + kWsOffVs, p.v_scale + ph * kPage, 32, &full[s]);
+                    bulk_g2s(st + kWsOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
                 } else {
                     atomicOr(p.status, WC_DEV_BAD_PAGE);
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
@@ -637,13 +688,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
                     dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) {
-                    const int t = g + 8 * (i >> 1);
-                    *reinterpret_cast<uint4*>(st + kWsOffKd + dither_chunk(t, 2 * c + (i & 1))) = dk[i];
-                }
+                for (int i = 0; i < 4; ++i)
+                    *reinterpret_cast<uint4*>(st + kWsOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
 #pragma unroll
                 for (int j = 0; j < 4; ++j)
-                    *reinterpret_cast<uint4*>(st + kWsOffVd + dither_chunk(tv[j], g)) = dv[j];
+                    *reinterpret_cast<uint4*>(st + kWsOffVd + swz(tv[j], g)) = dv[j];
             }
             __syncwarp();
             if (lane == 0)   // second arrival: dither tiles and header are written
@@ -657,14 +706,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 
     // ---------------------------- consumer warps ------------------------------------
     const bool row_valid = g < G;
-    const uint4* qsrc = reinterpret_cast<const uint4*>(
-        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
-    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
-        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
-    }
+    uint32_t qw[16];
+    load_q_frag(p, b, h, G, g, c, qw);
     float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -718,15 +761,15 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         if (*reinterpret_cast<const int*>(st + kWsOffHdr) >= 0) {
             const int nvalid = min(kPage, ctx - lp * kPage);
 
-            // ---------------- QK: S[token][head] --------------------------------
+            // ---------------- QK: S[token][head] = code.q - h'.q -------------------
             float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {
-                const int o = 32 * c + 16 * gp;
-                const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + o);
-                const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + o);
-                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + dither_chunk(g, 2 * c + gp));
-                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + dither_chunk(g + 8, 2 * c + gp));
+                const int q16 = 2 * c + gp;   // 16-byte chunk: channels 32c + 16gp .. +15
+                const uint4 ka = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g, q16));
+                const uint4 kb = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g + 8, q16));
+                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g, q16));
+                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g + 8, q16));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const int ks = 4 * gp + kk;
@@ -743,13 +786,13 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             // ---------------- logits, bound, softmax ------------------------------
             float cb[4] = {0.f, 0.f, 0.f, 0.f};
             {
-                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kOffW + (g * kBands + 2 * c) * 2);
-                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kOffW + ((g + 8) * kBands + 2 * c) * 2);
+                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (g * kBands + 2 * c) * 2);
+                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kWsOffW + ((g + 8) * kBands + 2 * c) * 2);
                 mma1688(cb, wa, wb, a_hi);
                 mma1688(cb, wa, wb, a_lo);
             }
-            const __half* ksc = reinterpret_cast<const __half*>(st + kOffKs);
-            const __half* vsc = reinterpret_cast<const __half*>(st + kOffVs);
+            const __half* ksc = reinterpret_cast<const __half*>(st + kWsOffKs);
+            const __half* vsc = reinterpret_cast<const __half*>(st + kWsOffVs);
             float sk[2] = {__half2float(ksc[g]), __half2float(ksc[g + 8])};
             float sv[2] = {__half2float(vsc[g]), __half2float(vsc[g + 8])};
             float y[4], P[4];
@@ -829,8 +872,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             {
                 uint4 vq[4];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    vq[j] = *reinterpret_cast<const uint4*>(st + kOffV + tv[j] * kHeadDim + 16 * g);
+                for (int j = 0; j < 4; ++j) vq[j] = *reinterpret_cast<const uint4*>(st + kWsOffV + swz(tv[j], g));
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     const int wi = mt >> 1, pos = 2 * (mt & 1);
@@ -851,8 +893,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
                 uint4 dv[4];
 #pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + dither_chunk(tv[j], g));
+                for (int j = 0; j < 4; ++j) dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + swz(tv[j], g));
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     const int wi = mt >> 1, pos = 2 * (mt & 1);
@@ -947,7 +988,6 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             dst[kHeadDim + 2] = s4.y;
         }
     }
-    grid_dep_launch();
 }
 
 // Merge of the per-split partials of one (sequence, query head), 32 output
@@ -958,6 +998,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 constexpr int kMergeWarps = 8;
 
 __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_constant__ DecodeParams p) {
+    grid_dep_launch();   // the next kernel waits for this grid before reading its outputs
     grid_dep_wait();
     const int chunk = blockIdx.x, hq = blockIdx.y, b = blockIdx.z;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -1086,6 +1127,37 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
                       stream, p);
 }
 
+// cuTensorMapEncodeTiled through the runtime's driver entry point (the
+// library does not link the driver library itself).
+static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static std::once_flag once;
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+    });
+    return fn;
+}
+
+// One layer's code array [num_pages][Hkv][16][128] bytes as a 3-D tensor
+// (channel, slot, page * Hkv + head); a box is one page of one head, written
+// to shared memory with the 128-byte swizzle.
+static bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, int num_kv_heads) {
+    PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+    if (!enc) return false;
+    const cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)kPage, (cuuint64_t)num_pages * num_kv_heads};
+    const cuuint64_t strides[2] = {(cuuint64_t)kHeadDim, (cuuint64_t)kHeadDim * kPage};
+    const cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)kPage, 1};
+    const cuuint32_t elem[3] = {1, 1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<void*>(codes), dims, strides, box, elem,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;
     if (!configured) {
@@ -1100,8 +1172,13 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
+    WsParams wp;
+    wp.p = p;
+    if (!encode_page_map(&wp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
+        !encode_page_map(&wp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
+        return cudaErrorInvalidValue;
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_ws_kernel, grid, dim3(kWsThreads), kWsSmemBytes, stream, p);
+    cudaError_t e = launch_pdl(decode_ws_kernel, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
     return launch_pdl(merge_kernel, dim3(kHeadDim / 32, p.num_q_heads, p.batch), dim3(32 * kMergeWarps), 0,
                       stream, p);
