@@ -626,10 +626,31 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     // (griddepcontrol.wait), and it launches only once every CTA of this grid
     // has started, so its CTAs never hold resources this grid still needs
     grid_dep_launch();
-    grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
-
     const int p0 = split * p.pages_per_split;
     const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+    if (lane == 0 && p.max_pages > 0) {
+        // While the preceding kernel drains: warm L2 with this pair's first page
+        // and the CTA's query rows.  The context length and page-table entry read
+        // here may still be changing, so they serve only as prefetch addresses
+        // (clamped into the cache); the loads bypass L1, which therefore holds
+        // no copy that the reads after the wait could hit.
+        if (producer) {
+            const int ctx_hint = __ldcg(p.ctx_lens + b);
+            if (p0 + pw < p.max_pages && (p0 + pw) * kPage < ctx_hint) {
+                const int ph_hint = min(max(__ldcg(bt_row + p0 + pw), 0), p.num_pages - 1);
+                const size_t z = (size_t)ph_hint * p.num_kv_heads + h;
+                bulk_prefetch_l2(p.k_codes + z * (kPage * kHeadDim), kPage * kHeadDim);
+                bulk_prefetch_l2(p.v_codes + z * (kPage * kHeadDim), kPage * kHeadDim);
+                bulk_prefetch_l2(p.k_scale + z * kPage, 32);
+                bulk_prefetch_l2(p.v_scale + z * kPage, 32);
+                bulk_prefetch_l2(p.k_witness + z * (kPage * kBands), 256);
+            }
+        } else if (pw == 0) {
+            bulk_prefetch_l2(p.q + ((size_t)b * p.num_q_heads + (size_t)h * G) * kHeadDim, G * kHeadDim * 2);
+        }
+    }
+    grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
+
     // this pair's first page-table entry, loaded alongside the context length
     // (in bounds whatever the length; used only if the pair has pages)
     int phys_next = (producer && p.max_pages > 0) ? __ldg(bt_row + min(p0 + pw, p.max_pages - 1)) : -1;
@@ -1101,6 +1122,33 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
     return pl;
 }
 
+// The merge is launched early (programmatic dependent) and its CTAs become
+// resident on the SMs the decode grid frees first.  When the merge grid fits
+// in one wave, each CTA also reserves more than half of an SM's shared memory
+// (unused), so no two share an SM and the merge runs spread over the GPU
+// instead of packed onto the first few SMs to free up.
+constexpr int kMergeSpreadSmem = 118784;
+
+static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
+    static std::once_flag once;
+    static int num_sms = 0;   // 0: the spread request is not used
+    std::call_once(once, [] {
+        int dev = 0, n = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+            cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSpreadSmem) ==
+                cudaSuccess)
+            num_sms = n;
+        (void)cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                   (int)cudaSharedmemCarveoutMaxShared);
+        (void)cudaGetLastError();   // a refused hint leaves no sticky error behind
+    });
+    const dim3 grid(kHeadDim / 32, p.num_q_heads, p.batch);
+    const long ctas = (long)grid.x * grid.y * grid.z;
+    const size_t smem = (num_sms > 0 && ctas <= num_sms) ? kMergeSpreadSmem : 0;
+    return launch_pdl(merge_kernel, grid, dim3(32 * kMergeWarps), smem, stream, p);
+}
+
 template <int kScheme, int kBits>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;   // per process; the attributes are per function
@@ -1113,9 +1161,6 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
         e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 (int)cudaSharedmemCarveoutMaxShared);
-        if (e != cudaSuccess) return e;
         configured = true;
     }
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
@@ -1123,8 +1168,7 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     if (e != cudaSuccess) return e;
     // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
-    return launch_pdl(merge_kernel, dim3(kHeadDim / 32, p.num_q_heads, p.batch), dim3(32 * kMergeWarps), 0,
-                      stream, p);
+    return launch_merge(p, stream);
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (the
@@ -1167,9 +1211,6 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
         e = cudaFuncSetAttribute(decode_ws_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 (int)cudaSharedmemCarveoutMaxShared);
-        if (e != cudaSuccess) return e;
         configured = true;
     }
     WsParams wp;
@@ -1180,8 +1221,7 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
     cudaError_t e = launch_pdl(decode_ws_kernel, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
-    return launch_pdl(merge_kernel, dim3(kHeadDim / 32, p.num_q_heads, p.batch), dim3(32 * kMergeWarps), 0,
-                      stream, p);
+    return launch_merge(p, stream);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
