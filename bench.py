@@ -304,7 +304,8 @@ def run_ours(args, rank, world, local):
                    "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step > 129 MB L2; no flush"},
         "hbm_gbs_step": step_gbs,
         "decode_call_ms": dec_avg_ms,
-        "roofline": {"kernel": "decode_kernel + merge_kernel (one metered_decode_attention call)",
+        "roofline": {"kernel": ("decode_ws_kernel" if wl.scheme == 0 and args.dither_bits == 8 else "decode_kernel")
+                               + " + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "traffic": _traffic(wl.name),
                      "frac_of_nominal_8tbs": achieved / 8000.0,
@@ -388,7 +389,7 @@ def _oracle_sample(wl, budget_s, seed_layer=0):
     sm = W.slot_mapping(wl, bt)
     done_tokens, spent, layers = 0, 0.0, 0
     seqs = min(wl.batch, 2)
-    while spent < budget_s and layers < wl.n_layers:
+    while layers == 0 or (spent < budget_s and layers < wl.n_layers):   # at least one layer
         layer = (seed_layer + layers) % wl.n_layers
         k, v = W.layer_kv(wl, layer, seq_range=(0, seqs))
         q = W.layer_queries(wl, layer)
