@@ -2,10 +2,11 @@
 // K band-norm residual witness (§6.2.1 write kernel; §4.1 Eq. witness;
 // §4.2 subtractive dither).
 //
-// One warp handles two (token, KV head) units.  Lanes 8r .. 8r+7 own row r of
-// {K unit0, V unit0, K unit1, V unit1}; each lane owns 16 consecutive
-// channels, so it loads 32 B of fp16, stores 16 B of codes, and (for the
-// dither scheme) consumes exactly one Philox4x32-10 call per 16 channels.
+// A CTA of 4 warps handles eight (token, KV head) units: warps 0 and 2 the K
+// rows, warps 1 and 3 the V rows, 8 lanes per row.  Each lane owns 16
+// consecutive channels, so it loads 32 B of fp16, stores 16 B of codes, and
+// (for the dither scheme) consumes exactly one Philox4x32-10 call per 16
+// channels.
 #include "wc_kernels.cuh"
 
 namespace wc {
@@ -29,30 +30,17 @@ __device__ __forceinline__ float exact_round(float x, float s, float xi, float k
     return fminf(127.0f, fmaxf(-127.0f, k));
 }
 
-// Low byte of the integer held (exactly) in float k, |k| < 2^22: two's complement.
-__device__ __forceinline__ uint32_t code_byte(float k) {
-    return __float_as_uint(k + 12582912.0f) & 0xFFu;    // 1.5 * 2^23 bias
-}
+// Rounding bias 1.5 * 2^23: for |k| < 2^22, t = k + kBias holds k exactly and
+// the low byte of its bits is k's two's-complement byte.
+constexpr float kBias = 12582912.0f;
 
+// Dither word byte (i % 4) placed as the float 1 + j/2^15 (bits 0x3F80jj00).
+__device__ __forceinline__ uint32_t xi_sel(int i) { return 0x7604u | ((uint32_t)(i & 3) << 4); }
+
+// One row (K or V) of one (token, KV head): 8 lanes, 16 channels each.
 template <int kScheme, int kBits>
-__global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ WriteParams p) {
-    grid_dep_wait();      // inputs may come from the preceding kernel
-    grid_dep_launch();    // a dependent decode waits for this whole grid anyway
-    const int lane = threadIdx.x & 31;
-    const int unit = (blockIdx.x * 4 + (threadIdx.x >> 5)) * 2 + (lane >> 4);  // token*Hkv + h
-    const int row = (lane >> 3) & 1;                                             // 0 = K, 1 = V
-    const int sub = lane & 7;                                                    // 16-channel chunk
-    const bool live_unit = unit < p.n_tok * p.num_kv_heads;
-    const int tok = live_unit ? unit / p.num_kv_heads : 0;
-    const int h = live_unit ? unit % p.num_kv_heads : 0;
-    const int slot = live_unit ? __ldg(p.slot_mapping + tok) : -1;
-    // the row loads do not depend on the slot: issue them alongside its load
-    const __half* src = (row == 0 ? p.k : p.v) + ((size_t)tok * p.num_kv_heads + h) * kHeadDim + sub * 16;
-    uint4 raw[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)};
-    if (live_unit) {
-        raw[0] = __ldg(reinterpret_cast<const uint4*>(src));
-        raw[1] = __ldg(reinterpret_cast<const uint4*>(src) + 1);
-    }
+__device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2], int slot, bool live_unit, int h,
+                                          int row, int sub) {
     const bool bad = slot >= p.num_pages * kPage;
     const bool active = live_unit && slot >= 0 && !bad;
     if (live_unit && bad && sub == 0 && row == 0 && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_SLOT);
@@ -69,7 +57,7 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
     }
 
     uint32_t codes[4];
-    float r[16];
+    float lo = 0.0f, hi = 0.0f;   // K rows: squared residual sums over dims 16*sub + [0,8), + [8,16)
     float s = 0.0f;
     if constexpr (kScheme == WC_SCHEME_DITHER_INT8) {
         float amax = 0.0f;
@@ -96,44 +84,55 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
                 dw[4 * gi + 0] = w.x; dw[4 * gi + 1] = w.y; dw[4 * gi + 2] = w.z; dw[4 * gi + 3] = w.w;
             }
         }
-        uint32_t cb[16];
-        float xis[16], ks[16];
+        // With s a normal fp16 (or 0), |x| <= amax <= 126.5 s (1 + 2^-11), so
+        // |x/s + xi| < 127.06 and the clamp to [-127, 127] cannot bind; only rows
+        // whose scale fell into the fp16 subnormals need it.
+        const bool need_clamp = !__all_sync(0xffffffffu, s == 0.0f || s >= 6.103515625e-05f);
+        // xi = (j + 1/2)/N - 1/2 built exactly from the bits of j (recomputed
+        // where needed rather than held in registers)
+        auto xi_of = [&](int i) -> float {
+            if constexpr (kBits == 8) {
+                // 1 + j/2^15 from one byte permute; 128 (1 + j/2^15) - (128 + 255/512)
+                // = (j + 1/2)/256 - 1/2 is exact in one fma
+                const float f = __uint_as_float(prmt(dw[i >> 2], 0x3F800000u, xi_sel(i)));
+                return fmaf(f, 128.0f, -128.498046875f);
+            } else {
+                const int sh = 16 * (i & 1);             // field i%2 of word i/2
+                const uint32_t mant = ((dw[i >> 1] >> sh) & 0x3FFu) << 13;
+                constexpr float kOff = 1.0f + 1023.0f / 2048.0f;
+                return __uint_as_float(0x3F800000u | mant) - kOff;
+            }
+        };
+        uint32_t tb[16];   // bits of t = k + kBias: the low byte is the code
         uint32_t near_tie = 0u;
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-            // xi = (j + 1/2)/N - 1/2 built exactly from the bits of j:
-            // (1 + j/N) - (1 + (N-1)/(2N))
-            uint32_t mant;
-            if constexpr (kBits == 8) {
-                const int sh = 8 * (i & 3);              // byte i%4 of word i/4
-                mant = ((dw[i >> 2] >> sh) & 0xFFu) << 15;
-            } else {
-                const int sh = 16 * (i & 1);             // field i%2 of word i/2
-                mant = ((dw[i >> 1] >> sh) & 0x3FFu) << 13;
-            }
-            constexpr float kOff = 1.0f + (float)((1 << kBits) - 1) / (float)(2 << kBits);
-            const float xi = __uint_as_float(0x3F800000u | mant) - kOff;   // exact
-            // clamp first (values beyond +-127 saturate), then round to nearest
-            // even with the 1.5 * 2^23 bias; s = 0 gives x = 0, est = xi, k = 0
-            const float est = fminf(127.0f, fmaxf(-127.0f, fmaf(x[i], inv_s, xi)));
-            const float kr = (est + 12582912.0f) - 12582912.0f;
-            if (fabsf(est - kr) > 0.4999f) near_tie |= 1u << i;
-            xis[i] = xi;
-            ks[i] = kr;
+            const float xi = xi_of(i);
+            // round to nearest even with the 1.5 * 2^23 bias; s = 0 gives x = 0,
+            // est = xi, k = 0
+            float est = fmaf(x[i], inv_s, xi);
+            if (need_clamp) est = fminf(127.0f, fmaxf(-127.0f, est));
+            const float t = est + kBias;
+            if (fabsf(est - (t - kBias)) > 0.4999f) near_tie |= 1u << i;
+            tb[i] = __float_as_uint(t);
         }
         if (__any_sync(0xffffffffu, near_tie != 0u)) {
 #pragma unroll
             for (int i = 0; i < 16; ++i)
-                if (near_tie & (1u << i)) ks[i] = exact_round(x[i], s, xis[i], ks[i]);
+                if (near_tie & (1u << i))
+                    tb[i] = __float_as_uint(exact_round(x[i], s, xi_of(i), __uint_as_float(tb[i]) - kBias) + kBias);
         }
+        if (row == 0) {
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            r[i] = fmaf(s, ks[i] - xis[i], -x[i]);        // x^ - x, one rounding
-            cb[i] = code_byte(ks[i]);
+            for (int i = 0; i < 16; ++i) {
+                const float r = fmaf(s, (__uint_as_float(tb[i]) - kBias) - xi_of(i), -x[i]);   // x^ - x, one rounding
+                if (i < 8) lo = fmaf(r, r, lo);
+                else hi = fmaf(r, r, hi);
+            }
         }
 #pragma unroll
         for (int i = 0; i < 4; ++i)
-            codes[i] = prmt(prmt(cb[4 * i], cb[4 * i + 1], 0x0040u), prmt(cb[4 * i + 2], cb[4 * i + 3], 0x0040u),
+            codes[i] = prmt(prmt(tb[4 * i], tb[4 * i + 1], 0x0040u), prmt(tb[4 * i + 2], tb[4 * i + 3], 0x0040u),
                             0x5410u);
     } else {
         const uint32_t* hw = reinterpret_cast<const uint32_t*>(raw);
@@ -144,10 +143,13 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
             const uint32_t cc = (uint32_t)c2;   // low half -> low byte
             if ((i & 1) == 0) codes[i >> 1] = cc;
             else codes[i >> 1] |= cc << 16;
-            const uint32_t back = e4m3x2_to_h2(cc);
-            const float2 xr = __half22float2(*reinterpret_cast<const __half2*>(&back));
-            r[2 * i] = xr.x - x[2 * i];
-            r[2 * i + 1] = xr.y - x[2 * i + 1];
+            if (row == 0) {
+                const uint32_t back = e4m3x2_to_h2(cc);
+                const float2 xr = __half22float2(*reinterpret_cast<const __half2*>(&back));
+                const float r0 = xr.x - x[2 * i], r1 = xr.y - x[2 * i + 1];
+                if (i < 4) lo = fmaf(r1, r1, fmaf(r0, r0, lo));
+                else hi = fmaf(r1, r1, fmaf(r0, r0, hi));
+            }
         }
     }
 
@@ -161,16 +163,12 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
             if (sub == 0) (row == 0 ? p.k_scale : p.v_scale)[rowidx] = __float2half_rn(s);
         }
     }
+    if (row != 0) return;   // warp-uniform
 
-    // ---- witness (K rows only) --------------------------------------------
-    float lo = 0.0f, hi = 0.0f;   // sums over dims 16*sub + [0,8) and + [8,16)
-#pragma unroll
-    for (int i = 0; i < 8; ++i) lo = fmaf(r[i], r[i], lo);
-#pragma unroll
-    for (int i = 8; i < 16; ++i) hi = fmaf(r[i], r[i], hi);
+    // ---- witness (K warps) --------------------------------------------------
     const float lo_p = __shfl_xor_sync(0xffffffffu, lo, 4);
     const float hi_p = __shfl_xor_sync(0xffffffffu, hi, 4);
-    if (active && row == 0) {
+    if (active) {
         // fp32 sums carry < 2^-20 relative error; inflate by that margin
         // before rounding up so the stored witness never under-states.
         constexpr float kMargin = 1.0f + 1.0f / (1 << 19);
@@ -190,17 +188,77 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
     }
 }
 
+
+// Tasks of 4 tokens per warp whose loads are all issued before any is used:
+// more bytes in flight per SM (the kernel is otherwise bound by load latency).
+constexpr int kWriteTasks = 2;
+constexpr int kWriteUnitsPerCta = 2 * 4 * kWriteTasks;   // two warps per row type
+constexpr int kPerHeadMinTokens = 16;                     // per-head grid from this many tokens on
+
+// Two ways of cutting the units (token, KV head) into 4-unit tasks:
+//  kPerHead: grid (token groups, Hkv), a task = 4 consecutive tokens of one
+//            head, so a warp's code, scale and witness stores are contiguous
+//            runs of consecutive slots (prefill);
+//  else:     one index over units u = token * Hkv + h, a task = 4 consecutive
+//            units, so a one-token write of up to 8 KV heads is a single CTA
+//            (decode steps, where every SM the next decode needs counts).
+template <int kScheme, int kBits, bool kPerHead>
+__global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ WriteParams p) {
+    grid_dep_launch();    // a dependent decode may be scheduled now: it waits for this whole grid
+    grid_dep_wait();      // inputs may come from the preceding kernel
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    // Warps 0, 2 take the K rows and warps 1, 3 the V rows of the same units,
+    // so the residual and witness work stays in whole warps; lanes 8i .. 8i+7
+    // own unit i of a 4-unit task.
+    const int row = warp & 1;                                                  // 0 = K, 1 = V
+    const int sub = lane & 7;                                                  // 16-channel chunk
+    const int first = (blockIdx.x * 2 + (warp >> 1)) * (4 * kWriteTasks) + (lane >> 3);
+    const int n_first = kPerHead ? p.n_tok : p.n_tok * p.num_kv_heads;
+    bool live[kWriteTasks];
+    int slot[kWriteTasks], hs[kWriteTasks];
+    uint4 raw[kWriteTasks][2];
+#pragma unroll
+    for (int t = 0; t < kWriteTasks; ++t) {
+        const int idx = first + 4 * t;   // a token (kPerHead) or a unit
+        live[t] = idx < n_first;
+        int tok = 0, h = 0;
+        if (live[t]) {
+            if (kPerHead) {
+                tok = idx;
+                h = blockIdx.y;
+            } else {
+                tok = idx / p.num_kv_heads;
+                h = idx - tok * p.num_kv_heads;
+            }
+        }
+        hs[t] = h;
+        slot[t] = live[t] ? __ldg(p.slot_mapping + tok) : -1;
+        raw[t][0] = raw[t][1] = make_uint4(0, 0, 0, 0);
+        if (live[t]) {
+            const uint4* src = reinterpret_cast<const uint4*>(
+                (row == 0 ? p.k : p.v) + ((size_t)tok * p.num_kv_heads + h) * kHeadDim + sub * 16);
+            raw[t][0] = __ldg(src);
+            raw[t][1] = __ldg(src + 1);
+        }
+    }
+#pragma unroll
+    for (int t = 0; t < kWriteTasks; ++t)
+        if (__any_sync(0xffffffffu, live[t]))   // warp-uniform: a task past the end is skipped whole
+            write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub);
+}
+
 }  // namespace
 
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream) {
-    const int units = p.n_tok * p.num_kv_heads;
-    const int blocks = (units + 7) / 8;
-    if (blocks == 0) return cudaSuccess;
+    if (p.n_tok == 0) return cudaSuccess;
     static bool configured = false;   // same carveout as the decode kernels: no L1/shared reconfiguration
     if (!configured) {
-        const void* fns[3] = {(const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8>,
-                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8>,
-                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10>};
+        const void* fns[6] = {(const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8, false>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8, false>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10, false>,
+                              (const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8, true>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8, true>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10, true>};
         for (const void* f : fns) {
             cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
                                                  (int)cudaSharedmemCarveoutMaxShared);
@@ -208,10 +266,17 @@ cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_
         }
         configured = true;
     }
+    const bool per_head = p.n_tok >= kPerHeadMinTokens;
+    const dim3 grid = per_head ? dim3((p.n_tok + kWriteUnitsPerCta - 1) / kWriteUnitsPerCta, p.num_kv_heads)
+                               : dim3((p.n_tok * p.num_kv_heads + kWriteUnitsPerCta - 1) / kWriteUnitsPerCta);
+    auto go = [&](auto kernel) { return launch_pdl(kernel, grid, dim3(128), 0, stream, p); };
     if (scheme == WC_SCHEME_FP8_E4M3)
-        return launch_pdl(write_kernel<WC_SCHEME_FP8_E4M3, 8>, dim3(blocks), dim3(128), 0, stream, p);
-    if (bits == 8) return launch_pdl(write_kernel<WC_SCHEME_DITHER_INT8, 8>, dim3(blocks), dim3(128), 0, stream, p);
-    return launch_pdl(write_kernel<WC_SCHEME_DITHER_INT8, 10>, dim3(blocks), dim3(128), 0, stream, p);
+        return per_head ? go(write_kernel<WC_SCHEME_FP8_E4M3, 8, true>) : go(write_kernel<WC_SCHEME_FP8_E4M3, 8, false>);
+    if (bits == 8)
+        return per_head ? go(write_kernel<WC_SCHEME_DITHER_INT8, 8, true>)
+                        : go(write_kernel<WC_SCHEME_DITHER_INT8, 8, false>);
+    return per_head ? go(write_kernel<WC_SCHEME_DITHER_INT8, 10, true>)
+                    : go(write_kernel<WC_SCHEME_DITHER_INT8, 10, false>);
 }
 
 }  // namespace wc

@@ -79,6 +79,27 @@ def test_write_edge_rows():
         _compare(ocache, gpu_cache_to_numpy(gcache))
 
 
+@pytest.mark.parametrize("n_tok", [1, 5, 15, 16, 17])
+@pytest.mark.parametrize("hkv", [1, 4, 8])
+def test_write_small_batches_match_oracle(n_tok, hkv):
+    """Decode-step sized writes (one index over (token, head) units below 16
+    tokens, a per-head grid from 16 on), scattered slots, both schemes."""
+    import paper_2607_28699_gb300 as wc
+    rng = np.random.default_rng(100 * n_tok + hkv)
+    k = (rng.normal(size=(n_tok, hkv, 128)) * rng.lognormal(0, 0.5, size=128)).astype(np.float16)
+    v = (rng.normal(size=(n_tok, hkv, 128)) * rng.lognormal(0, 0.5, size=128)).astype(np.float16)
+    slots = rng.permutation(6 * 16)[:n_tok].astype(np.int32)
+    for scheme, bits in [(0, 8), (1, 8)]:
+        od, gd = descs(hkv, hkv, 6, scheme, bits, 0, seed=11)
+        ocache = OP.empty_cache(od)
+        OP.write_tokens(od, 3, k, v, slots, ocache)
+        gcache = wc.LayerCache.empty(gd)
+        wc.kv_quantize_witness(gd, 3, torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(),
+                               torch.from_numpy(slots).cuda(), gcache)
+        torch.cuda.synchronize()
+        _compare(ocache, gpu_cache_to_numpy(gcache))
+
+
 def test_write_bad_slot_sets_status_and_skips():
     import paper_2607_28699_gb300 as wc
     od, gd = descs(4, 2, 2, 0, 8, 0)
