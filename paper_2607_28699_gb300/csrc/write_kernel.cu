@@ -35,6 +35,27 @@ __device__ __forceinline__ float exact_round(float x, float s, float xi, float k
     return fminf(127.0f, fmaxf(-127.0f, k));
 }
 
+// Band norm for the witness, rounded up to fp16: the smallest fp16 h with
+// h * h >= S, S = sum inflated by 2^-18 (rounded up), which covers the fp32
+// accumulation error of the sum (< 2^-20 relative).  So h is never below the
+// exact norm rounded up and at most one fp16 step above it.  h * h is exact in
+// fp32 (11 significant bits), so one check on each side of the rounded-up
+// approximate root fixes it.
+__device__ __forceinline__ __half norm_up_fp16(float sum) {
+    const float S = __fmul_ru(sum, 1.0f + 1.0f / (1 << 18));
+    float y;
+    asm("sqrt.approx.f32 %0, %1;" : "=f"(y) : "f"(S));
+    unsigned short hb = __half_as_ushort(__float2half_ru(y));
+    const float hf = __half2float(__ushort_as_half(hb));
+    if (hf * hf < S) {
+        ++hb;
+    } else if (hb != 0) {
+        const float pf = __half2float(__ushort_as_half((unsigned short)(hb - 1)));
+        if (pf * pf >= S) --hb;
+    }
+    return __ushort_as_half(hb);
+}
+
 // Rounding bias 1.5 * 2^23: for |k| < 2^22, t = k + kBias holds k exactly and
 // the low byte of its bits is k's two's-complement byte.
 constexpr float kBias = 12582912.0f;
@@ -191,21 +212,15 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
     const float lo_p = __shfl_xor_sync(0xffffffffu, lo, 4);
     const float hi_p = __shfl_xor_sync(0xffffffffu, hi, 4);
     if (active) {
-        // fp32 sums carry < 2^-20 relative error; inflate by that margin
-        // before rounding up so the stored witness never under-states.
-        constexpr float kMargin = 1.0f + 1.0f / (1 << 19);
         __half* wdst = p.k_witness + rowidx * kBands;
         if (p.rope_layout == WC_ROPE_HALF) {
             // dims 16*sub..+7 and +8..+15 are the first (sub < 4) or second
             // (sub >= 4) halves of bands 2*(sub&3) and 2*(sub&3)+1.
-            if (sub < 4) {
-                const float b0 = __fmul_ru(__fsqrt_ru(lo + lo_p), kMargin);
-                const float b1 = __fmul_ru(__fsqrt_ru(hi + hi_p), kMargin);
-                const __half2 w2 = __halves2half2(__float2half_ru(b0), __float2half_ru(b1));
-                *reinterpret_cast<__half2*>(wdst + 2 * sub) = w2;
-            }
+            if (sub < 4)
+                *reinterpret_cast<__half2*>(wdst + 2 * sub) =
+                    __halves2half2(norm_up_fp16(lo + lo_p), norm_up_fp16(hi + hi_p));
         } else {
-            wdst[sub] = __float2half_ru(__fmul_ru(__fsqrt_ru(lo + hi), kMargin));
+            wdst[sub] = norm_up_fp16(lo + hi);
         }
     }
 }
