@@ -1106,15 +1106,34 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
 
 static bool use_ws(int scheme, int bits) { return scheme == WC_SCHEME_DITHER_INT8 && bits == 8; }
 
+// Split plan.  A CTA's 8 page streams (warps or warp pairs) each take every
+// 8th page of its split, so a split of P pages costs ceil(P / 8) page steps,
+// and a wave of resident CTAs adds a fixed prologue / epilogue of about one
+// and a half page steps.  The split count minimises
+//     waves * (ceil(pages_per_split / 8) + 1.5),   waves = ceil(CTAs / resident CTAs),
+// so a grid never spills a small remainder into an extra wave; splits keep at
+// least 8 pages (one per stream).  Ties go to fewer splits (less to merge).
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits) {
     DecodePlan pl;
     const long units = (long)batch * num_kv_heads;
-    const long target = (long)num_sms * (use_ws(scheme, bits) ? 1 : kMinBlocks);   // resident CTAs
-    long pps = (max_pages * units + target - 1) / target;
-    pps = std::max<long>(pps, 16);
-    pps = std::min<long>(pps, std::max(max_pages, 1));
-    pl.pages_per_split = (int)pps;
-    pl.splits = (int)std::max<long>(1, (max_pages + pps - 1) / pps);
+    const long slots = std::max<long>(1, (long)num_sms * (use_ws(scheme, bits) ? 1 : kMinBlocks));
+    constexpr long kStreams = 8;      // page streams per CTA
+    constexpr long kWaveCost2 = 3;    // per-wave fixed cost, in half page steps
+    const long max_splits = std::max<long>(1, std::min<long>(max_pages / kStreams, 4 * slots));
+    long best_pps = std::max(max_pages, 1), best_cost = -1;
+    for (long sp = 1; sp <= max_splits; ++sp) {
+        const long pps = (max_pages + sp - 1) / sp;
+        const long splits = (max_pages + pps - 1) / pps;
+        if (splits != sp) continue;   // same plan as a smaller split count
+        const long waves = (splits * units + slots - 1) / slots;
+        const long cost = waves * (2 * ((pps + kStreams - 1) / kStreams) + kWaveCost2);
+        if (best_cost < 0 || cost < best_cost) {
+            best_cost = cost;
+            best_pps = pps;
+        }
+    }
+    pl.pages_per_split = (int)best_pps;
+    pl.splits = (int)std::max<long>(1, (max_pages + best_pps - 1) / best_pps);
     auto align = [](size_t x) { return (x + 255) & ~(size_t)255; };
     pl.counters_off = 256;
     pl.partials_off = 256;
