@@ -535,7 +535,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 // Warp-specialized variant for the dithered INT8 cache with 8-bit dither.
 //
 // One CTA per SM with 8 consumer / 8 producer warp pairs.  Producer warp w
-// serves consumer warp w through a 3-stage ring: it issues the page's copies
+// serves consumer warp w through a 2-stage ring: it issues the page's copies
 // (K and V code tiles by tensor-map TMA with the 128-byte swizzle, scales and
 // witness by bulk copy) and regenerates the page's dither (Philox4x32-10) in
 // registers, storing it as byte tiles j[token][channel] under the same
@@ -548,7 +548,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 // ---------------------------------------------------------------------------
 constexpr int kWsPairs = 8;
 constexpr int kWsThreads = 64 * kWsPairs;
-constexpr int kWsStages = 3;
+constexpr int kWsStages = 2;
 constexpr int kWsOffK = 0;          // K codes [16][128], swizzled (1024-aligned)
 constexpr int kWsOffV = 2048;       // V codes [16][128], swizzled
 constexpr int kWsOffKd = 4096;      // K dither bytes [16][128], swizzled
