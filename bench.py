@@ -131,11 +131,20 @@ def barrier(world):
 
 
 def max_over_ranks(x, world):
+    """Largest value over the ranks (the slowest rank's time); the only
+    collective, outside the timed region."""
     if world == 1:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if torch.distributed.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return float(t.item())
+
+
+def rank_workload(config, seed, rank):
+    """Replicas: every rank runs the same workload shape on its own seeded
+    data (no data-path exchange; weak scaling)."""
+    return W.config(config, seed=seed + rank)
 
 
 # ---------------------------------------------------------------------------
@@ -230,7 +239,7 @@ def capture(fn):
 
 
 def run_ours(args, rank, world, local):
-    wl = W.config(args.config, seed=args.seed + rank)
+    wl = rank_workload(args.config, args.seed, rank)
     if args.layers:
         wl.n_layers = args.layers
     st = Setup(wl, dither_bits=args.dither_bits)
