@@ -20,6 +20,16 @@ numerically careful evaluation, "in the log domain").
 §4.1 Thm. "Sound black-box logit bound": |eps_t| = |q . r_t| / sqrt(d)
 <= (1/sqrt(d)) sum_b ||q_b|| w_{t,b} =: c_t.
 
+§4.2 Tier B (controlled quantizer, subtractive dither): Lemma "Uniform
+sub-Gaussian proxy" gives the logit error of token t the variance proxy
+varsigma_t^2 = (1/d) sum_c q_c^2 s_{c,t}^2 / 12, and with probability at
+least 1 - delta_loc jointly over the S tokens |eps_t| <= u_t =
+sqrt(2 varsigma_t^2 log(2S / delta_loc)); u_t then replaces c_t in the
+e-form meter.  Here the scale is one stored fp16 value per (token, KV head)
+(§6.2.2 per-token granularity), so varsigma_t^2 = ||q||^2 s_t^2 / (12 d).
+The guarantee is probabilistic and holds for non-adaptive queries (§4.2
+"Scope of the probabilistic guarantee").
+
 Gate (§6 meter-loop box; §4.3 certified vs risk-ranked): a (layer, head)
 falls back when its meter exceeds tau.  Reading: keep the compressed path
 iff meter_raw <= tau (so equality keeps, NaN falls back), evaluated in
@@ -86,6 +96,18 @@ def tier_a_bound(q, w, num_bands, rope_layout):
     qn = quantizer.band_norms(q, num_bands, rope_layout)          # [..., B]
     w = np.asarray(w, dtype=np.float64)
     return np.einsum("...b,...sb->...s", qn, w) / np.sqrt(d)
+
+
+def tier_b_bound(q, s, ctx_len, delta_loc):
+    """u_t = sqrt(2 varsigma_t^2 log(2 S / delta_loc)), varsigma_t^2 = ||q||^2 s_t^2 / (12 d).
+
+    q: [..., d] query; s: [..., S] stored K scales of the S tokens; returns [..., S].
+    """
+    q = np.asarray(q, dtype=np.float64)
+    d = q.shape[-1]
+    s = np.asarray(s, dtype=np.float64)
+    var = np.sum(q * q, axis=-1)[..., None] * s * s / (12.0 * d)
+    return np.sqrt(2.0 * var * np.log(2.0 * ctx_len / delta_loc))
 
 
 def logits(q, k):

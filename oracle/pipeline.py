@@ -116,20 +116,25 @@ def reconstruct(desc, layer, kv_head, slots, cache):
 
 
 def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
-                    k_exact=None, v_exact=None):
+                    k_exact=None, v_exact=None, delta_loc=None):
     """metered_decode_attention for one sequence: q16 [Hq, d] post-RoPE.
 
     Returns a dict with float64 ``out`` [Hq, d], ``meter``/``meter_raw``
     [Hq]; with the exact fp16 keys/values [S, Hkv, d] also ``tv`` [Hq]
     (the true TV between exact and compressed attention) and
-    ``out_exact`` [Hq, d].
+    ``out_exact`` [Hq, d]; with ``delta_loc`` (dithered INT8 only) also the
+    Tier-B meters ``meter_b``/``meter_b_raw`` [Hq] (§4.2).
     """
     G = desc.num_q_heads // desc.num_kv_heads
     d = desc.head_dim
     slots = slots_of(desc, block_table_row, ctx_len)
     res = {k: np.zeros((desc.num_q_heads, d)) for k in ("out", "out_exact")}
-    for k in ("meter", "meter_raw", "tv", "A"):
+    for k in ("meter", "meter_raw", "tv", "A", "meter_b", "meter_b_raw"):
         res[k] = np.zeros(desc.num_q_heads)
+    tier_b = delta_loc is not None
+    if tier_b and desc.scheme != SCHEME_DITHER_INT8:
+        raise ValueError("Tier B needs the dithered INT8 cache (a controlled quantizer)")
+    page, off = slots // desc.page_size, slots % desc.page_size
     for h in range(desc.num_kv_heads):
         khat, vhat, w = reconstruct(desc, layer, h, slots, cache)
         for g in range(G):
@@ -139,6 +144,9 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
             c = M.tier_a_bound(q, w, desc.num_bands, desc.rope_layout)
             res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.eform_meter(p_tilde, c)
             res["out"][hq] = M.attend(p_tilde, vhat)
+            if tier_b:
+                u = M.tier_b_bound(q, cache["k_scale"][page, h, off].astype(np.float64), ctx_len, delta_loc)
+                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
             if k_exact is not None:
                 p = M.softmax(M.logits(q, np.asarray(k_exact)[:ctx_len, h]))
                 res["tv"][hq] = M.total_variation(p, p_tilde)
