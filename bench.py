@@ -219,6 +219,21 @@ class Setup:
         for layer in range(self.wl.n_layers):
             self.decode(layer)
 
+    TIER_B_DELTA_REQ = 1e-2   # request-level budget, split over layers, query heads and one step
+
+    def decode_all_tier_b(self):
+        """The same calls with the Tier-B certificate as well (§4.2; dithered INT8 only)."""
+        wl = self.wl
+        if not hasattr(self, "meter_b"):
+            self.meter_b = torch.empty_like(self.meter)
+            self.meter_b_raw = torch.empty_like(self.raw)
+        delta_loc = self.TIER_B_DELTA_REQ / (wl.n_layers * wl.n_q_heads)
+        for layer in range(wl.n_layers):
+            self.wc.metered_decode_attention_tier_b(
+                self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer], self.ws, delta_loc,
+                out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
+                meter_b=self.meter_b[layer], meter_b_raw=self.meter_b_raw[layer])
+
     def launches_per_step(self):
         # per layer: write kernel, decode kernel, merge kernel; then one gate
         return 3 * self.wl.n_layers + 1
@@ -278,6 +293,24 @@ def run_ours(args, rank, world, local):
     torch.cuda.synchronize()
     dec_avg_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
 
+    # ---- the same calls with the Tier-B certificate too (its marginal cost) ----
+    tier_b = None
+    if wl.scheme == 0:
+        bgraph = capture(st.decode_all_tier_b)
+        for _ in range(args.warmup):
+            bgraph.replay()
+        torch.cuda.synchronize()
+        d0.record()
+        for _ in range(args.steps):
+            bgraph.replay()
+        d1.record()
+        torch.cuda.synchronize()
+        tb_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
+        mb = st.meter_b_raw.reshape(-1)
+        tier_b = {"decode_call_ms": tb_ms, "overhead_vs_tier_a": tb_ms / dec_avg_ms - 1.0,
+                  "delta_req": st.TIER_B_DELTA_REQ, "kept_frac_at_tau": float((mb <= st.tau).float().mean()),
+                  "meter_b_raw_median": float(mb.median())}
+
     kv_tokens_step = wl.kv_tokens
     value = kv_tokens_step * world / (ms / 1e3)
     algo_bytes = st.decode_bytes_per_launch()
@@ -313,6 +346,7 @@ def run_ours(args, rank, world, local):
                    "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step > 129 MB L2; no flush"},
         "hbm_gbs_step": step_gbs,
         "decode_call_ms": dec_avg_ms,
+        "tier_b": tier_b,
         "roofline": {"kernel": ("decode_ws_kernel" if wl.scheme == 0 and args.dither_bits == 8 else "decode_kernel")
                                + " + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

@@ -167,6 +167,37 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer,
                                       void* stream);
 
 /*
+ * Metered decode attention with the Tier-B sub-Gaussian certificate as well
+ * (§4.2, Lemma "Uniform sub-Gaussian proxy"; dithered INT8 cache only).
+ *
+ * Same computation, arguments and outputs as wc_metered_decode_attention,
+ * plus, for every sequence b and query head hq over its S = ctx_lens[b]
+ * tokens:
+ *   u_t             = sqrt(2 varsigma_t^2 log(2 S / delta_loc)),
+ *   varsigma_t^2    = ||q||^2 s_t^2 / (12 * 128)   (s_t the stored fp16 K scale),
+ *   meter_b_raw     = 1/2 (A_B^2 - 1), A_B = sum_t p~_t e^{u_t}  (+inf on overflow),
+ *   meter_b         = min(1, meter_b_raw).
+ * With probability at least 1 - delta_loc over the dither, |eps_t| <= u_t for
+ * all S tokens and then TV <= meter_b_raw; the guarantee assumes queries that
+ * do not depend on the stored dither (non-adaptive, §4.2 "Scope").  The
+ * request-level budget delta_loc = delta_req / (L * H * T) is the caller's.
+ *   delta_loc            in (0, 1), else WC_ERR_INVALID_ARG
+ *   meter_b, meter_b_raw [batch][Hq] fp32, device
+ * Returns WC_ERR_UNSUPPORTED for the fp8 scheme (no controlled quantizer).
+ */
+wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t layer,
+                                             const void* q, const int32_t* block_table,
+                                             int32_t max_pages, const int32_t* ctx_lens,
+                                             int32_t batch,
+                                             const void* k_codes, const void* v_codes,
+                                             const void* k_scale, const void* v_scale,
+                                             const void* k_witness, double delta_loc,
+                                             float* out, float* meter, float* meter_raw,
+                                             float* meter_b, float* meter_b_raw,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream);
+
+/*
  * Allocation-free metered decode.  The paper has no counterpart: this is a
  * deployment convenience for callers that cannot allocate device memory at
  * decode time (a runtime that pre-plans every buffer, code running inside an

@@ -31,6 +31,7 @@ ROPE_HALF = 0
 ROPE_INTERLEAVED = 1
 DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT = 1, 2, 4, 8
 EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
+           "wc_metered_decode_attention_tier_b", "wc_metered_decode_attention_noalloc",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -53,6 +54,10 @@ def _load():
     lib.wc_metered_decode_attention.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp,
                                                 vp, vp, vp, vp, ctypes.c_size_t, vp]
     lib.wc_metered_decode_attention.restype = ctypes.c_int
+    lib.wc_metered_decode_attention_tier_b.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp,
+                                                       ctypes.c_double, vp, vp, vp, vp, vp, vp, ctypes.c_size_t,
+                                                       vp]
+    lib.wc_metered_decode_attention_tier_b.restype = ctypes.c_int
     lib.wc_gate.argtypes = [vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]
     lib.wc_gate.restype = ctypes.c_int
     lib.wc_read_status.argtypes = [vp, i32, vp, vp]
@@ -195,6 +200,28 @@ def metered_decode_attention(desc: CacheDesc, layer: int, q: torch.Tensor, block
         _ptr(cache.k_witness), _ptr(out), _ptr(meter), _ptr(meter_raw), ws.ptr(), ws.nbytes,
         _stream(stream)))
     return out, meter, meter_raw
+
+
+def metered_decode_attention_tier_b(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
+                                    ctx_lens: torch.Tensor, cache: LayerCache, ws: Workspace, delta_loc: float,
+                                    out=None, meter=None, meter_raw=None, meter_b=None, meter_b_raw=None,
+                                    stream=None):
+    """``wc_metered_decode_attention_tier_b``; returns (out, meter, meter_raw, meter_b, meter_b_raw)."""
+    batch, max_pages = block_table.shape
+    dev = q.device
+    cells = (batch, desc.num_q_heads)
+    out = torch.empty(batch, desc.num_q_heads, desc.head_dim, dtype=torch.float32, device=dev) if out is None else out
+    meter = torch.empty(cells, dtype=torch.float32, device=dev) if meter is None else meter
+    meter_raw = torch.empty(cells, dtype=torch.float32, device=dev) if meter_raw is None else meter_raw
+    meter_b = torch.empty(cells, dtype=torch.float32, device=dev) if meter_b is None else meter_b
+    meter_b_raw = torch.empty(cells, dtype=torch.float32, device=dev) if meter_b_raw is None else meter_b_raw
+    d = desc.c()
+    _check(lib.wc_metered_decode_attention_tier_b(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), float(delta_loc), _ptr(out), _ptr(meter), _ptr(meter_raw), _ptr(meter_b),
+        _ptr(meter_b_raw), ws.ptr(), ws.nbytes, _stream(stream)))
+    return out, meter, meter_raw, meter_b, meter_b_raw
 
 
 def gate(meter_raw: torch.Tensor, group: int, tau: float, keep_q=None, keep_kv=None, n_kept=None,

@@ -1,4 +1,5 @@
 // extern "C" boundary: host-side argument checks and kernel launches.
+#include <cmath>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -130,13 +131,23 @@ size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_p
     return wc::plan_decode(batch, desc->num_kv_heads, max_pages, sms, desc->scheme, desc->dither_bits).total;
 }
 
-wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, const void* q,
-                                      const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
-                                      int32_t batch, const void* k_codes, const void* v_codes,
-                                      const void* k_scale, const void* v_scale, const void* k_witness,
-                                      float* out, float* meter, float* meter_raw, void* workspace,
-                                      size_t workspace_bytes, void* stream) {
+// Metered decode with a caller workspace; meter_b != NULL also asks for the
+// Tier-B meters (dithered INT8 only).
+static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                       const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                       int32_t batch, const void* k_codes, const void* v_codes,
+                                       const void* k_scale, const void* v_scale, const void* k_witness,
+                                       float* out, float* meter, float* meter_raw, float* meter_b,
+                                       float* meter_b_raw, double delta_loc, void* workspace,
+                                       size_t workspace_bytes, void* stream) {
     if (wc_status st = check_desc(desc)) return st;
+    if (meter_b || meter_b_raw) {
+        if (desc->scheme != WC_SCHEME_DITHER_INT8)
+            return fail(WC_ERR_UNSUPPORTED, "Tier B needs the dithered INT8 cache (a controlled quantizer)");
+        if (!meter_b || !meter_b_raw) return fail(WC_ERR_INVALID_ARG, "meter_b and meter_b_raw must not be NULL");
+        if (!(delta_loc > 0.0 && delta_loc < 1.0))
+            return fail(WC_ERR_INVALID_ARG, "delta_loc must be in (0, 1) (got %g)", delta_loc);
+    }
     if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
     if (batch < 0 || batch > 65535) return fail(WC_ERR_INVALID_ARG, "batch must be in [0, 65535] (got %d)", batch);
     if (max_pages < 1) return fail(WC_ERR_INVALID_ARG, "max_pages must be positive (got %d)", max_pages);
@@ -166,6 +177,9 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
     p.out = out;
     p.meter = meter;
     p.meter_raw = meter_raw;
+    p.meter_b = meter_b;
+    p.meter_b_raw = meter_b_raw;
+    p.tb_log_2_over_delta = meter_b ? (float)std::log(2.0 / delta_loc) : 0.0f;
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
@@ -182,6 +196,30 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
     p.keys = wc::make_philox_keys(desc->seed);
     cudaError_t e = wc::launch_decode(p, desc->scheme, desc->dither_bits, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? WC_OK : cuda_fail(e, "decode kernel launch");
+}
+
+wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                      const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                      int32_t batch, const void* k_codes, const void* v_codes,
+                                      const void* k_scale, const void* v_scale, const void* k_witness,
+                                      float* out, float* meter, float* meter_raw, void* workspace,
+                                      size_t workspace_bytes, void* stream) {
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, workspace,
+                                 workspace_bytes, stream);
+}
+
+wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                             const int32_t* block_table, int32_t max_pages,
+                                             const int32_t* ctx_lens, int32_t batch, const void* k_codes,
+                                             const void* v_codes, const void* k_scale, const void* v_scale,
+                                             const void* k_witness, double delta_loc, float* out, float* meter,
+                                             float* meter_raw, float* meter_b, float* meter_b_raw,
+                                             void* workspace, size_t workspace_bytes, void* stream) {
+    if (!meter_b || !meter_b_raw) return fail(WC_ERR_INVALID_ARG, "meter_b and meter_b_raw must not be NULL");
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, meter_b, meter_b_raw, delta_loc,
+                                 workspace, workspace_bytes, stream);
 }
 
 wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau, uint8_t* keep_q,
@@ -296,6 +334,9 @@ extern "C" wc_status wc_metered_decode_attention_noalloc(
     p.out = out;
     p.meter = meter;
     p.meter_raw = meter_raw;
+    p.meter_b = nullptr;
+    p.meter_b_raw = nullptr;
+    p.tb_log_2_over_delta = 0.0f;
     p.status = dev_status ? dev_status : reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);

@@ -79,7 +79,7 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
     return y;
 }
 
-template <int kScheme, int kBits>
+template <int kScheme, int kBits, bool kTierB>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecodeParams p) {
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -164,6 +164,18 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     }
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+    // Tier B (§4.2): u_t = alpha s_t with alpha = sqrt(2 log(2S/delta) ||q||^2 / (12 d)),
+    // for this thread's softmax heads 2c and 2c+1
+    float alpha0 = 0.f, alpha1 = 0.f;
+    if constexpr (kTierB) {
+        float qn2 = part[0] + part[1] + part[2] + part[3];   // ||q_g||^2 over channels 32c .. 32c+31
+        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
+        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 2);
+        const float lg = p.tb_log_2_over_delta + logf((float)max(ctx, 1));   // log(2S / delta)
+        const float al = sqrtf(2.0f * lg * qn2 * (1.0f / (12.0f * kHeadDim)));
+        alpha0 = __shfl_sync(0xffffffffu, al, 8 * c);
+        alpha1 = __shfl_sync(0xffffffffu, al, 8 * c + 4);
+    }
     float band_a, band_b;   // squared norms of bands 2c and 2c+1 of head g
     if (p.rope_layout == WC_ROPE_HALF) {
         // lane c holds the first (c < 2) or second (c >= 2) halves of bands 4(c&1) + i
@@ -196,6 +208,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     // exceeds it by more than 8 (P may reach 2^8 in between).
     float m_run[2] = {-INFINITY, -INFINITY};
     float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
+    float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
@@ -305,6 +318,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             }
             if (!ok0) sv[0] = 0.f;
             if (!ok1) sv[1] = 0.f;
+            if constexpr (kTierB) {
+                if (!ok0) sk[0] = 0.f;
+                if (!ok1) sk[1] = 0.f;
+            }
             float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
@@ -317,8 +334,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -331,6 +348,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 const float pe = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
                 l_part[e] += pe;
                 d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                if constexpr (kTierB)
+                    db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
@@ -461,6 +480,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         for (int e = 0; e < 2; ++e) {
             l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
             d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+            if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
             spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
         }
     const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
@@ -488,6 +508,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
             }
         }
     }
@@ -518,6 +539,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             } else {
                 s.x = fmaf(wt, src[0], s.x);   // l
                 s.y = fmaf(wt, src[1], s.y);   // D
+                s.z = fmaf(wt, src[2], s.z);   // Tier-B D
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -527,6 +549,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             dst[kHeadDim] = M;
             dst[kHeadDim + 1] = s.x;
             dst[kHeadDim + 2] = s.y;
+            dst[kHeadDim + 3] = s.z;
         }
     }
 }
@@ -600,6 +623,7 @@ __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h,
     }
 }
 
+template <bool kTierB>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -738,6 +762,18 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     }
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+    // Tier B (§4.2): u_t = alpha s_t with alpha = sqrt(2 log(2S/delta) ||q||^2 / (12 d)),
+    // for this thread's softmax heads 2c and 2c+1
+    float alpha0 = 0.f, alpha1 = 0.f;
+    if constexpr (kTierB) {
+        float qn2 = part[0] + part[1] + part[2] + part[3];   // ||q_g||^2 over channels 32c .. 32c+31
+        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
+        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 2);
+        const float lg = p.tb_log_2_over_delta + logf((float)max(ctx, 1));   // log(2S / delta)
+        const float al = sqrtf(2.0f * lg * qn2 * (1.0f / (12.0f * kHeadDim)));
+        alpha0 = __shfl_sync(0xffffffffu, al, 8 * c);
+        alpha1 = __shfl_sync(0xffffffffu, al, 8 * c + 4);
+    }
     float band_a, band_b;
     if (p.rope_layout == WC_ROPE_HALF) {
 #pragma unroll
@@ -764,6 +800,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 
     float m_run[2] = {-INFINITY, -INFINITY};
     float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
+    float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
@@ -828,6 +865,10 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             }
             if (!ok0) sv[0] = 0.f;
             if (!ok1) sv[1] = 0.f;
+            if constexpr (kTierB) {
+                if (!ok0) sk[0] = 0.f;
+                if (!ok1) sk[1] = 0.f;
+            }
             float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
@@ -840,8 +881,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -854,6 +895,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const float pe = fast_exp2(y[i] - m_run[e]);
                 l_part[e] += pe;
                 d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                if constexpr (kTierB)
+                    db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
@@ -943,6 +986,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         for (int e = 0; e < 2; ++e) {
             l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
             d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+            if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
             spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
         }
     const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
@@ -969,6 +1013,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
             }
         }
     }
@@ -998,6 +1043,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             } else {
                 s4.x = fmaf(wt, src[0], s4.x);
                 s4.y = fmaf(wt, src[1], s4.y);
+                s4.z = fmaf(wt, src[2], s4.z);
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -1007,6 +1053,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             dst[kHeadDim] = M;
             dst[kHeadDim + 1] = s4.x;
             dst[kHeadDim + 2] = s4.y;
+            dst[kHeadDim + 3] = s4.z;
         }
     }
 }
@@ -1032,20 +1079,22 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     // all of this warp's split rows of a round are loaded before any is
     // combined, so the loads overlap (one memory latency per round, not per split)
     constexpr int kMaxRows = 16;   // rows per warp and round
-    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f;
+    const bool tier_b = p.meter_b != nullptr;
+    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f;
     for (int s0 = warp; s0 < p.splits; s0 += kMergeWarps * kMaxRows) {
-        float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows];
+        float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows], dbs[kMaxRows];
 #pragma unroll
         for (int i = 0; i < kMaxRows; ++i) {
             const int s = s0 + i * kMergeWarps;
             ms[i] = -INFINITY;
-            v[i] = ls[i] = ds[i] = 0.f;
+            v[i] = ls[i] = ds[i] = dbs[i] = 0.f;
             if (s < p.splits) {
                 const float* ps = base + s * split_stride;
                 ms[i] = __ldcg(ps + kHeadDim);
                 v[i] = __ldcg(ps + 32 * chunk + lane);
                 ls[i] = __ldcg(ps + kHeadDim + 1);
                 ds[i] = __ldcg(ps + kHeadDim + 2);
+                if (tier_b) dbs[i] = __ldcg(ps + kHeadDim + 3);
             }
         }
         float Mr = M;
@@ -1054,7 +1103,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
         if (Mr == -INFINITY) continue;
         if (Mr > M) {   // move the running sums to the new reference
             const float f = (M == -INFINITY) ? 0.f : fast_exp2(M - Mr);
-            acc *= f; L *= f; Dn *= f;
+            acc *= f; L *= f; Dn *= f; Db *= f;
             M = Mr;
         }
 #pragma unroll
@@ -1064,6 +1113,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             acc = fmaf(w, v[i], acc);
             L = fmaf(w, ls[i], L);
             Dn = fmaf(w, ds[i], Dn);
+            Db = fmaf(w, dbs[i], Db);
         }
     }
     red[warp][lane] = acc;
@@ -1071,13 +1121,14 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
         red[warp][32] = M;
         red[warp][33] = L;
         red[warp][34] = Dn;
+        red[warp][35] = Db;
     }
     __syncthreads();
     if (warp == 0) {
         float Mt = -INFINITY;
 #pragma unroll
         for (int w = 0; w < kMergeWarps; ++w) Mt = fmaxf(Mt, red[w][32]);
-        float a = 0.f, l = 0.f, dn = 0.f;
+        float a = 0.f, l = 0.f, dn = 0.f, db = 0.f;
         if (Mt != -INFINITY) {
 #pragma unroll
             for (int w = 0; w < kMergeWarps; ++w) {
@@ -1086,6 +1137,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
                 a = fmaf(f, red[w][lane], a);
                 l = fmaf(f, red[w][33], l);
                 dn = fmaf(f, red[w][34], dn);
+                db = fmaf(f, red[w][35], db);
             }
         }
         const size_t cell = (size_t)b * p.num_q_heads + hq;
@@ -1098,6 +1150,15 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             }
             p.meter_raw[cell] = raw;
             p.meter[cell] = fminf(1.0f, raw);
+            if (tier_b) {
+                float rb = 0.f;
+                if (l > 0.f) {
+                    const float D = db / l;
+                    rb = 0.5f * D * (D + 2.0f);
+                }
+                p.meter_b_raw[cell] = rb;
+                p.meter_b[cell] = fminf(1.0f, rb);
+            }
         }
     }
 }
@@ -1168,22 +1229,22 @@ static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
     return launch_pdl(merge_kernel, grid, dim3(32 * kMergeWarps), smem, stream, p);
 }
 
-template <int kScheme, int kBits>
+template <int kScheme, int kBits, bool kTierB>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;   // per process; the attributes are per function
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>,
+        cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kTierB>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;
         // the library's kernels all prefer the largest shared-memory carveout,
         // so consecutive launches do not reconfigure the L1 / shared split
-        e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kTierB>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
     }
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits>, grid, dim3(kThreads), kSmemBytes, stream, p);
+    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kTierB>, grid, dim3(kThreads), kSmemBytes, stream, p);
     if (e != cudaSuccess) return e;
     // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
@@ -1221,13 +1282,14 @@ static bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+template <bool kTierB>
 static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel<kTierB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kWsSmemBytes);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(decode_ws_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(decode_ws_kernel<kTierB>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -1238,16 +1300,18 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
         !encode_page_map(&wp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_ws_kernel, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
+    cudaError_t e = launch_pdl(decode_ws_kernel<kTierB>, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
     return launch_merge(p, stream);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.batch == 0) return cudaSuccess;
-    if (scheme == WC_SCHEME_FP8_E4M3) return launch_one<WC_SCHEME_FP8_E4M3, 8>(p, stream);
-    if (use_ws(scheme, bits)) return launch_ws(p, stream);
-    return launch_one<WC_SCHEME_DITHER_INT8, 10>(p, stream);
+    const bool tier_b = p.meter_b != nullptr;   // dithered INT8 only (checked by the caller)
+    if (scheme == WC_SCHEME_FP8_E4M3) return launch_one<WC_SCHEME_FP8_E4M3, 8, false>(p, stream);
+    if (use_ws(scheme, bits)) return tier_b ? launch_ws<true>(p, stream) : launch_ws<false>(p, stream);
+    return tier_b ? launch_one<WC_SCHEME_DITHER_INT8, 10, true>(p, stream)
+                  : launch_one<WC_SCHEME_DITHER_INT8, 10, false>(p, stream);
 }
 
 }  // namespace wc

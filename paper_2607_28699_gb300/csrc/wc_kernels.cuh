@@ -33,6 +33,9 @@ struct DecodeParams {
     float* out;
     float* meter;
     float* meter_raw;
+    float* meter_b;       // Tier-B meters (§4.2), nullptr: not computed
+    float* meter_b_raw;
+    float tb_log_2_over_delta;   // log(2 / delta_loc) for Tier B
     uint32_t* status;     // workspace word
     uint32_t* counters;   // [batch * Hkv], zero between calls
     float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
@@ -41,7 +44,7 @@ struct DecodeParams {
     PhiloxKeys keys;
 };
 
-// Per (query head, split) partial: acc[128] | m | l | D | pad.
+// Per (query head, split) partial: acc[128] | m | l | D | Tier-B D.
 constexpr int kPartialStride = kHeadDim + 4;
 
 // Workspace layout (bytes): [0, 256) status word, then counters, then

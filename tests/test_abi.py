@@ -53,3 +53,19 @@ def test_host_validation_without_gpu(lib):
     assert lib.wc_gate(None, 7, 2, ctypes.c_float(0.1), None, None, None, None) == 1
     assert lib.wc_kv_quantize_witness(None, 0, None, None, None, 0, None, None, None, None,
                                       None, None, None) == 1
+
+
+def test_tier_b_host_validation_without_gpu(lib):
+    """Tier B is refused before any launch for the fp8 scheme, for delta_loc
+    outside (0, 1) and without its output pointers."""
+    import paper_2607_28699_gb300 as wc
+    f = lib.wc_metered_decode_attention_tier_b
+    fp8 = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4, scheme=wc.SCHEME_FP8_E4M3).c()
+    dummy = ctypes.c_void_p(16)
+    args = lambda d, delta, mb: (ctypes.byref(d), 0, None, None, 1, None, 1, None, None, None, None, None,
+                                 ctypes.c_double(delta), None, None, None, mb, mb, None, 0, None)
+    assert f(*args(fp8, 0.01, dummy)) == 2 and b"Tier B" in lib.wc_last_error()
+    int8 = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4).c()
+    for bad in (0.0, 1.0, -0.5, float("nan")):
+        assert f(*args(int8, bad, dummy)) == 1 and b"delta_loc" in lib.wc_last_error()
+    assert f(*args(int8, 0.01, None)) == 1 and b"meter_b" in lib.wc_last_error()
