@@ -30,6 +30,14 @@ e-form meter.  Here the scale is one stored fp16 value per (token, KV head)
 The guarantee is probabilistic and holds for non-adaptive queries (§4.2
 "Scope of the probabilistic guarantee").
 
+§3 output propagation and §4.2 "Value side and the joint event": with
+rho^v_t = ||v^_t - v_t||, ||y - y^|| <= 2 TV max_t ||v_t|| + sum_t p~_t rho^v_t;
+with TV bounded by the meter this is an output-error bound computable from
+stored per-token values.  Reading (the paper names pass_V without a
+formula): pass_V holds when the value term sum_t p~_t rho^v_t is at most
+tau_V max_t ||v_t||, and the joint gate keeps a cell iff pass_K (meter_raw
+<= tau_K) and pass_V, both decided in float32.
+
 Gate (§6 meter-loop box; §4.3 certified vs risk-ranked): a (layer, head)
 falls back when its meter exceeds tau.  Reading: keep the compressed path
 iff meter_raw <= tau (so equality keeps, NaN falls back), evaluated in
@@ -110,6 +118,16 @@ def tier_b_bound(q, s, ctx_len, delta_loc):
     return np.sqrt(2.0 * var * np.log(2.0 * ctx_len / delta_loc))
 
 
+def value_term(p_tilde, rho):
+    """sum_t p~_t rho^v_t."""
+    return np.sum(np.asarray(p_tilde, np.float64) * np.asarray(rho, np.float64), axis=-1)
+
+
+def output_bound(meter, v_max, vterm):
+    """||y - y^|| <= 2 TV max_t ||v_t|| + sum_t p~_t rho^v_t, with TV <= meter (<= 1)."""
+    return 2.0 * np.asarray(meter, np.float64) * np.asarray(v_max, np.float64) + np.asarray(vterm, np.float64)
+
+
 def logits(q, k):
     """z_t = q . k_t / sqrt(d); q [..., d], k [..., S, d] -> [..., S]."""
     q = np.asarray(q, dtype=np.float64)
@@ -130,6 +148,20 @@ def gate(meter_raw, tau, group):
     """
     mr = np.asarray(meter_raw, dtype=np.float32)
     keep_q = mr <= np.float32(tau)
+    n = keep_q.shape[-1]
+    if n % group:
+        raise ValueError("cells must come in whole groups")
+    keep_kv = np.all(keep_q.reshape(keep_q.shape[:-1] + (n // group, group)), axis=-1)
+    return keep_q, keep_kv, int(np.sum(keep_q)), int(np.sum(keep_kv))
+
+
+def joint_gate(meter_raw, vterm, v_max, tau_k, tau_v, group):
+    """Joint keep decisions (pass_K and pass_V) in float32, with the same
+    layout and counts as ``gate``."""
+    mr = np.asarray(meter_raw, dtype=np.float32)
+    vt = np.asarray(vterm, dtype=np.float32)
+    vm = np.asarray(v_max, dtype=np.float32)
+    keep_q = (mr <= np.float32(tau_k)) & (vt <= np.float32(tau_v) * vm)
     n = keep_q.shape[-1]
     if n % group:
         raise ValueError("cells must come in whole groups")

@@ -49,6 +49,7 @@ def empty_cache(desc):
         "k_codes": np.zeros(shp + (desc.head_dim,), code_t),
         "v_codes": np.zeros(shp + (desc.head_dim,), code_t),
         "k_witness": np.zeros(shp + (desc.num_bands,), np.float16),
+        "v_witness": np.zeros(shp + (2,), np.float16),       # (rho^v, ||v||), rounded up
     }
     if desc.scheme == SCHEME_DITHER_INT8:
         cache["k_scale"] = np.zeros(shp, np.float16)
@@ -82,7 +83,7 @@ def write_tokens(desc, layer, k16, v16, slot_mapping, cache):
         kr = np.asarray(k16)[live, h, :]
         vr = np.asarray(v16)[live, h, :]
         kc, ks, khat = quantize_rows(desc, layer, h, kr, slots, 0)
-        vc, vs, _ = quantize_rows(desc, layer, h, vr, slots, 1)
+        vc, vs, vhat = quantize_rows(desc, layer, h, vr, slots, 1)
         cache["k_codes"][page, h, off] = kc
         cache["v_codes"][page, h, off] = vc
         if ks is not None:
@@ -91,6 +92,7 @@ def write_tokens(desc, layer, k16, v16, slot_mapping, cache):
         resid = khat - kr.astype(np.float64)
         cache["k_witness"][page, h, off] = quantizer.witness(
             resid, desc.num_bands, desc.rope_layout)
+        cache["v_witness"][page, h, off] = quantizer.value_witness(vhat - vr.astype(np.float64), vr)
 
 
 def slots_of(desc, block_table_row, ctx_len):
@@ -129,7 +131,8 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
     d = desc.head_dim
     slots = slots_of(desc, block_table_row, ctx_len)
     res = {k: np.zeros((desc.num_q_heads, d)) for k in ("out", "out_exact")}
-    for k in ("meter", "meter_raw", "tv", "A", "meter_b", "meter_b_raw"):
+    for k in ("meter", "meter_raw", "tv", "A", "meter_b", "meter_b_raw", "value_term", "v_max", "out_bound",
+              "out_err"):
         res[k] = np.zeros(desc.num_q_heads)
     tier_b = delta_loc is not None
     if tier_b and desc.scheme != SCHEME_DITHER_INT8:
@@ -144,6 +147,10 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
             c = M.tier_a_bound(q, w, desc.num_bands, desc.rope_layout)
             res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.eform_meter(p_tilde, c)
             res["out"][hq] = M.attend(p_tilde, vhat)
+            vw = cache["v_witness"][page, h, off].astype(np.float64)        # [S, 2]
+            res["value_term"][hq] = M.value_term(p_tilde, vw[:, 0])
+            res["v_max"][hq] = np.max(vw[:, 1]) if ctx_len else 0.0
+            res["out_bound"][hq] = M.output_bound(res["meter"][hq], res["v_max"][hq], res["value_term"][hq])
             if tier_b:
                 u = M.tier_b_bound(q, cache["k_scale"][page, h, off].astype(np.float64), ctx_len, delta_loc)
                 res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
@@ -151,4 +158,5 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
                 p = M.softmax(M.logits(q, np.asarray(k_exact)[:ctx_len, h]))
                 res["tv"][hq] = M.total_variation(p, p_tilde)
                 res["out_exact"][hq] = M.attend(p, np.asarray(v_exact)[:ctx_len, h])
+                res["out_err"][hq] = np.linalg.norm(res["out_exact"][hq] - res["out"][hq])
     return res

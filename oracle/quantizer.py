@@ -131,3 +131,14 @@ def band_norms(v, num_bands, rope_layout):
 def witness(residual, num_bands, rope_layout):
     """Stored witness: fp16 round-up of the per-band residual norms."""
     return fp.fp16_ru(band_norms(residual, num_bands, rope_layout))
+
+
+def value_witness(residual, v):
+    """Value-side witness of each row (§3 output bound, rho^v_t := ||v^_t - v_t||):
+    [..., 2] fp16 = (rho^v rounded up, ||v|| rounded up).  Reading: the value
+    norm is stored too (rounded up), so that max_t ||v_t|| in the output bound
+    is available at decode time without the exact values."""
+    r = np.asarray(residual, dtype=np.float64)
+    v = np.asarray(v, dtype=np.float64)
+    return np.stack([fp.fp16_ru(np.sqrt(np.sum(r * r, axis=-1))),
+                     fp.fp16_ru(np.sqrt(np.sum(v * v, axis=-1)))], axis=-1)
