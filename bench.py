@@ -16,6 +16,7 @@ the slowest rank's time is used (weak scaling).
 """
 
 import argparse
+import dataclasses
 import json
 import os
 import statistics
@@ -167,12 +168,17 @@ class Setup:
         self.ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
         last = np.cumsum(wl.ctx_lens) - 1                       # index of each sequence's newest token
         self.new_slots = self.sm[torch.from_numpy(last).cuda()].contiguous()
-        self.caches, self.k_new, self.v_new = [], [], []
+        self.caches, self.k_new, self.v_new, self.vcaches = [], [], [], []
         for layer in range(wl.n_layers):
             k, v = W.layer_kv(wl, layer, device="cuda")
             cache = wc.LayerCache.empty(self.desc)
             wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, cache)   # prefill write
             self.caches.append(cache)
+            # the same cache viewed with a value witness too (value-side measurement only)
+            vc = dataclasses.replace(cache, v_witness=torch.zeros(cache.k_witness.shape[:-1] + (2,),
+                                                                  dtype=torch.float16, device="cuda"))
+            wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, vc)
+            self.vcaches.append(vc)
             li = torch.from_numpy(last).cuda()
             self.k_new.append(k[li].contiguous())
             self.v_new.append(v[li].contiguous())
@@ -190,6 +196,12 @@ class Setup:
         e.record()
         e.synchronize()
         self.write_call_s = s.elapsed_time(e) / 1e3 / reps
+        s.record()                                   # the same with the value witness stored too
+        for _ in range(reps):
+            wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.vcaches[-1])
+        e.record()
+        e.synchronize()
+        self.write_v_call_s = s.elapsed_time(e) / 1e3 / reps
         del k, v
         self.q = torch.stack([W.layer_queries(wl, layer, device="cuda") for layer in range(wl.n_layers)])
         self.ws = wc.Workspace(self.desc, wl.batch, wl.max_pages)
@@ -218,6 +230,16 @@ class Setup:
     def decode_all(self):
         for layer in range(self.wl.n_layers):
             self.decode(layer)
+
+    def decode_all_value(self):
+        """The same calls with the value-side terms and output bound (§3, §4.2)."""
+        if not hasattr(self, "vterm"):
+            self.vterm, self.vmax, self.obound = (torch.empty_like(self.meter) for _ in range(3))
+        for layer in range(self.wl.n_layers):
+            self.wc.metered_decode_attention_v(
+                self.desc, layer, self.q[layer], self.bt, self.ctx, self.vcaches[layer], self.ws,
+                out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
+                value_term=self.vterm[layer], v_max=self.vmax[layer], out_bound=self.obound[layer])
 
     TIER_B_DELTA_REQ = 1e-2   # request-level budget, split over layers, query heads and one step
 
@@ -293,6 +315,26 @@ def run_ours(args, rank, world, local):
     torch.cuda.synchronize()
     dec_avg_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
 
+    # ---- the same calls with the value side too (its marginal cost) ----
+    vgraph = capture(st.decode_all_value)
+    for _ in range(args.warmup):
+        vgraph.replay()
+    torch.cuda.synchronize()
+    d0.record()
+    for _ in range(args.steps):
+        vgraph.replay()
+    d1.record()
+    torch.cuda.synchronize()
+    v_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
+    kq, _, _ = st.wc.gate_joint(st.raw.reshape(-1), st.vterm.reshape(-1), st.vmax.reshape(-1), wl.group,
+                                st.tau, st.tau)
+    value_side = {"decode_call_ms": v_ms, "overhead_vs_plain": v_ms / dec_avg_ms - 1.0,
+                  "write_ms_per_layer_prefill": st.write_v_call_s * 1e3,
+                  "write_overhead_vs_plain": st.write_v_call_s / st.write_call_s - 1.0,
+                  "joint_kept_frac_at_tau": float(kq.float().mean()),
+                  "out_bound_median": float(st.obound.median()),
+                  "rel_value_term_median": float((st.vterm / st.vmax.clamp_min(1e-30)).median())}
+
     # ---- the same calls with the Tier-B certificate too (its marginal cost) ----
     tier_b = None
     if wl.scheme == 0:
@@ -347,6 +389,7 @@ def run_ours(args, rank, world, local):
         "hbm_gbs_step": step_gbs,
         "decode_call_ms": dec_avg_ms,
         "tier_b": tier_b,
+        "value_side": value_side,
         "roofline": {"kernel": ("decode_ws_kernel" if wl.scheme == 0 and args.dither_bits == 8 else "decode_kernel")
                                + " + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

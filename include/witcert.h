@@ -31,6 +31,8 @@
  *                                               or fp8 e4m3fn bytes (WC_SCHEME_FP8_E4M3)
  *   k_scale, v_scale [num_pages][Hkv][16]       fp16, dither scheme only (else NULL)
  *   k_witness        [num_pages][Hkv][16][8]    fp16, per-band residual norms
+ *   v_witness        [num_pages][Hkv][16][2]    fp16 (||v^ - v||, ||v||) rounded up;
+ *                                               optional, for the value side only
  */
 #ifndef WITCERT_H
 #define WITCERT_H
@@ -124,6 +126,19 @@ wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer,
                                  uint32_t* dev_status, void* stream);
 
 /*
+ * wc_kv_quantize_witness that also stores the value witness of every written
+ * V row (§3 output bound, §4.2 "Value side"): v_witness[slot] =
+ * (||v^ - v||, ||v||), each rounded up to fp16 (never below the exact norm,
+ * at most one fp16 step above).  v_witness 16-byte aligned, not NULL.
+ */
+wc_status wc_kv_quantize_witness_v(const wc_cache_desc* desc, int32_t layer,
+                                   const void* k, const void* v,
+                                   const int32_t* slot_mapping, int32_t n_tok,
+                                   void* k_codes, void* v_codes,
+                                   void* k_scale, void* v_scale, void* k_witness,
+                                   void* v_witness, uint32_t* dev_status, void* stream);
+
+/*
  * Bytes of workspace wc_metered_decode_attention needs for `batch`
  * sequences whose block tables hold `max_pages` pages, on the current
  * device (the split count depends on its SM count).  Returns 0 and sets
@@ -198,6 +213,30 @@ wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t 
                                              void* stream);
 
 /*
+ * Metered decode attention with the value-side terms and the output bound
+ * (§3: ||y - y^|| <= 2 TV max_t ||v_t|| + sum_t p~_t rho^v_t; §4.2 "Value side
+ * and the joint event").  Same computation, arguments and outputs as
+ * wc_metered_decode_attention, plus for every sequence b and query head hq:
+ *   value_term[b][hq] = sum_t p~_t rho^v_t          (rho^v from v_witness)
+ *   v_max[b][hq]      = max_t ||v_t||                (over the KV head's tokens)
+ *   out_bound[b][hq]  = 2 * meter[b][hq] * v_max + value_term   (bounds ||y - y^||)
+ * The value term is deterministic given p~: it needs no probability budget.
+ *   v_witness  as written by wc_kv_quantize_witness_v, 16-byte aligned
+ *   value_term, v_max, out_bound [batch][Hq] fp32, device, not NULL
+ */
+wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer,
+                                        const void* q, const int32_t* block_table,
+                                        int32_t max_pages, const int32_t* ctx_lens,
+                                        int32_t batch,
+                                        const void* k_codes, const void* v_codes,
+                                        const void* k_scale, const void* v_scale,
+                                        const void* k_witness, const void* v_witness,
+                                        float* out, float* meter, float* meter_raw,
+                                        float* value_term, float* v_max, float* out_bound,
+                                        void* workspace, size_t workspace_bytes,
+                                        void* stream);
+
+/*
  * Allocation-free metered decode.  The paper has no counterpart: this is a
  * deployment convenience for callers that cannot allocate device memory at
  * decode time (a runtime that pre-plans every buffer, code running inside an
@@ -211,7 +250,7 @@ wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t 
  *   dev_status  optional device uint32 that collects WC_DEV_* bits (OR); when
  *               NULL the bits go to a word inside the built-in scratch.
  * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
- * more scratch than 4 MiB (about 990 (sequence, KV head, split) partial
+ * more scratch than 4 MiB (about 960 (sequence, KV head, split) partial
  * results; the split count follows wc_workspace_size's plan).
  * The first call on each device looks up the scratch address and clears its
  * status word (a synchronous cudaMemset); make that first call before any
@@ -243,6 +282,18 @@ wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t
  */
 wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau,
                   uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept, void* stream);
+
+/*
+ * Joint gate (§4.2 "Value side and the joint event"): pass_K and pass_V.
+ * keep_q[i] = (meter_raw[i] <= tau_k) && (value_term[i] <= tau_v * v_max[i]),
+ * all in fp32 (the product rounded once); otherwise as wc_gate.  Reading:
+ * the paper names pass_V without a formula; here it bounds the value term
+ * relative to the largest value norm.
+ *   value_term, v_max [n_cells] fp32, device (from wc_metered_decode_attention_v)
+ */
+wc_status wc_gate_joint(const float* meter_raw, const float* value_term, const float* v_max,
+                        int32_t n_cells, int32_t group, float tau_k, float tau_v,
+                        uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept, void* stream);
 
 /*
  * Synchronises `stream`, copies the device status word held in `workspace`

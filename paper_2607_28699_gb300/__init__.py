@@ -32,6 +32,7 @@ ROPE_INTERLEAVED = 1
 DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT = 1, 2, 4, 8
 EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
            "wc_metered_decode_attention_tier_b", "wc_metered_decode_attention_noalloc",
+           "wc_kv_quantize_witness_v", "wc_metered_decode_attention_v", "wc_gate_joint",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -60,6 +61,13 @@ def _load():
     lib.wc_metered_decode_attention_tier_b.restype = ctypes.c_int
     lib.wc_gate.argtypes = [vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]
     lib.wc_gate.restype = ctypes.c_int
+    lib.wc_gate_joint.argtypes = [vp, vp, vp, i32, i32, ctypes.c_float, ctypes.c_float, vp, vp, vp, vp]
+    lib.wc_gate_joint.restype = ctypes.c_int
+    lib.wc_kv_quantize_witness_v.argtypes = [vp, i32, vp, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp]
+    lib.wc_kv_quantize_witness_v.restype = ctypes.c_int
+    lib.wc_metered_decode_attention_v.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp, vp,
+                                                  vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.wc_metered_decode_attention_v.restype = ctypes.c_int
     lib.wc_read_status.argtypes = [vp, i32, vp, vp]
     lib.wc_read_status.restype = ctypes.c_int
     lib.wc_last_error.argtypes = []
@@ -131,9 +139,10 @@ class LayerCache:
     k_scale: Optional[torch.Tensor]
     v_scale: Optional[torch.Tensor]
     k_witness: torch.Tensor
+    v_witness: Optional[torch.Tensor] = None   # (||v^ - v||, ||v||) per slot, value side only
 
     @staticmethod
-    def empty(desc: CacheDesc, device="cuda"):
+    def empty(desc: CacheDesc, device="cuda", value_witness=False):
         shp = (desc.num_pages, desc.num_kv_heads, desc.page_size)
         code_t = torch.int8 if desc.scheme == SCHEME_DITHER_INT8 else torch.uint8
         dither = desc.scheme == SCHEME_DITHER_INT8
@@ -142,22 +151,31 @@ class LayerCache:
             torch.zeros(shp + (desc.head_dim,), dtype=code_t, device=device),
             torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
             torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
-            torch.zeros(shp + (desc.num_bands,), dtype=torch.float16, device=device))
+            torch.zeros(shp + (desc.num_bands,), dtype=torch.float16, device=device),
+            torch.zeros(shp + (2,), dtype=torch.float16, device=device) if value_witness else None)
 
     def nbytes(self):
         return sum(t.numel() * t.element_size() for t in
-                   (self.k_codes, self.v_codes, self.k_scale, self.v_scale, self.k_witness) if t is not None)
+                   (self.k_codes, self.v_codes, self.k_scale, self.v_scale, self.k_witness, self.v_witness)
+                   if t is not None)
 
 
 def kv_quantize_witness(desc: CacheDesc, layer: int, k: torch.Tensor, v: torch.Tensor,
                         slot_mapping: torch.Tensor, cache: LayerCache,
                         dev_status: Optional[torch.Tensor] = None, stream=None):
-    """``wc_kv_quantize_witness``: k, v fp16 [n_tok, Hkv, 128]; slots int32 [n_tok]."""
+    """``wc_kv_quantize_witness`` (``_v`` when the cache holds a value witness):
+    k, v fp16 [n_tok, Hkv, 128]; slots int32 [n_tok]."""
     d = desc.c()
-    _check(lib.wc_kv_quantize_witness(
-        ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
-        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
-        _ptr(cache.k_witness), _ptr(dev_status), _stream(stream)))
+    if cache.v_witness is None:
+        _check(lib.wc_kv_quantize_witness(
+            ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
+            _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+            _ptr(cache.k_witness), _ptr(dev_status), _stream(stream)))
+    else:
+        _check(lib.wc_kv_quantize_witness_v(
+            ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
+            _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+            _ptr(cache.k_witness), _ptr(cache.v_witness), _ptr(dev_status), _stream(stream)))
 
 
 def workspace_size(desc: CacheDesc, batch: int, max_pages: int) -> int:
@@ -222,6 +240,40 @@ def metered_decode_attention_tier_b(desc: CacheDesc, layer: int, q: torch.Tensor
         _ptr(cache.k_witness), float(delta_loc), _ptr(out), _ptr(meter), _ptr(meter_raw), _ptr(meter_b),
         _ptr(meter_b_raw), ws.ptr(), ws.nbytes, _stream(stream)))
     return out, meter, meter_raw, meter_b, meter_b_raw
+
+
+def metered_decode_attention_v(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
+                               ctx_lens: torch.Tensor, cache: LayerCache, ws: Workspace, out=None, meter=None,
+                               meter_raw=None, value_term=None, v_max=None, out_bound=None, stream=None):
+    """``wc_metered_decode_attention_v``; returns (out, meter, meter_raw, value_term, v_max, out_bound)."""
+    if cache.v_witness is None:
+        raise ValueError("the cache holds no value witness (LayerCache.empty(..., value_witness=True))")
+    batch, max_pages = block_table.shape
+    dev = q.device
+    cells = (batch, desc.num_q_heads)
+    new = lambda t: torch.empty(cells, dtype=torch.float32, device=dev) if t is None else t
+    out = torch.empty(batch, desc.num_q_heads, desc.head_dim, dtype=torch.float32, device=dev) if out is None else out
+    meter, meter_raw, value_term, v_max, out_bound = map(new, (meter, meter_raw, value_term, v_max, out_bound))
+    d = desc.c()
+    _check(lib.wc_metered_decode_attention_v(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(cache.v_witness), _ptr(out), _ptr(meter), _ptr(meter_raw),
+        _ptr(value_term), _ptr(v_max), _ptr(out_bound), ws.ptr(), ws.nbytes, _stream(stream)))
+    return out, meter, meter_raw, value_term, v_max, out_bound
+
+
+def gate_joint(meter_raw: torch.Tensor, value_term: torch.Tensor, v_max: torch.Tensor, group: int, tau_k: float,
+               tau_v: float, keep_q=None, keep_kv=None, n_kept=None, stream=None):
+    """``wc_gate_joint``: returns (keep_q uint8 [n], keep_kv uint8 [n/group], n_kept int32 [2])."""
+    n = meter_raw.numel()
+    dev = meter_raw.device
+    keep_q = torch.empty(n, dtype=torch.uint8, device=dev) if keep_q is None else keep_q
+    keep_kv = torch.empty(n // group, dtype=torch.uint8, device=dev) if keep_kv is None else keep_kv
+    n_kept = torch.empty(2, dtype=torch.int32, device=dev) if n_kept is None else n_kept
+    _check(lib.wc_gate_joint(_ptr(meter_raw), _ptr(value_term), _ptr(v_max), n, group, float(tau_k), float(tau_v),
+                             _ptr(keep_q), _ptr(keep_kv), _ptr(n_kept), _stream(stream)))
+    return keep_q, keep_kv, n_kept
 
 
 def gate(meter_raw: torch.Tensor, group: int, tau: float, keep_q=None, keep_kv=None, n_kept=None,

@@ -84,10 +84,10 @@ int32_t wc_version(void) { return (1 << 16) | 0; }
 
 const char* wc_last_error(void) { return g_last_error.c_str(); }
 
-wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
-                                 const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
-                                 void* k_scale, void* v_scale, void* k_witness, uint32_t* dev_status,
-                                 void* stream) {
+static wc_status write_tokens(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
+                              const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
+                              void* k_scale, void* v_scale, void* k_witness, void* v_witness,
+                              uint32_t* dev_status, void* stream) {
     if (wc_status st = check_desc(desc)) return st;
     if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
     if (n_tok < 0) return fail(WC_ERR_INVALID_ARG, "n_tok must be >= 0 (got %d)", n_tok);
@@ -96,6 +96,7 @@ wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const
     if (n_tok > 0 && (!k || !v || !slot_mapping)) return fail(WC_ERR_INVALID_ARG, "k, v, slot_mapping must not be NULL");
     if (!aligned16(k) || !aligned16(v)) return fail(WC_ERR_INVALID_ARG, "k and v must be 16-byte aligned");
     if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
+    if (v_witness && !aligned16(v_witness)) return fail(WC_ERR_INVALID_ARG, "v_witness must be 16-byte aligned");
     if (n_tok == 0) return WC_OK;
     wc::WriteParams p;
     p.k = static_cast<const __half*>(k);
@@ -106,6 +107,7 @@ wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const
     p.k_scale = static_cast<__half*>(k_scale);
     p.v_scale = static_cast<__half*>(v_scale);
     p.k_witness = static_cast<__half*>(k_witness);
+    p.v_witness = static_cast<__half*>(v_witness);
     p.dev_status = dev_status;
     p.n_tok = n_tok;
     p.num_kv_heads = desc->num_kv_heads;
@@ -115,6 +117,23 @@ wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const
     p.keys = wc::make_philox_keys(desc->seed);
     cudaError_t e = wc::launch_write(p, desc->scheme, desc->dither_bits, static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? WC_OK : cuda_fail(e, "write kernel launch");
+}
+
+wc_status wc_kv_quantize_witness(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
+                                 const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
+                                 void* k_scale, void* v_scale, void* k_witness, uint32_t* dev_status,
+                                 void* stream) {
+    return write_tokens(desc, layer, k, v, slot_mapping, n_tok, k_codes, v_codes, k_scale, v_scale, k_witness,
+                        nullptr, dev_status, stream);
+}
+
+wc_status wc_kv_quantize_witness_v(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
+                                   const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
+                                   void* k_scale, void* v_scale, void* k_witness, void* v_witness,
+                                   uint32_t* dev_status, void* stream) {
+    if (!v_witness) return fail(WC_ERR_INVALID_ARG, "v_witness must not be NULL");
+    return write_tokens(desc, layer, k, v, slot_mapping, n_tok, k_codes, v_codes, k_scale, v_scale, k_witness,
+                        v_witness, dev_status, stream);
 }
 
 size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_pages) {
@@ -138,9 +157,16 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
                                        int32_t batch, const void* k_codes, const void* v_codes,
                                        const void* k_scale, const void* v_scale, const void* k_witness,
                                        float* out, float* meter, float* meter_raw, float* meter_b,
-                                       float* meter_b_raw, double delta_loc, void* workspace,
+                                       float* meter_b_raw, double delta_loc, const void* v_witness,
+                                       float* value_term, float* v_max, float* out_bound, void* workspace,
                                        size_t workspace_bytes, void* stream) {
     if (wc_status st = check_desc(desc)) return st;
+    if (value_term || v_max || out_bound || v_witness) {
+        if (!value_term || !v_max || !out_bound || !v_witness)
+            return fail(WC_ERR_INVALID_ARG, "v_witness, value_term, v_max and out_bound must not be NULL");
+        if (!aligned16(v_witness)) return fail(WC_ERR_INVALID_ARG, "v_witness must be 16-byte aligned");
+        if (meter_b) return fail(WC_ERR_UNSUPPORTED, "Tier B and the value side are separate calls");
+    }
     if (meter_b || meter_b_raw) {
         if (desc->scheme != WC_SCHEME_DITHER_INT8)
             return fail(WC_ERR_UNSUPPORTED, "Tier B needs the dithered INT8 cache (a controlled quantizer)");
@@ -180,6 +206,10 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.meter_b = meter_b;
     p.meter_b_raw = meter_b_raw;
     p.tb_log_2_over_delta = meter_b ? (float)std::log(2.0 / delta_loc) : 0.0f;
+    p.v_witness = static_cast<const __half*>(v_witness);
+    p.value_term = value_term;
+    p.v_max = v_max;
+    p.out_bound = out_bound;
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
@@ -205,8 +235,8 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
                                       float* out, float* meter, float* meter_raw, void* workspace,
                                       size_t workspace_bytes, void* stream) {
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
-                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, workspace,
-                                 workspace_bytes, stream);
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
+                                 nullptr, nullptr, workspace, workspace_bytes, stream);
 }
 
 wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t layer, const void* q,
@@ -219,19 +249,47 @@ wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t 
     if (!meter_b || !meter_b_raw) return fail(WC_ERR_INVALID_ARG, "meter_b and meter_b_raw must not be NULL");
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, meter_b, meter_b_raw, delta_loc,
-                                 workspace, workspace_bytes, stream);
+                                 nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream);
 }
 
-wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau, uint8_t* keep_q,
-                  uint8_t* keep_kv, int32_t* n_kept, void* stream) {
+wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                        const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                        int32_t batch, const void* k_codes, const void* v_codes,
+                                        const void* k_scale, const void* v_scale, const void* k_witness,
+                                        const void* v_witness, float* out, float* meter, float* meter_raw,
+                                        float* value_term, float* v_max, float* out_bound, void* workspace,
+                                        size_t workspace_bytes, void* stream) {
+    if (!v_witness || !value_term || !v_max || !out_bound)
+        return fail(WC_ERR_INVALID_ARG, "v_witness, value_term, v_max and out_bound must not be NULL");
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, v_witness,
+                                 value_term, v_max, out_bound, workspace, workspace_bytes, stream);
+}
+
+static wc_status gate_impl(const float* meter_raw, const float* value_term, const float* v_max, int32_t n_cells,
+                          int32_t group, float tau, float tau_v, uint8_t* keep_q, uint8_t* keep_kv,
+                          int32_t* n_kept, void* stream) {
     if (n_cells < 0 || group < 1 || n_cells % group != 0)
         return fail(WC_ERR_INVALID_ARG, "n_cells (%d) must be a non-negative multiple of group (%d)", n_cells, group);
     if (!n_kept) return fail(WC_ERR_INVALID_ARG, "n_kept must not be NULL");
     if (n_cells > 0 && (!meter_raw || !keep_q || !keep_kv))
         return fail(WC_ERR_INVALID_ARG, "meter_raw, keep_q, keep_kv must not be NULL");
-    cudaError_t e = wc::launch_gate(meter_raw, n_cells, group, tau, keep_q, keep_kv, n_kept,
+    cudaError_t e = wc::launch_gate(meter_raw, value_term, v_max, n_cells, group, tau, tau_v, keep_q, keep_kv, n_kept,
                                     static_cast<cudaStream_t>(stream));
     return e == cudaSuccess ? WC_OK : cuda_fail(e, "gate kernel launch");
+}
+
+wc_status wc_gate(const float* meter_raw, int32_t n_cells, int32_t group, float tau, uint8_t* keep_q,
+                  uint8_t* keep_kv, int32_t* n_kept, void* stream) {
+    return gate_impl(meter_raw, nullptr, nullptr, n_cells, group, tau, 0.0f, keep_q, keep_kv, n_kept, stream);
+}
+
+wc_status wc_gate_joint(const float* meter_raw, const float* value_term, const float* v_max, int32_t n_cells,
+                        int32_t group, float tau_k, float tau_v, uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept,
+                        void* stream) {
+    if (n_cells > 0 && (!value_term || !v_max))
+        return fail(WC_ERR_INVALID_ARG, "value_term and v_max must not be NULL");
+    return gate_impl(meter_raw, value_term, v_max, n_cells, group, tau_k, tau_v, keep_q, keep_kv, n_kept, stream);
 }
 
 wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word, uint32_t* bits, void* stream) {
@@ -337,6 +395,10 @@ extern "C" wc_status wc_metered_decode_attention_noalloc(
     p.meter_b = nullptr;
     p.meter_b_raw = nullptr;
     p.tb_log_2_over_delta = 0.0f;
+    p.v_witness = nullptr;
+    p.value_term = nullptr;
+    p.v_max = nullptr;
+    p.out_bound = nullptr;
     p.status = dev_status ? dev_status : reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);

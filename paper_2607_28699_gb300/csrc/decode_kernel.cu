@@ -36,9 +36,15 @@ constexpr int kWarps = 8;
 constexpr int kThreads = 32 * kWarps;
 constexpr int kStages = 3;
 constexpr int kMinBlocks = 2;            // two CTAs (16 warps) per SM
-constexpr int kStageBytes = 4416;        // K codes | V codes | K scale | V scale | witness
+constexpr int kStageBytes = 4416;        // copy bytes: K codes | V codes | K scale | V scale | witness
 constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
-constexpr int kSmemBytes = kWarps * kStages * kStageBytes + kWarps * kStages * 8;
+constexpr int kOffVw = 4416;             // value witness [16][2] fp16 (value side)
+constexpr int kStageStride = 4480;       // stage buffer size
+constexpr int kSmemBytes = kWarps * kStages * kStageStride + kWarps * kStages * 8;
+
+// Extra outputs compiled into a decode kernel (template bit mask).
+constexpr int kXTierB = 1;   // Tier-B meter (§4.2)
+constexpr int kXValue = 2;   // value-side witness terms and output bound (§3, §4.2)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRsd = 0.08838834764831845f;                      // 1/sqrt(128)
 constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;
@@ -79,8 +85,9 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
     return y;
 }
 
-template <int kScheme, int kBits, bool kTierB>
+template <int kScheme, int kBits, int kX>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecodeParams p) {
+    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0;
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
@@ -88,8 +95,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     const int G = p.group;
     constexpr bool kInt8 = (kScheme == WC_SCHEME_DITHER_INT8);
 
-    uint8_t* my_stages = smem + warp * kStages * kStageBytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageBytes) + warp * kStages;
+    uint8_t* my_stages = smem + warp * kStages * kStageStride;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageStride) + warp * kStages;
     if (lane == 0)
         for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
     fence_barrier_init();
@@ -138,9 +145,9 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
             return;
         }
-        uint8_t* st = my_stages + (k % kStages) * kStageBytes;
+        uint8_t* st = my_stages + (k % kStages) * kStageStride;
         const size_t ph = (size_t)phys * p.num_kv_heads + h;
-        constexpr uint32_t bytes = kInt8 ? kStageBytes : (2048 + 2048 + 256);
+        constexpr uint32_t bytes = (kInt8 ? kStageBytes : (2048 + 2048 + 256)) + (kValue ? 64 : 0);
         mbar_arrive_expect_tx(bar, bytes);
         bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, bar);
         bulk_g2s(st + kOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, bar);
@@ -149,6 +156,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             bulk_g2s(st + kOffVs, p.v_scale + ph * kPage, 32, bar);
         }
         bulk_g2s(st + kOffW, p.k_witness + ph * (kPage * kBands), 256, bar);
+        if constexpr (kValue) bulk_g2s(st + kOffVw, p.v_witness + ph * (kPage * 2), 64, bar);
     };
     __syncwarp();
 #pragma unroll
@@ -209,6 +217,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     float m_run[2] = {-INFINITY, -INFINITY};
     float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
     float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
+    float vt_part[2] = {0.f, 0.f};   // value side: sum p~ rho^v (kValue)
+    float vmax = 0.f;                // value side: max ||v|| over this thread's tokens
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
@@ -231,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         }
         consumed = k + 1;
         if (page_ok) {
-            const uint8_t* st = my_stages + (k % kStages) * kStageBytes;
+            const uint8_t* st = my_stages + (k % kStages) * kStageStride;
             const uint32_t slot0 = (uint32_t)phys * kPage;
             const int nvalid = min(kPage, ctx - lp * kPage);
 
@@ -322,6 +332,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 if (!ok0) sk[0] = 0.f;
                 if (!ok1) sk[1] = 0.f;
             }
+            float rho[2] = {0.f, 0.f};   // value witness of tokens g, g+8 (0 past the context)
+            if constexpr (kValue) {
+                const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kOffVw + 4 * g));
+                const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kOffVw + 4 * (g + 8)));
+                if (ok0) { rho[0] = w0.x; vmax = fmaxf(vmax, w0.y); }
+                if (ok1) { rho[1] = w1.x; vmax = fmaxf(vmax, w1.y); }
+            }
             float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
@@ -334,8 +351,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0; vt_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1; vt_part[1] *= a1;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -350,6 +367,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
                 if constexpr (kTierB)
                     db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
+                if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
@@ -481,8 +499,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
             d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
             if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
+            if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
             spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
         }
+    if constexpr (kValue)
+        for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
     const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
     const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
 
@@ -509,6 +530,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
             }
         }
     }
@@ -540,6 +563,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 s.x = fmaf(wt, src[0], s.x);   // l
                 s.y = fmaf(wt, src[1], s.y);   // D
                 s.z = fmaf(wt, src[2], s.z);   // Tier-B D
+                s.w = fmaf(wt, src[3], s.w);   // value term
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -550,6 +574,13 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             dst[kHeadDim + 1] = s.x;
             dst[kHeadDim + 2] = s.y;
             dst[kHeadDim + 3] = s.z;
+            if constexpr (kValue) {
+                float vm = 0.f;
+                for (int w = 0; w < kWarps; ++w)
+                    vm = fmaxf(vm, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim + 5]);
+                dst[kHeadDim + 4] = s.w;
+                dst[kHeadDim + 5] = vm;
+            }
         }
     }
 }
@@ -580,8 +611,9 @@ constexpr int kWsOffKs = 8192;      // K scales [16] fp16
 constexpr int kWsOffVs = 8224;      // V scales [16] fp16
 constexpr int kWsOffW = 8256;       // witness [16][8] fp16
 constexpr int kWsOffHdr = 8512;     // physical page (or -1)
+constexpr int kWsOffVw = 8528;      // value witness [16][2] fp16 (value side)
 constexpr int kWsStageBytes = 9216;
-static_assert(kWsOffHdr + 16 <= kWsStageBytes && kWsStageBytes % 1024 == 0, "stage layout");
+static_assert(kWsOffVw + 64 <= kWsStageBytes && kWsStageBytes % 1024 == 0, "stage layout");
 constexpr int kWsBarBytes = kWsPairs * kWsStages * 2 * 8;
 constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsBarBytes + 1024;   // + alignment slack
 static_assert(kWsSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
@@ -623,8 +655,9 @@ __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h,
     }
 }
 
-template <bool kTierB>
+template <int kX>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
+    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0;
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -709,12 +742,13 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 if (ok) {
                     const int z = phys * p.num_kv_heads + h;
                     const size_t ph = (size_t)z;
-                    mbar_arrive_expect_tx(&full[s], (uint32_t)kStageBytes);
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)(kStageBytes + (kValue ? 64 : 0)));
                     tma_page(st + kWsOffK, &wp.k_map, z, &full[s]);
                     tma_page(st + kWsOffV, &wp.v_map, z, &full[s]);
                     bulk_g2s(st + kWsOffKs, p.k_scale + ph * kPage, 32, &full[s]);
                     bulk_g2s(st + kWsOffVs, p.v_scale + ph * kPage, 32, &full[s]);
                     bulk_g2s(st + kWsOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
+                    if constexpr (kValue) bulk_g2s(st + kWsOffVw, p.v_witness + ph * (kPage * 2), 64, &full[s]);
                 } else {
                     atomicOr(p.status, WC_DEV_BAD_PAGE);
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
@@ -801,6 +835,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     float m_run[2] = {-INFINITY, -INFINITY};
     float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
     float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
+    float vt_part[2] = {0.f, 0.f};   // value side: sum p~ rho^v (kValue)
+    float vmax = 0.f;                // value side: max ||v|| over this thread's tokens
     float acc[8][4];
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
@@ -869,6 +905,13 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 if (!ok0) sk[0] = 0.f;
                 if (!ok1) sk[1] = 0.f;
             }
+            float rho[2] = {0.f, 0.f};   // value witness of tokens g, g+8 (0 past the context)
+            if constexpr (kValue) {
+                const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * g));
+                const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * (g + 8)));
+                if (ok0) { rho[0] = w0.x; vmax = fmaxf(vmax, w0.y); }
+                if (ok1) { rho[1] = w1.x; vmax = fmaxf(vmax, w1.y); }
+            }
             float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
 #pragma unroll
             for (int o = 4; o < 32; o <<= 1) {
@@ -881,8 +924,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0; vt_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1; vt_part[1] *= a1;
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -897,6 +940,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
                 if constexpr (kTierB)
                     db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
+                if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
@@ -987,8 +1031,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
             d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
             if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
+            if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
             spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
         }
+    if constexpr (kValue)
+        for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
     const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
 
     // ---- CTA merge over the consumer warps: one partial per CTA ------------------------
@@ -1014,6 +1061,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
             }
         }
     }
@@ -1044,6 +1093,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 s4.x = fmaf(wt, src[0], s4.x);
                 s4.y = fmaf(wt, src[1], s4.y);
                 s4.z = fmaf(wt, src[2], s4.z);
+                s4.w = fmaf(wt, src[3], s4.w);
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -1054,6 +1104,13 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             dst[kHeadDim + 1] = s4.x;
             dst[kHeadDim + 2] = s4.y;
             dst[kHeadDim + 3] = s4.z;
+            if constexpr (kValue) {
+                float vm = 0.f;
+                for (int w = 0; w < kWsPairs; ++w)
+                    vm = fmaxf(vm, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim + 5]);
+                dst[kHeadDim + 4] = s4.w;
+                dst[kHeadDim + 5] = vm;
+            }
         }
     }
 }
@@ -1065,6 +1122,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 // warp folds its splits with a running maximum in one pass.
 constexpr int kMergeWarps = 8;
 
+template <int kX>
 __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_constant__ DecodeParams p) {
     grid_dep_launch();   // the next kernel waits for this grid before reading its outputs
     grid_dep_wait();
@@ -1074,20 +1132,20 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     const size_t unit = (size_t)b * p.num_kv_heads + h;
     const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride) + hh * kPartialStride;
     const size_t split_stride = kMaxGroup * kPartialStride;
-    __shared__ float red[kMergeWarps][36];
+    __shared__ float red[kMergeWarps][38];
 
     // all of this warp's split rows of a round are loaded before any is
     // combined, so the loads overlap (one memory latency per round, not per split)
     constexpr int kMaxRows = 16;   // rows per warp and round
-    const bool tier_b = p.meter_b != nullptr;
-    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f;
+    constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0;
+    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f, Vt = 0.f, Vm = 0.f;
     for (int s0 = warp; s0 < p.splits; s0 += kMergeWarps * kMaxRows) {
-        float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows], dbs[kMaxRows];
+        float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows], dbs[kMaxRows], vts[kMaxRows];
 #pragma unroll
         for (int i = 0; i < kMaxRows; ++i) {
             const int s = s0 + i * kMergeWarps;
             ms[i] = -INFINITY;
-            v[i] = ls[i] = ds[i] = dbs[i] = 0.f;
+            v[i] = ls[i] = ds[i] = dbs[i] = vts[i] = 0.f;
             if (s < p.splits) {
                 const float* ps = base + s * split_stride;
                 ms[i] = __ldcg(ps + kHeadDim);
@@ -1095,6 +1153,10 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
                 ls[i] = __ldcg(ps + kHeadDim + 1);
                 ds[i] = __ldcg(ps + kHeadDim + 2);
                 if (tier_b) dbs[i] = __ldcg(ps + kHeadDim + 3);
+                if (vside) {
+                    vts[i] = __ldcg(ps + kHeadDim + 4);
+                    Vm = fmaxf(Vm, __ldcg(ps + kHeadDim + 5));
+                }
             }
         }
         float Mr = M;
@@ -1103,7 +1165,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
         if (Mr == -INFINITY) continue;
         if (Mr > M) {   // move the running sums to the new reference
             const float f = (M == -INFINITY) ? 0.f : fast_exp2(M - Mr);
-            acc *= f; L *= f; Dn *= f; Db *= f;
+            acc *= f; L *= f; Dn *= f; Db *= f; Vt *= f;
             M = Mr;
         }
 #pragma unroll
@@ -1114,6 +1176,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             L = fmaf(w, ls[i], L);
             Dn = fmaf(w, ds[i], Dn);
             Db = fmaf(w, dbs[i], Db);
+            Vt = fmaf(w, vts[i], Vt);
         }
     }
     red[warp][lane] = acc;
@@ -1122,13 +1185,17 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
         red[warp][33] = L;
         red[warp][34] = Dn;
         red[warp][35] = Db;
+        red[warp][36] = Vt;
+        red[warp][37] = Vm;
     }
     __syncthreads();
     if (warp == 0) {
         float Mt = -INFINITY;
 #pragma unroll
         for (int w = 0; w < kMergeWarps; ++w) Mt = fmaxf(Mt, red[w][32]);
-        float a = 0.f, l = 0.f, dn = 0.f, db = 0.f;
+        float a = 0.f, l = 0.f, dn = 0.f, db = 0.f, vt = 0.f, vm = 0.f;
+        if (vside)
+            for (int w = 0; w < kMergeWarps; ++w) vm = fmaxf(vm, red[w][37]);
         if (Mt != -INFINITY) {
 #pragma unroll
             for (int w = 0; w < kMergeWarps; ++w) {
@@ -1138,6 +1205,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
                 l = fmaf(f, red[w][33], l);
                 dn = fmaf(f, red[w][34], dn);
                 db = fmaf(f, red[w][35], db);
+                vt = fmaf(f, red[w][36], vt);
             }
         }
         const size_t cell = (size_t)b * p.num_q_heads + hq;
@@ -1158,6 +1226,12 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
                 }
                 p.meter_b_raw[cell] = rb;
                 p.meter_b[cell] = fminf(1.0f, rb);
+            }
+            if (vside) {   // ||y - y^|| <= 2 TV max ||v|| + sum p~ rho^v, TV <= meter
+                const float vterm = l > 0.f ? vt / l : 0.f;
+                p.value_term[cell] = vterm;
+                p.v_max[cell] = vm;
+                p.out_bound[cell] = 2.0f * fminf(1.0f, raw) * vm + vterm;
             }
         }
     }
@@ -1209,6 +1283,7 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
 // instead of packed onto the first few SMs to free up.
 constexpr int kMergeSpreadSmem = 118784;
 
+template <int kX>
 static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
     static std::once_flag once;
     static int num_sms = 0;   // 0: the spread request is not used
@@ -1216,39 +1291,39 @@ static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
         int dev = 0, n = 0;
         if (cudaGetDevice(&dev) == cudaSuccess &&
             cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
-            cudaFuncSetAttribute(merge_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSpreadSmem) ==
+            cudaFuncSetAttribute(merge_kernel<kX>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMergeSpreadSmem) ==
                 cudaSuccess)
             num_sms = n;
-        (void)cudaFuncSetAttribute(merge_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+        (void)cudaFuncSetAttribute(merge_kernel<kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                    (int)cudaSharedmemCarveoutMaxShared);
         (void)cudaGetLastError();   // a refused hint leaves no sticky error behind
     });
     const dim3 grid(kHeadDim / 32, p.num_q_heads, p.batch);
     const long ctas = (long)grid.x * grid.y * grid.z;
     const size_t smem = (num_sms > 0 && ctas <= num_sms) ? kMergeSpreadSmem : 0;
-    return launch_pdl(merge_kernel, grid, dim3(32 * kMergeWarps), smem, stream, p);
+    return launch_pdl(merge_kernel<kX>, grid, dim3(32 * kMergeWarps), smem, stream, p);
 }
 
-template <int kScheme, int kBits, bool kTierB>
+template <int kScheme, int kBits, int kX>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;   // per process; the attributes are per function
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kTierB>,
+        cudaError_t e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kX>,
                                              cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBytes);
         if (e != cudaSuccess) return e;
         // the library's kernels all prefer the largest shared-memory carveout,
         // so consecutive launches do not reconfigure the L1 / shared split
-        e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kTierB>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(decode_kernel<kScheme, kBits, kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
     }
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kTierB>, grid, dim3(kThreads), kSmemBytes, stream, p);
+    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kX>, grid, dim3(kThreads), kSmemBytes, stream, p);
     if (e != cudaSuccess) return e;
     // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
-    return launch_merge(p, stream);
+    return launch_merge<kX>(p, stream);
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (the
@@ -1282,14 +1357,14 @@ static bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, 
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <bool kTierB>
+template <int kX>
 static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;
     if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel<kTierB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel<kX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                              kWsSmemBytes);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(decode_ws_kernel<kTierB>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(decode_ws_kernel<kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -1300,18 +1375,25 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
         !encode_page_map(&wp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_ws_kernel<kTierB>, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
+    cudaError_t e = launch_pdl(decode_ws_kernel<kX>, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
-    return launch_merge(p, stream);
+    return launch_merge<kX>(p, stream);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.batch == 0) return cudaSuccess;
-    const bool tier_b = p.meter_b != nullptr;   // dithered INT8 only (checked by the caller)
-    if (scheme == WC_SCHEME_FP8_E4M3) return launch_one<WC_SCHEME_FP8_E4M3, 8, false>(p, stream);
-    if (use_ws(scheme, bits)) return tier_b ? launch_ws<true>(p, stream) : launch_ws<false>(p, stream);
-    return tier_b ? launch_one<WC_SCHEME_DITHER_INT8, 10, true>(p, stream)
-                  : launch_one<WC_SCHEME_DITHER_INT8, 10, false>(p, stream);
+    // Tier B (dithered INT8 only) and the value side are requested by separate
+    // entry points, never together (checked by the caller)
+    const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0);
+    if (scheme == WC_SCHEME_FP8_E4M3)
+        return x == kXValue ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
+                            : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
+    if (use_ws(scheme, bits))
+        return x == kXTierB ? launch_ws<kXTierB>(p, stream)
+             : x == kXValue ? launch_ws<kXValue>(p, stream) : launch_ws<0>(p, stream);
+    return x == kXTierB ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
+         : x == kXValue ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
+                        : launch_one<WC_SCHEME_DITHER_INT8, 10, 0>(p, stream);
 }
 
 }  // namespace wc

@@ -1,6 +1,8 @@
 // Gate (§6 meter-loop box; certified vs risk-ranked thresholds, §4.3):
 // keep the compressed path of a query-head cell iff meter_raw <= tau, and of
-// a KV head iff all of its G query heads keep (any-of-G fallback).
+// a KV head iff all of its G query heads keep (any-of-G fallback).  The joint
+// gate (§4.2 "Value side and the joint event") also requires the value term
+// to be at most tau_v * max ||v|| (pass_V), decided in float32.
 #include "wc_kernels.cuh"
 
 namespace wc {
@@ -9,16 +11,20 @@ namespace {
 
 constexpr int kGateThreads = 256;
 
-__global__ void __launch_bounds__(kGateThreads) gate_kernel(const float* __restrict__ meter_raw, int n_cells,
-                                                            int group, float tau, uint8_t* keep_q,
+__global__ void __launch_bounds__(kGateThreads) gate_kernel(const float* __restrict__ meter_raw,
+                                                            const float* __restrict__ value_term,
+                                                            const float* __restrict__ v_max, int n_cells,
+                                                            int group, float tau, float tau_v, uint8_t* keep_q,
                                                             uint8_t* keep_kv, int32_t* n_kept) {
     int kept_q = 0, kept_kv = 0;
     const int n_kv = n_cells / group;
     for (int i = threadIdx.x; i < n_kv; i += kGateThreads) {
         bool all = true;
         for (int j = 0; j < group; ++j) {
-            const bool k = meter_raw[(size_t)i * group + j] <= tau;   // NaN -> false
-            keep_q[(size_t)i * group + j] = k ? 1 : 0;
+            const size_t cell = (size_t)i * group + j;
+            bool k = meter_raw[cell] <= tau;                                    // NaN -> false
+            if (value_term) k = k && value_term[cell] <= __fmul_rn(tau_v, v_max[cell]);
+            keep_q[cell] = k ? 1 : 0;
             kept_q += k;
             all = all && k;
         }
@@ -49,8 +55,9 @@ __global__ void __launch_bounds__(kGateThreads) gate_kernel(const float* __restr
 
 }  // namespace
 
-cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float tau, uint8_t* keep_q,
-                        uint8_t* keep_kv, int32_t* n_kept, cudaStream_t stream) {
+cudaError_t launch_gate(const float* meter_raw, const float* value_term, const float* v_max, int n_cells, int group,
+                        float tau, float tau_v, uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept,
+                        cudaStream_t stream) {
     static bool configured = false;   // same carveout as the decode kernels
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(gate_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -58,7 +65,8 @@ cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float ta
         if (e != cudaSuccess) return e;
         configured = true;
     }
-    gate_kernel<<<1, kGateThreads, 0, stream>>>(meter_raw, n_cells, group, tau, keep_q, keep_kv, n_kept);
+    gate_kernel<<<1, kGateThreads, 0, stream>>>(meter_raw, value_term, v_max, n_cells, group, tau, tau_v, keep_q,
+                                                keep_kv, n_kept);
     return cudaGetLastError();
 }
 

@@ -16,6 +16,7 @@ struct WriteParams {
     __half* k_scale;
     __half* v_scale;
     __half* k_witness;
+    __half* v_witness;    // [slot][2] (rho^v, ||v||) rounded up, nullptr: not stored
     uint32_t* dev_status;
     int32_t n_tok, num_kv_heads, num_pages, layer, rope_layout;
     PhiloxKeys keys;
@@ -36,6 +37,10 @@ struct DecodeParams {
     float* meter_b;       // Tier-B meters (§4.2), nullptr: not computed
     float* meter_b_raw;
     float tb_log_2_over_delta;   // log(2 / delta_loc) for Tier B
+    const __half* v_witness;     // [slot][2] (rho^v, ||v||) for the value side
+    float* value_term;           // value side outputs, nullptr: not computed
+    float* v_max;
+    float* out_bound;
     uint32_t* status;     // workspace word
     uint32_t* counters;   // [batch * Hkv], zero between calls
     float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
@@ -44,8 +49,9 @@ struct DecodeParams {
     PhiloxKeys keys;
 };
 
-// Per (query head, split) partial: acc[128] | m | l | D | Tier-B D.
-constexpr int kPartialStride = kHeadDim + 4;
+// Per (query head, split) partial: acc[128] | m | l | D | Tier-B D | value
+// term | max ||v|| | pad.
+constexpr int kPartialStride = kHeadDim + 8;
 
 // Workspace layout (bytes): [0, 256) status word, then counters, then
 // partials, each 256-byte aligned.
@@ -76,7 +82,8 @@ inline cudaError_t launch_pdl(Kernel kernel, dim3 grid, dim3 block, size_t smem,
 
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
-cudaError_t launch_gate(const float* meter_raw, int n_cells, int group, float tau, uint8_t* keep_q,
-                        uint8_t* keep_kv, int32_t* n_kept, cudaStream_t stream);
+cudaError_t launch_gate(const float* meter_raw, const float* value_term, const float* v_max, int n_cells, int group,
+                        float tau, float tau_v, uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept,
+                        cudaStream_t stream);
 
 }  // namespace wc

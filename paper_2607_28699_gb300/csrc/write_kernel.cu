@@ -35,9 +35,10 @@ __device__ __forceinline__ float exact_round(float x, float s, float xi, float k
     return fminf(127.0f, fmaxf(-127.0f, k));
 }
 
-// Band norm for the witness, rounded up to fp16: the smallest fp16 h with
+// Norm for a witness, rounded up to fp16: the smallest fp16 h with
 // h * h >= S, S = sum inflated by 2^-18 (rounded up), which covers the fp32
-// accumulation error of the sum (< 2^-20 relative).  So h is never below the
+// accumulation error of the sum (a band: 16 squares, < 2^-20 relative; a
+// whole row: 128 squares in 16 FMAs and 3 shuffle adds per lane, < 2^-19.7).  So h is never below the
 // exact norm rounded up and at most one fp16 step above it.  h * h is exact in
 // fp32 (11 significant bits), so one check on each side of the rounded-up
 // approximate root fixes it.
@@ -83,7 +84,10 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
     }
 
     uint32_t codes[4];
-    float lo = 0.0f, hi = 0.0f;   // K rows: squared residual sums over dims 16*sub + [0,8), + [8,16)
+    // K rows, and V rows when the value witness is stored: squared residual
+    // sums over dims 16*sub + [0,8), + [8,16)
+    float lo = 0.0f, hi = 0.0f;
+    const bool resid = row == 0 || p.v_witness != nullptr;   // warp-uniform
     float s = 0.0f;
     if constexpr (kScheme == WC_SCHEME_DITHER_INT8) {
         float amax = 0.0f;
@@ -155,7 +159,7 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         };
         bool exact = need_clamp;
         if (!exact) {
-            const float dev = row == 0 ? fast_pass(std::true_type{}) : fast_pass(std::false_type{});
+            const float dev = resid ? fast_pass(std::true_type{}) : fast_pass(std::false_type{});
             exact = __any_sync(0xffffffffu, dev > 0.49998f);
         }
         if (exact) {
@@ -166,7 +170,7 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
                 const float est = fminf(127.0f, fmaxf(-127.0f, fmaf(x[i], inv_s, xi)));
                 const float k = exact_round(x[i], s, xi, (est + kBias) - kBias);
                 tb[i] = __float_as_uint(k + kBias);
-                if (row == 0) {
+                if (resid) {
                     const float r = fmaf(s, k - xi, -x[i]);
                     if (i < 8) lo = fmaf(r, r, lo);
                     else hi = fmaf(r, r, hi);
@@ -186,7 +190,7 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
             const uint32_t cc = (uint32_t)c2;   // low half -> low byte
             if ((i & 1) == 0) codes[i >> 1] = cc;
             else codes[i >> 1] |= cc << 16;
-            if (row == 0) {
+            if (resid) {
                 const uint32_t back = e4m3x2_to_h2(cc);
                 const float2 xr = __half22float2(*reinterpret_cast<const __half2*>(&back));
                 const float r0 = xr.x - x[2 * i], r1 = xr.y - x[2 * i + 1];
@@ -206,7 +210,23 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
             if (sub == 0) (row == 0 ? p.k_scale : p.v_scale)[rowidx] = __float2half_rn(s);
         }
     }
-    if (row != 0) return;   // warp-uniform
+    if (row != 0) {   // warp-uniform
+        if (p.v_witness != nullptr) {
+            // value witness (§3 output bound): ||v^ - v|| and ||v|| of the row, rounded up
+            float rr = lo + hi, vv = 0.0f;
+#pragma unroll
+            for (int i = 0; i < 16; ++i) vv = fmaf(x[i], x[i], vv);
+#pragma unroll
+            for (int o = 1; o < 8; o <<= 1) {
+                rr += __shfl_xor_sync(0xffffffffu, rr, o);
+                vv += __shfl_xor_sync(0xffffffffu, vv, o);
+            }
+            if (active && sub == 0)
+                *reinterpret_cast<__half2*>(p.v_witness + rowidx * 2) =
+                    __halves2half2(norm_up_fp16(rr), norm_up_fp16(vv));
+        }
+        return;
+    }
 
     // ---- witness (K warps) --------------------------------------------------
     const float lo_p = __shfl_xor_sync(0xffffffffu, lo, 4);

@@ -52,12 +52,16 @@ def gpu_cache_to_numpy(cache):
     if cache.k_scale is not None:
         out["k_scale"] = cache.k_scale.cpu().numpy()
         out["v_scale"] = cache.v_scale.cpu().numpy()
+    if cache.v_witness is not None:
+        out["v_witness"] = cache.v_witness.cpu().numpy()
     return out
 
 
-def numpy_cache_to_gpu(cache, desc_g):
+def numpy_cache_to_gpu(cache, desc_g, value_witness=False):
     import paper_2607_28699_gb300 as wc
-    c = wc.LayerCache.empty(desc_g)
+    c = wc.LayerCache.empty(desc_g, value_witness=value_witness)
+    if value_witness:
+        c.v_witness.copy_(torch.from_numpy(cache["v_witness"]))
     c.k_codes.copy_(torch.from_numpy(cache["k_codes"]))
     c.v_codes.copy_(torch.from_numpy(cache["v_codes"]))
     c.k_witness.copy_(torch.from_numpy(cache["k_witness"]))

@@ -69,3 +69,15 @@ def test_tier_b_host_validation_without_gpu(lib):
     for bad in (0.0, 1.0, -0.5, float("nan")):
         assert f(*args(int8, bad, dummy)) == 1 and b"delta_loc" in lib.wc_last_error()
     assert f(*args(int8, 0.01, None)) == 1 and b"meter_b" in lib.wc_last_error()
+
+
+def test_value_side_host_validation_without_gpu(lib):
+    import paper_2607_28699_gb300 as wc
+    d = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4).c()
+    assert lib.wc_kv_quantize_witness_v(ctypes.byref(d), 0, None, None, None, 0, None, None, None, None, None,
+                                        None, None, None) == 1 and b"v_witness" in lib.wc_last_error()
+    assert lib.wc_metered_decode_attention_v(ctypes.byref(d), 0, None, None, 1, None, 1, None, None, None, None,
+                                             None, None, None, None, None, None, None, None, None, 0,
+                                             None) == 1 and b"v_witness" in lib.wc_last_error()
+    assert lib.wc_gate_joint(None, None, None, 4, 2, ctypes.c_float(0.1), ctypes.c_float(0.1), None, None, None,
+                             None) == 1
