@@ -250,7 +250,7 @@ wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer
  *   dev_status  optional device uint32 that collects WC_DEV_* bits (OR); when
  *               NULL the bits go to a word inside the built-in scratch.
  * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
- * more scratch than 4 MiB (about 960 (sequence, KV head, split) partial
+ * more scratch than 4 MiB (about 930 (sequence, KV head, split) partial
  * results; the split count follows wc_workspace_size's plan).
  * The first call on each device looks up the scratch address and clears its
  * status word (a synchronous cudaMemset); make that first call before any

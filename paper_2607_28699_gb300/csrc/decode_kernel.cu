@@ -351,8 +351,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0; vt_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1; vt_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
+                if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -529,9 +531,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                if constexpr (kValue) {
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                }
             }
         }
     }
@@ -562,8 +566,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             } else {
                 s.x = fmaf(wt, src[0], s.x);   // l
                 s.y = fmaf(wt, src[1], s.y);   // D
-                s.z = fmaf(wt, src[2], s.z);   // Tier-B D
-                s.w = fmaf(wt, src[3], s.w);   // value term
+                if constexpr (kTierB) s.z = fmaf(wt, src[2], s.z);   // Tier-B D
+                if constexpr (kValue) s.w = fmaf(wt, src[3], s.w);   // value term
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -573,7 +577,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             dst[kHeadDim] = M;
             dst[kHeadDim + 1] = s.x;
             dst[kHeadDim + 2] = s.y;
-            dst[kHeadDim + 3] = s.z;
+            if constexpr (kTierB) dst[kHeadDim + 3] = s.z;
             if constexpr (kValue) {
                 float vm = 0.f;
                 for (int w = 0; w < kWarps; ++w)
@@ -924,8 +928,10 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                 if (mv0) m_run[0] = mx0;
                 if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0; db_part[0] *= a0; vt_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1; db_part[1] *= a1; vt_part[1] *= a1;
+                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
+                if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
 #pragma unroll
                 for (int mt = 0; mt < 8; ++mt) {
                     acc[mt][0] *= a0; acc[mt][2] *= a0;
@@ -1060,9 +1066,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
                 wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                if constexpr (kValue) {
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                }
             }
         }
     }
@@ -1092,8 +1100,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             } else {
                 s4.x = fmaf(wt, src[0], s4.x);
                 s4.y = fmaf(wt, src[1], s4.y);
-                s4.z = fmaf(wt, src[2], s4.z);
-                s4.w = fmaf(wt, src[3], s4.w);
+                if constexpr (kTierB) s4.z = fmaf(wt, src[2], s4.z);
+                if constexpr (kValue) s4.w = fmaf(wt, src[3], s4.w);
             }
         }
         float* dst = part_out + hh * kPartialStride;
@@ -1103,7 +1111,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             dst[kHeadDim] = M;
             dst[kHeadDim + 1] = s4.x;
             dst[kHeadDim + 2] = s4.y;
-            dst[kHeadDim + 3] = s4.z;
+            if constexpr (kTierB) dst[kHeadDim + 3] = s4.z;
             if constexpr (kValue) {
                 float vm = 0.f;
                 for (int w = 0; w < kWsPairs; ++w)

@@ -50,8 +50,10 @@ struct DecodeParams {
 };
 
 // Per (query head, split) partial: acc[128] | m | l | D | Tier-B D | value
-// term | max ||v|| | pad.
-constexpr int kPartialStride = kHeadDim + 8;
+// term | max ||v|| | pad.  140 floats: in the CTA merge's shared buffer the
+// rows of the heads one warp instruction touches then start in distinct bank
+// groups (12 words apart modulo 32; 136 would put two heads on each group).
+constexpr int kPartialStride = kHeadDim + 12;
 
 // Workspace layout (bytes): [0, 256) status word, then counters, then
 // partials, each 256-byte aligned.
