@@ -38,6 +38,13 @@ formula): pass_V holds when the value term sum_t p~_t rho^v_t is at most
 tau_V max_t ||v_t||, and the joint gate keeps a cell iff pass_K (meter_raw
 <= tau_K) and pass_V, both decided in float32.
 
+§6.4 "Block-level paging": the e-form certificate is block decomposable.
+With p~ held fixed, replacing page j's keys by their exact values sets c_t = 0
+for its tokens and lowers D = A - 1 by exactly C_j = sum_{t in j} p~_t
+expm1(c_t).  Paging in pages by decreasing C_j until 1/2 D (D + 2) <= tau
+uses the fewest pages (all C_j >= 0).  Reading: ties in C_j go to the lower
+logical page index.
+
 Gate (§6 meter-loop box; §4.3 certified vs risk-ranked): a (layer, head)
 falls back when its meter exceeds tau.  Reading: keep the compressed path
 iff meter_raw <= tau (so equality keeps, NaN falls back), evaluated in
@@ -167,3 +174,33 @@ def joint_gate(meter_raw, vterm, v_max, tau_k, tau_v, group):
         raise ValueError("cells must come in whole groups")
     keep_kv = np.all(keep_q.reshape(keep_q.shape[:-1] + (n // group, group)), axis=-1)
     return keep_q, keep_kv, int(np.sum(keep_q)), int(np.sum(keep_kv))
+
+
+def page_contributions(p_tilde, c, page_of_token, n_pages):
+    """C_j = sum over the tokens of logical page j of p~_t expm1(c_t)."""
+    p_tilde = np.asarray(p_tilde, np.float64)
+    with np.errstate(over="ignore", invalid="ignore"):
+        terms = p_tilde * np.expm1(np.asarray(c, np.float64))
+        terms = np.where(p_tilde == 0, 0.0, terms)      # as in eform_meter
+    return np.bincount(np.asarray(page_of_token, dtype=np.int64), weights=terms, minlength=n_pages)
+
+
+def repair_plan(contrib, tau):
+    """Fewest pages whose exact values bring the meter to tau or below.
+
+    Pages rank by decreasing C_j (NaN first, ties to the lower index); the
+    remaining excess after paging in the first k is R_k = the sum of the
+    contributions not yet paged in, and k is the least with
+    1/2 R_k (R_k + 2) <= tau (all pages when tau < 0).
+    Returns (pages in paging order, R_k).
+    """
+    C = np.asarray(contrib, np.float64)
+    n = len(C)
+    order = sorted(range(n), key=lambda j: (not np.isnan(C[j]), 0.0 if np.isnan(C[j]) else -C[j], j))
+    sorted_c = C[order]
+    # R[k] = sum(sorted_c[k:]), R[n] = 0
+    R = np.concatenate([np.cumsum(sorted_c[::-1])[::-1], [0.0]])
+    with np.errstate(invalid="ignore", over="ignore"):
+        ok = 0.5 * R * (R + 2.0) <= tau
+    k = int(np.argmax(ok)) if np.any(ok) else n
+    return [int(j) for j in order[:k]], float(R[k])

@@ -118,14 +118,16 @@ def reconstruct(desc, layer, kv_head, slots, cache):
 
 
 def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
-                    k_exact=None, v_exact=None, delta_loc=None):
+                    k_exact=None, v_exact=None, delta_loc=None, repair_tau=None):
     """metered_decode_attention for one sequence: q16 [Hq, d] post-RoPE.
 
     Returns a dict with float64 ``out`` [Hq, d], ``meter``/``meter_raw``
     [Hq]; with the exact fp16 keys/values [S, Hkv, d] also ``tv`` [Hq]
     (the true TV between exact and compressed attention) and
     ``out_exact`` [Hq, d]; with ``delta_loc`` (dithered INT8 only) also the
-    Tier-B meters ``meter_b``/``meter_b_raw`` [Hq] (§4.2).
+    Tier-B meters ``meter_b``/``meter_b_raw`` [Hq] (§4.2); with ``repair_tau``
+    also ``contrib`` [Hq, pages] (page contributions to D) and ``repair``
+    (per query head: the logical pages to page in, in order, §6.4).
     """
     G = desc.num_q_heads // desc.num_kv_heads
     d = desc.head_dim
@@ -135,6 +137,10 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
               "out_err"):
         res[k] = np.zeros(desc.num_q_heads)
     tier_b = delta_loc is not None
+    n_pages = (ctx_len + desc.page_size - 1) // desc.page_size
+    if repair_tau is not None:
+        res["contrib"] = np.zeros((desc.num_q_heads, n_pages))
+        res["repair"] = [None] * desc.num_q_heads
     if tier_b and desc.scheme != SCHEME_DITHER_INT8:
         raise ValueError("Tier B needs the dithered INT8 cache (a controlled quantizer)")
     page, off = slots // desc.page_size, slots % desc.page_size
@@ -147,6 +153,9 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
             c = M.tier_a_bound(q, w, desc.num_bands, desc.rope_layout)
             res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.eform_meter(p_tilde, c)
             res["out"][hq] = M.attend(p_tilde, vhat)
+            if repair_tau is not None:
+                res["contrib"][hq] = M.page_contributions(p_tilde, c, np.arange(ctx_len) // desc.page_size, n_pages)
+                res["repair"][hq] = M.repair_plan(res["contrib"][hq], repair_tau)[0]
             vw = cache["v_witness"][page, h, off].astype(np.float64)        # [S, 2]
             res["value_term"][hq] = M.value_term(p_tilde, vw[:, 0])
             res["v_max"][hq] = np.max(vw[:, 1]) if ctx_len else 0.0
