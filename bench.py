@@ -256,6 +256,34 @@ class Setup:
                 out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
                 meter_b=self.meter_b[layer], meter_b_raw=self.meter_b_raw[layer])
 
+    def decode_all_repair(self):
+        """The same calls emitting the per-page meter terms, the gate, then the
+        block-level repair selection of every cell the gate flagged (§6.4)."""
+        wc, wl = self.wc, self.wl
+        L, B, Hq = wl.n_layers, wl.batch, wl.n_q_heads
+        if not hasattr(self, "page_terms"):
+            f32, i32 = dict(dtype=torch.float32, device="cuda"), dict(dtype=torch.int32, device="cuda")
+            self.page_terms = torch.empty(L, B, Hq, wl.max_pages, 2, **f32)
+            self.softmax_norm = torch.empty(L, B, Hq, 2, **f32)
+            self.rep_pages = torch.empty(L, B, Hq, wl.max_pages, **i32)
+            self.n_rep = torch.empty(L, B, Hq, **i32)
+            self.d_after = torch.empty(L, B, Hq, **f32)
+        for layer in range(L):
+            wc.metered_decode_attention_repair(
+                self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer], self.ws,
+                out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
+                page_terms=self.page_terms[layer], softmax_norm=self.softmax_norm[layer])
+        wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
+        self.select_all()
+
+    def select_all(self):
+        L, B, Hq = self.wl.n_layers, self.wl.batch, self.wl.n_q_heads
+        keep = self.keep_q.view(L, B, Hq)
+        for layer in range(L):
+            self.wc.repair_select(self.page_terms[layer], self.softmax_norm[layer], self.ctx, self.tau,
+                                  keep_q=keep[layer], contrib=False, repair_pages=self.rep_pages[layer],
+                                  n_repair=self.n_rep[layer], d_after=self.d_after[layer])
+
     def launches_per_step(self):
         # per layer: write kernel, decode kernel, merge kernel; then one gate
         return 3 * self.wl.n_layers + 1
@@ -353,6 +381,32 @@ def run_ours(args, rank, world, local):
                   "delta_req": st.TIER_B_DELTA_REQ, "kept_frac_at_tau": float((mb <= st.tau).float().mean()),
                   "meter_b_raw_median": float(mb.median())}
 
+    # ---- the same calls emitting the repair terms, gate, repair selection (§6.4) ----
+    def graph_ms(fn, per):
+        g = capture(fn)
+        for _ in range(args.warmup):
+            g.replay()
+        torch.cuda.synchronize()
+        d0.record()
+        for _ in range(args.steps):
+            g.replay()
+        d1.record()
+        torch.cuda.synchronize()
+        return d0.elapsed_time(d1) / (args.steps * per)
+
+    rep_ms = graph_ms(st.decode_all_repair, wl.n_layers)        # decode + gate + selection, per layer
+    sel_ms = graph_ms(st.select_all, wl.n_layers)               # selection alone, per layer
+    flag = st.keep_q.view(st.n_rep.shape) == 0
+    n_pages = torch.tensor([(c + 15) // 16 for c in wl.ctx_lens], device="cuda").view(1, -1, 1).expand_as(st.n_rep)
+    nr = st.n_rep[flag].float()
+    repair = {"select_call_ms": sel_ms, "decode_gate_select_ms_per_layer": rep_ms,
+              "overhead_vs_plain_decode": rep_ms / dec_avg_ms - 1.0,
+              "flagged_cells": int(flag.sum()),
+              "pages_per_flagged_cell_median": float(nr.median()) if nr.numel() else 0.0,
+              "pages_per_flagged_cell_mean": float(nr.mean()) if nr.numel() else 0.0,
+              "page_in_frac_vs_whole_head": float(nr.sum() / n_pages[flag].float().sum()) if nr.numel() else 0.0,
+              "d_after_max": float(st.d_after[flag].max()) if nr.numel() else 0.0}
+
     kv_tokens_step = wl.kv_tokens
     value = kv_tokens_step * world / (ms / 1e3)
     algo_bytes = st.decode_bytes_per_launch()
@@ -390,6 +444,7 @@ def run_ours(args, rank, world, local):
         "decode_call_ms": dec_avg_ms,
         "tier_b": tier_b,
         "value_side": value_side,
+        "repair": repair,
         "roofline": {"kernel": ("decode_ws_kernel" if wl.scheme == 0 and args.dither_bits == 8 else "decode_kernel")
                                + " + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

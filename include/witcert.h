@@ -269,6 +269,62 @@ wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t
                                               uint32_t* dev_status, void* stream);
 
 /*
+ * Metered decode attention with the per-page terms of block-level repair
+ * selection (§6.4 "Block-level paging").  Same computation, arguments and
+ * outputs as wc_metered_decode_attention, plus for every sequence b, query
+ * head hq and logical page j < ceil(ctx_lens[b] / 16):
+ *   page_terms[b][hq][j]  = (m_j, d_j) fp32: page j's share of D = A - 1,
+ *                           d_j = sum_{t in j} 2^(y_t - m_j) (e^{c_t} - 1), summed
+ *                           against a reference m_j (y_t the logit in log2 units)
+ *   softmax_norm[b][hq]   = (M, L) fp32 with p~_t = 2^(y_t - M) / L
+ * so that page j contributes C_j = d_j 2^(m_j - M) / L to D.  Entries of
+ * pages at or past the context are not written; a page outside the pool (see
+ * WC_DEV_BAD_PAGE) gets (-inf, 0).  The outputs feed wc_repair_select.
+ *   page_terms    [batch][Hq][max_pages][2] fp32, device, 8-byte aligned
+ *   softmax_norm  [batch][Hq][2] fp32, device, 8-byte aligned
+ */
+wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t layer,
+                                             const void* q, const int32_t* block_table,
+                                             int32_t max_pages, const int32_t* ctx_lens,
+                                             int32_t batch,
+                                             const void* k_codes, const void* v_codes,
+                                             const void* k_scale, const void* v_scale,
+                                             const void* k_witness,
+                                             float* out, float* meter, float* meter_raw,
+                                             float* page_terms, float* softmax_norm,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream);
+
+/*
+ * Block-level repair selection (§6.4 "Block-level paging").  With p~ held
+ * fixed, paging in the exact keys of logical page j (witness 0) lowers D by
+ * exactly C_j, so the fewest pages that bring the meter to tau are the
+ * largest contributions.  For every cell (b, hq), with n = ceil(ctx_lens[b]/16):
+ *   contrib[b][hq][j]    = C_j, j < n (fp32; optional, NULL: not stored)
+ *   repair_pages[b][hq][0 .. k-1] = logical pages by decreasing C_j (ties to the
+ *                          lower page; a NaN contribution ranks first), where k
+ *                          is the least count with 1/2 R_k (R_k + 2) <= tau in fp32,
+ *                          R_k = the sum of the contributions not in the list;
+ *                          k = n when no count is enough (tau < 0 or NaN)
+ *   n_repair[b][hq]      = k;  d_after[b][hq] = R_k
+ * Cells with keep_q[cell] != 0 (the gate kept them) get k = 0 and
+ * d_after = D.  keep_q may be NULL: every cell is selected.  Entries of
+ * repair_pages past k are not written.  One CTA per cell; the sort holds
+ * max_pages 8-byte keys in shared memory, so max_pages <= 16384
+ * (WC_ERR_UNSUPPORTED above).
+ *   page_terms, softmax_norm  as written by wc_metered_decode_attention_repair
+ *   ctx_lens     [batch] int32 (as for the decode); keep_q [batch][Hq] uint8 or NULL
+ *   contrib      [batch][Hq][max_pages] fp32 or NULL; repair_pages [batch][Hq][max_pages]
+ *                int32; n_repair [batch][Hq] int32; d_after [batch][Hq] fp32 -- device
+ *   dev_status   optional device uint32 that collects WC_DEV_BAD_CTX (OR)
+ */
+wc_status wc_repair_select(const float* page_terms, const float* softmax_norm,
+                           const int32_t* ctx_lens, int32_t batch, int32_t num_q_heads,
+                           int32_t max_pages, const uint8_t* keep_q, float tau,
+                           float* contrib, int32_t* repair_pages, int32_t* n_repair,
+                           float* d_after, uint32_t* dev_status, void* stream);
+
+/*
  * Gate (§6 meter-loop box; certified tau < 1 vs risk-ranked tau >= 1, §4.3).
  *
  * keep_q[i] = (meter_raw[i] <= tau) in fp32 (equality keeps the compressed

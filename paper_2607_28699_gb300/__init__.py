@@ -33,6 +33,7 @@ DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT = 1, 2, 4, 8
 EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
            "wc_metered_decode_attention_tier_b", "wc_metered_decode_attention_noalloc",
            "wc_kv_quantize_witness_v", "wc_metered_decode_attention_v", "wc_gate_joint",
+           "wc_metered_decode_attention_repair", "wc_repair_select",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -68,6 +69,11 @@ def _load():
     lib.wc_metered_decode_attention_v.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp, vp,
                                                   vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
     lib.wc_metered_decode_attention_v.restype = ctypes.c_int
+    lib.wc_metered_decode_attention_repair.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp,
+                                                       vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.wc_metered_decode_attention_repair.restype = ctypes.c_int
+    lib.wc_repair_select.argtypes = [vp, vp, vp, i32, i32, i32, vp, ctypes.c_float, vp, vp, vp, vp, vp, vp]
+    lib.wc_repair_select.restype = ctypes.c_int
     lib.wc_read_status.argtypes = [vp, i32, vp, vp]
     lib.wc_read_status.restype = ctypes.c_int
     lib.wc_last_error.argtypes = []
@@ -261,6 +267,52 @@ def metered_decode_attention_v(desc: CacheDesc, layer: int, q: torch.Tensor, blo
         _ptr(cache.k_witness), _ptr(cache.v_witness), _ptr(out), _ptr(meter), _ptr(meter_raw),
         _ptr(value_term), _ptr(v_max), _ptr(out_bound), ws.ptr(), ws.nbytes, _stream(stream)))
     return out, meter, meter_raw, value_term, v_max, out_bound
+
+
+def metered_decode_attention_repair(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
+                                    ctx_lens: torch.Tensor, cache: LayerCache, ws: Workspace, out=None, meter=None,
+                                    meter_raw=None, page_terms=None, softmax_norm=None, stream=None):
+    """``wc_metered_decode_attention_repair``; returns (out, meter, meter_raw, page_terms [B,Hq,max_pages,2],
+    softmax_norm [B,Hq,2])."""
+    batch, max_pages = block_table.shape
+    dev = q.device
+    cells = (batch, desc.num_q_heads)
+    out = torch.empty(batch, desc.num_q_heads, desc.head_dim, dtype=torch.float32, device=dev) if out is None else out
+    meter = torch.empty(cells, dtype=torch.float32, device=dev) if meter is None else meter
+    meter_raw = torch.empty(cells, dtype=torch.float32, device=dev) if meter_raw is None else meter_raw
+    if page_terms is None:
+        page_terms = torch.empty(batch, desc.num_q_heads, max_pages, 2, dtype=torch.float32, device=dev)
+    if softmax_norm is None:
+        softmax_norm = torch.empty(batch, desc.num_q_heads, 2, dtype=torch.float32, device=dev)
+    d = desc.c()
+    _check(lib.wc_metered_decode_attention_repair(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(out), _ptr(meter), _ptr(meter_raw), _ptr(page_terms), _ptr(softmax_norm),
+        ws.ptr(), ws.nbytes, _stream(stream)))
+    return out, meter, meter_raw, page_terms, softmax_norm
+
+
+def repair_select(page_terms: torch.Tensor, softmax_norm: torch.Tensor, ctx_lens: torch.Tensor, tau: float,
+                  keep_q=None, contrib=True, repair_pages=None, n_repair=None, d_after=None, dev_status=None,
+                  stream=None):
+    """``wc_repair_select``; returns (contrib [B,Hq,max_pages] fp32 or None, repair_pages int32
+    [B,Hq,max_pages] (the first n_repair entries of a row are meaningful), n_repair int32 [B,Hq],
+    d_after fp32 [B,Hq]).  ``contrib=False`` skips storing the contributions."""
+    batch, num_q_heads, max_pages = page_terms.shape[:3]
+    dev = page_terms.device
+    if contrib is True:
+        contrib = torch.zeros(batch, num_q_heads, max_pages, dtype=torch.float32, device=dev)
+    elif contrib is False:
+        contrib = None
+    if repair_pages is None:
+        repair_pages = torch.full((batch, num_q_heads, max_pages), -1, dtype=torch.int32, device=dev)
+    n_repair = torch.empty(batch, num_q_heads, dtype=torch.int32, device=dev) if n_repair is None else n_repair
+    d_after = torch.empty(batch, num_q_heads, dtype=torch.float32, device=dev) if d_after is None else d_after
+    _check(lib.wc_repair_select(_ptr(page_terms), _ptr(softmax_norm), _ptr(ctx_lens), batch, num_q_heads, max_pages,
+                                _ptr(keep_q), float(tau), _ptr(contrib), _ptr(repair_pages), _ptr(n_repair),
+                                _ptr(d_after), _ptr(dev_status), _stream(stream)))
+    return contrib, repair_pages, n_repair, d_after
 
 
 def gate_joint(meter_raw: torch.Tensor, value_term: torch.Tensor, v_max: torch.Tensor, group: int, tau_k: float,

@@ -158,9 +158,18 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
                                        const void* k_scale, const void* v_scale, const void* k_witness,
                                        float* out, float* meter, float* meter_raw, float* meter_b,
                                        float* meter_b_raw, double delta_loc, const void* v_witness,
-                                       float* value_term, float* v_max, float* out_bound, void* workspace,
-                                       size_t workspace_bytes, void* stream) {
+                                       float* value_term, float* v_max, float* out_bound, float* page_terms,
+                                       float* softmax_norm, void* workspace, size_t workspace_bytes,
+                                       void* stream) {
     if (wc_status st = check_desc(desc)) return st;
+    if (page_terms || softmax_norm) {
+        if (!page_terms || !softmax_norm)
+            return fail(WC_ERR_INVALID_ARG, "page_terms and softmax_norm must not be NULL");
+        if ((reinterpret_cast<uintptr_t>(page_terms) & 7u) || (reinterpret_cast<uintptr_t>(softmax_norm) & 7u))
+            return fail(WC_ERR_INVALID_ARG, "page_terms and softmax_norm must be 8-byte aligned");
+        if (meter_b || value_term)
+            return fail(WC_ERR_UNSUPPORTED, "the repair terms, Tier B and the value side are separate calls");
+    }
     if (value_term || v_max || out_bound || v_witness) {
         if (!value_term || !v_max || !out_bound || !v_witness)
             return fail(WC_ERR_INVALID_ARG, "v_witness, value_term, v_max and out_bound must not be NULL");
@@ -210,6 +219,8 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.value_term = value_term;
     p.v_max = v_max;
     p.out_bound = out_bound;
+    p.page_terms = reinterpret_cast<float2*>(page_terms);
+    p.softmax_norm = reinterpret_cast<float2*>(softmax_norm);
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
@@ -236,7 +247,7 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
                                       size_t workspace_bytes, void* stream) {
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
-                                 nullptr, nullptr, workspace, workspace_bytes, stream);
+                                 nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream);
 }
 
 wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t layer, const void* q,
@@ -249,7 +260,8 @@ wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t 
     if (!meter_b || !meter_b_raw) return fail(WC_ERR_INVALID_ARG, "meter_b and meter_b_raw must not be NULL");
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, meter_b, meter_b_raw, delta_loc,
-                                 nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream);
+                                 nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes,
+                                 stream);
 }
 
 wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer, const void* q,
@@ -263,7 +275,55 @@ wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer
         return fail(WC_ERR_INVALID_ARG, "v_witness, value_term, v_max and out_bound must not be NULL");
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, v_witness,
-                                 value_term, v_max, out_bound, workspace, workspace_bytes, stream);
+                                 value_term, v_max, out_bound, nullptr, nullptr, workspace, workspace_bytes, stream);
+}
+
+wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                             const int32_t* block_table, int32_t max_pages,
+                                             const int32_t* ctx_lens, int32_t batch, const void* k_codes,
+                                             const void* v_codes, const void* k_scale, const void* v_scale,
+                                             const void* k_witness, float* out, float* meter, float* meter_raw,
+                                             float* page_terms, float* softmax_norm, void* workspace,
+                                             size_t workspace_bytes, void* stream) {
+    if (!page_terms || !softmax_norm)
+        return fail(WC_ERR_INVALID_ARG, "page_terms and softmax_norm must not be NULL");
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
+                                 nullptr, nullptr, page_terms, softmax_norm, workspace, workspace_bytes, stream);
+}
+
+wc_status wc_repair_select(const float* page_terms, const float* softmax_norm, const int32_t* ctx_lens,
+                           int32_t batch, int32_t num_q_heads, int32_t max_pages, const uint8_t* keep_q, float tau,
+                           float* contrib, int32_t* repair_pages, int32_t* n_repair, float* d_after,
+                           uint32_t* dev_status, void* stream) {
+    if (batch < 0 || batch > 65535) return fail(WC_ERR_INVALID_ARG, "batch must be in [0, 65535] (got %d)", batch);
+    if (num_q_heads < 1 || num_q_heads > 65535)
+        return fail(WC_ERR_INVALID_ARG, "num_q_heads must be in [1, 65535] (got %d)", num_q_heads);
+    if (max_pages < 1) return fail(WC_ERR_INVALID_ARG, "max_pages must be positive (got %d)", max_pages);
+    if (max_pages > wc::kRepairMaxPages)
+        return fail(WC_ERR_UNSUPPORTED, "max_pages must be at most %d (got %d)", wc::kRepairMaxPages, max_pages);
+    if (batch == 0) return WC_OK;
+    if (!page_terms || !softmax_norm || !ctx_lens || !repair_pages || !n_repair || !d_after)
+        return fail(WC_ERR_INVALID_ARG,
+                    "page_terms, softmax_norm, ctx_lens, repair_pages, n_repair, d_after must not be NULL");
+    if ((reinterpret_cast<uintptr_t>(page_terms) & 7u) || (reinterpret_cast<uintptr_t>(softmax_norm) & 7u))
+        return fail(WC_ERR_INVALID_ARG, "page_terms and softmax_norm must be 8-byte aligned");
+    wc::RepairParams p;
+    p.page_terms = reinterpret_cast<const float2*>(page_terms);
+    p.softmax_norm = reinterpret_cast<const float2*>(softmax_norm);
+    p.ctx_lens = ctx_lens;
+    p.keep_q = keep_q;
+    p.contrib = contrib;
+    p.repair_pages = repair_pages;
+    p.n_repair = n_repair;
+    p.d_after = d_after;
+    p.status = dev_status;
+    p.batch = batch;
+    p.num_q_heads = num_q_heads;
+    p.max_pages = max_pages;
+    p.tau = tau;
+    cudaError_t e = wc::launch_repair_select(p, static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "repair selection kernel launch");
 }
 
 static wc_status gate_impl(const float* meter_raw, const float* value_term, const float* v_max, int32_t n_cells,

@@ -45,6 +45,7 @@ constexpr int kSmemBytes = kWarps * kStages * kStageStride + kWarps * kStages * 
 // Extra outputs compiled into a decode kernel (template bit mask).
 constexpr int kXTierB = 1;   // Tier-B meter (§4.2)
 constexpr int kXValue = 2;   // value-side witness terms and output bound (§3, §4.2)
+constexpr int kXRepair = 4;  // per-page meter terms for block-level repair selection (§6.4)
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRsd = 0.08838834764831845f;                      // 1/sqrt(128)
 constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;
@@ -85,9 +86,34 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
     return y;
 }
 
+// §6.4 "Block-level paging": the share of D of logical page lp for this
+// thread's softmax heads 2c, 2c+1, kept against the running maximum it was
+// summed under; with the final (M, L) the page contributes d 2^(m - M) / L.
+// dpg holds the thread's tokens g, g+8 on entry; the sum runs over the rows g.
+__device__ __forceinline__ void emit_page_terms(const DecodeParams& p, int b, int h, int G, int lp, int g, int c,
+                                                float (&dpg)[2], const float (&m_run)[2]) {
+#pragma unroll
+    for (int o = 4; o < 32; o <<= 1) {
+        dpg[0] += __shfl_xor_sync(0xffffffffu, dpg[0], o);
+        dpg[1] += __shfl_xor_sync(0xffffffffu, dpg[1], o);
+    }
+    if (g == 0) {
+        float2* dst = p.page_terms + ((size_t)b * p.num_q_heads + (size_t)h * G) * p.max_pages + lp;
+        if (2 * c < G) dst[(size_t)(2 * c) * p.max_pages] = make_float2(m_run[0], dpg[0]);
+        if (2 * c + 1 < G) dst[(size_t)(2 * c + 1) * p.max_pages] = make_float2(m_run[1], dpg[1]);
+    }
+}
+
+// A page the kernel could not read (outside the pool) contributes nothing.
+__device__ __forceinline__ void emit_skipped_page(const DecodeParams& p, int b, int h, int G, int lp, int lane) {
+    if (lane < G)
+        p.page_terms[((size_t)b * p.num_q_heads + (size_t)h * G + lane) * p.max_pages + lp] =
+            make_float2(-INFINITY, 0.f);
+}
+
 template <int kScheme, int kBits, int kX>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecodeParams p) {
-    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0;
+    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
     extern __shared__ __align__(128) uint8_t smem[];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
@@ -361,18 +387,22 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                     acc[mt][1] *= a1; acc[mt][3] *= a1;
                 }
             }
+            float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = i >> 1, e = i & 1;
                 const float pe = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
                 l_part[e] += pe;
-                d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
+                d_part[e] = fmaf(pe, em1, d_part[e]);
+                if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
                 if constexpr (kTierB)
                     db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                 if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
+            if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
             if constexpr (kInt8) {
                 const float smax = fmaxf(sv[0], sv[1]);
                 const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
@@ -480,6 +510,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                     mma16816(acc[mt], A, bl0, bl1);
                 }
             }
+        } else if constexpr (kRepair) {
+            emit_skipped_page(p, b, h, G, lp, lane);
         }
         __syncwarp();
         issue(k + kStages, phys_issue);
@@ -661,7 +693,7 @@ __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h,
 
 template <int kX>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
-    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0;
+    constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -938,18 +970,22 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                     acc[mt][1] *= a1; acc[mt][3] *= a1;
                 }
             }
+            float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = i >> 1, e = i & 1;
                 const float pe = fast_exp2(y[i] - m_run[e]);
                 l_part[e] += pe;
-                d_part[e] = fmaf(pe, fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
+                d_part[e] = fmaf(pe, em1, d_part[e]);
+                if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
                 if constexpr (kTierB)
                     db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                 if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
             }
+            if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
             {
                 const float smax = fmaxf(sv[0], sv[1]);
                 const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
@@ -1023,6 +1059,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                     mma16816(acc[mt], H, bm0, bm1);
                 }
             }
+        } else if constexpr (kRepair) {
+            emit_skipped_page(p, b, h, G, lp, lane);
         }
         __syncwarp();
         if (lane == 0)   // release the stage to the producer
@@ -1145,7 +1183,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     // all of this warp's split rows of a round are loaded before any is
     // combined, so the loads overlap (one memory latency per round, not per split)
     constexpr int kMaxRows = 16;   // rows per warp and round
-    constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0;
+    constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0, repair = (kX & kXRepair) != 0;
     float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f, Vt = 0.f, Vm = 0.f;
     for (int s0 = warp; s0 < p.splits; s0 += kMergeWarps * kMaxRows) {
         float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows], dbs[kMaxRows], vts[kMaxRows];
@@ -1226,6 +1264,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             }
             p.meter_raw[cell] = raw;
             p.meter[cell] = fminf(1.0f, raw);
+            if (repair) p.softmax_norm[cell] = make_float2(Mt, l);
             if (tier_b) {
                 float rb = 0.f;
                 if (l > 0.f) {
@@ -1390,18 +1429,21 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.batch == 0) return cudaSuccess;
-    // Tier B (dithered INT8 only) and the value side are requested by separate
-    // entry points, never together (checked by the caller)
-    const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0);
+    // Tier B (dithered INT8 only), the value side and the repair terms are
+    // requested by separate entry points, never together (checked by the caller)
+    const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0) | (p.page_terms ? kXRepair : 0);
     if (scheme == WC_SCHEME_FP8_E4M3)
-        return x == kXValue ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
-                            : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
+        return x == kXValue  ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
+             : x == kXRepair ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXRepair>(p, stream)
+                             : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
     if (use_ws(scheme, bits))
-        return x == kXTierB ? launch_ws<kXTierB>(p, stream)
-             : x == kXValue ? launch_ws<kXValue>(p, stream) : launch_ws<0>(p, stream);
-    return x == kXTierB ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
-         : x == kXValue ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
-                        : launch_one<WC_SCHEME_DITHER_INT8, 10, 0>(p, stream);
+        return x == kXTierB  ? launch_ws<kXTierB>(p, stream)
+             : x == kXValue  ? launch_ws<kXValue>(p, stream)
+             : x == kXRepair ? launch_ws<kXRepair>(p, stream) : launch_ws<0>(p, stream);
+    return x == kXTierB  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
+         : x == kXValue  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
+         : x == kXRepair ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXRepair>(p, stream)
+                         : launch_one<WC_SCHEME_DITHER_INT8, 10, 0>(p, stream);
 }
 
 }  // namespace wc

@@ -41,6 +41,12 @@ struct DecodeParams {
     float* value_term;           // value side outputs, nullptr: not computed
     float* v_max;
     float* out_bound;
+    // Block-level repair selection (§6.4), nullptr: not emitted.  Per page j of
+    // each (sequence, query head): (m_j, d_j), the page's share of D summed
+    // against the running maximum m_j, so that it contributes d_j 2^(m_j - M) / L;
+    // per (sequence, query head): (M, L), the final log2-domain maximum and sum.
+    float2* page_terms = nullptr;     // [batch][Hq][max_pages]
+    float2* softmax_norm = nullptr;   // [batch][Hq]
     uint32_t* status;     // workspace word
     uint32_t* counters;   // [batch * Hkv], zero between calls
     float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
@@ -82,8 +88,27 @@ inline cudaError_t launch_pdl(Kernel kernel, dim3 grid, dim3 block, size_t smem,
     return cudaLaunchKernelEx(&cfg, kernel, p);
 }
 
+struct RepairParams {
+    const float2* page_terms;     // [batch][Hq][max_pages] (m_j, d_j)
+    const float2* softmax_norm;   // [batch][Hq] (M, L)
+    const int32_t* ctx_lens;
+    const uint8_t* keep_q;        // [batch][Hq], nullptr: every cell is repaired
+    float* contrib;               // [batch][Hq][max_pages] C_j, nullptr: not stored
+    int32_t* repair_pages;        // [batch][Hq][max_pages] logical pages in paging order
+    int32_t* n_repair;            // [batch][Hq]
+    float* d_after;               // [batch][Hq] D left after the listed pages
+    uint32_t* status;             // optional device word, WC_DEV_BAD_CTX
+    int32_t batch, num_q_heads, max_pages;
+    float tau;
+};
+
+// Largest block-table width the selection handles (its sort holds one cell's
+// pages in shared memory).
+constexpr int kRepairMaxPages = 16384;
+
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
+cudaError_t launch_repair_select(const RepairParams& p, cudaStream_t stream);
 cudaError_t launch_gate(const float* meter_raw, const float* value_term, const float* v_max, int n_cells, int group,
                         float tau, float tau_v, uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept,
                         cudaStream_t stream);

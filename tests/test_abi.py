@@ -81,3 +81,25 @@ def test_value_side_host_validation_without_gpu(lib):
                                              None) == 1 and b"v_witness" in lib.wc_last_error()
     assert lib.wc_gate_joint(None, None, None, 4, 2, ctypes.c_float(0.1), ctypes.c_float(0.1), None, None, None,
                              None) == 1
+
+
+def test_repair_host_validation_without_gpu(lib):
+    import paper_2607_28699_gb300 as wc
+    d = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4).c()
+    vp = ctypes.c_void_p
+    args = lambda pt, sn: (ctypes.byref(d), 0, None, None, 1, None, 1, None, None, None, None, None,
+                           None, None, None, pt, sn, None, 0, None)
+    assert lib.wc_metered_decode_attention_repair(*args(None, vp(16))) == 1
+    assert b"page_terms" in lib.wc_last_error()
+    assert lib.wc_metered_decode_attention_repair(*args(vp(4), vp(16))) == 1
+    assert b"8-byte aligned" in lib.wc_last_error()
+    f = ctypes.c_float(0.1)
+    sel = lambda batch, hq, mp, pt=vp(16), sn=vp(16), rp=vp(16): lib.wc_repair_select(
+        pt, sn, vp(16), batch, hq, mp, None, f, None, rp, vp(16), vp(16), None, None)
+    assert sel(1, 8, 16385) == 2 and b"16384" in lib.wc_last_error()
+    assert sel(1, 8, 0) == 1
+    assert sel(1, 0, 4) == 1
+    assert sel(-1, 8, 4) == 1
+    assert sel(0, 8, 4) == 0                      # nothing to select, nothing launched
+    assert sel(1, 8, 4, rp=None) == 1 and b"repair_pages" in lib.wc_last_error()
+    assert sel(1, 8, 4, sn=vp(12)) == 1 and b"aligned" in lib.wc_last_error()
