@@ -256,7 +256,7 @@ class Setup:
                 out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
                 meter_b=self.meter_b[layer], meter_b_raw=self.meter_b_raw[layer])
 
-    def decode_all_repair(self):
+    def decode_all_repair(self, select=True):
         """The same calls emitting the per-page meter terms, the gate, then the
         block-level repair selection of every cell the gate flagged (§6.4)."""
         wc, wl = self.wc, self.wl
@@ -273,16 +273,20 @@ class Setup:
                 self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer], self.ws,
                 out=self.out[layer], meter=self.meter[layer], meter_raw=self.raw[layer],
                 page_terms=self.page_terms[layer], softmax_norm=self.softmax_norm[layer])
-        wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
-        self.select_all()
+        if select:
+            wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
+            self.select_all()
 
     def select_all(self):
-        L, B, Hq = self.wl.n_layers, self.wl.batch, self.wl.n_q_heads
-        keep = self.keep_q.view(L, B, Hq)
-        for layer in range(L):
-            self.wc.repair_select(self.page_terms[layer], self.softmax_norm[layer], self.ctx, self.tau,
-                                  keep_q=keep[layer], contrib=False, repair_pages=self.rep_pages[layer],
-                                  n_repair=self.n_rep[layer], d_after=self.d_after[layer])
+        """One selection call for the cells of all layers: layers stacked along
+        the batch dimension, each row with its sequence's context length."""
+        L, B, Hq, P = self.wl.n_layers, self.wl.batch, self.wl.n_q_heads, self.wl.max_pages
+        if not hasattr(self, "ctx_rows"):
+            self.ctx_rows = self.ctx.repeat(L)
+        self.wc.repair_select(self.page_terms.view(L * B, Hq, P, 2), self.softmax_norm.view(L * B, Hq, 2),
+                              self.ctx_rows, self.tau, keep_q=self.keep_q, contrib=False,
+                              repair_pages=self.rep_pages.view(L * B, Hq, P), n_repair=self.n_rep.view(L * B, Hq),
+                              d_after=self.d_after.view(L * B, Hq))
 
     def launches_per_step(self):
         # per layer: write kernel, decode kernel, merge kernel; then one gate
@@ -394,12 +398,15 @@ def run_ours(args, rank, world, local):
         torch.cuda.synchronize()
         return d0.elapsed_time(d1) / (args.steps * per)
 
+    terms_ms = graph_ms(lambda: st.decode_all_repair(select=False), wl.n_layers)   # decode with the terms
     rep_ms = graph_ms(st.decode_all_repair, wl.n_layers)        # decode + gate + selection, per layer
-    sel_ms = graph_ms(st.select_all, wl.n_layers)               # selection alone, per layer
+    sel_ms = graph_ms(st.select_all, wl.n_layers)               # selection alone (one call), per layer
     flag = st.keep_q.view(st.n_rep.shape) == 0
     n_pages = torch.tensor([(c + 15) // 16 for c in wl.ctx_lens], device="cuda").view(1, -1, 1).expand_as(st.n_rep)
     nr = st.n_rep[flag].float()
-    repair = {"select_call_ms": sel_ms, "decode_gate_select_ms_per_layer": rep_ms,
+    repair = {"decode_call_ms": terms_ms, "decode_overhead_vs_plain": terms_ms / dec_avg_ms - 1.0,
+              "select_ms_per_layer": sel_ms, "select_launches_per_step": 1,
+              "decode_gate_select_ms_per_layer": rep_ms,
               "overhead_vs_plain_decode": rep_ms / dec_avg_ms - 1.0,
               "flagged_cells": int(flag.sum()),
               "pages_per_flagged_cell_median": float(nr.median()) if nr.numel() else 0.0,

@@ -307,8 +307,10 @@ wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t 
  *                          R_k = the sum of the contributions not in the list;
  *                          k = n when no count is enough (tau < 0 or NaN)
  *   n_repair[b][hq]      = k;  d_after[b][hq] = R_k
- * Cells with keep_q[cell] != 0 (the gate kept them) get k = 0 and
- * d_after = D.  keep_q may be NULL: every cell is selected.  Entries of
+ * Cells of several layers can be selected in one call by stacking them along
+ * batch (the layouts are contiguous over [layer][batch]; ctx_lens then holds
+ * one entry per stacked row).  Cells with keep_q[cell] != 0 (the gate kept
+ * them) get k = 0 and d_after = D.  keep_q may be NULL: every cell is selected.  Entries of
  * repair_pages past k are not written.  One CTA per cell; the sort holds
  * max_pages 8-byte keys in shared memory, so max_pages <= 16384
  * (WC_ERR_UNSUPPORTED above).

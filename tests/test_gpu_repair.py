@@ -161,3 +161,25 @@ def test_selection_short_context_and_kept_cells():
     assert d_after.cpu().numpy()[0] == pytest.approx([0.01, 0.26], rel=1e-6)
     assert contrib[0, 0, :3].cpu().tolist() == pytest.approx([0.05, 0.2, 0.01])
     assert np.all(contrib[0, :, 3:].cpu().numpy() == 0)          # past the context: not written
+
+
+def test_layers_stacked_along_batch_select_as_separate_calls():
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("s", 2, 8, 2, [700, 160, 33], shuffle_pages=True, seed=13)
+    od, gd = descs(wl.n_q_heads, wl.n_kv_heads, wl.num_pages, 0, 8, 0, 3)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    terms, norms, raws = [], [], []
+    for layer in range(2):
+        bt, sm, k, v, q = make_inputs(wl, layer)
+        cache = wc.LayerCache.empty(gd)
+        wc.kv_quantize_witness(gd, layer, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
+        res = wc.metered_decode_attention_repair(gd, layer, q.cuda(), torch.from_numpy(bt).cuda(), ctx, cache, ws)
+        terms.append(res[3]); norms.append(res[4]); raws.append(res[2])
+    tau = float(torch.cat(raws).median()) * 0.5
+    stacked = wc.repair_select(torch.cat(terms), torch.cat(norms), ctx.repeat(2), tau)
+    for layer in range(2):
+        single = wc.repair_select(terms[layer], norms[layer], ctx, tau)
+        rows = slice(layer * wl.batch, (layer + 1) * wl.batch)
+        for a, b in zip(stacked, single):
+            assert torch.equal(a[rows], b)
