@@ -28,7 +28,9 @@ sqrt(2 varsigma_t^2 log(2S / delta_loc)); u_t then replaces c_t in the
 e-form meter.  Here the scale is one stored fp16 value per (token, KV head)
 (§6.2.2 per-token granularity), so varsigma_t^2 = ||q||^2 s_t^2 / (12 d).
 The guarantee is probabilistic and holds for non-adaptive queries (§4.2
-"Scope of the probabilistic guarantee").
+"Scope of the probabilistic guarantee").  With grouped scales (§6.2.3) the
+scale of channel c is its group's, and a bypassed channel is exact, so it
+carries no error: varsigma_t^2 = (1/(12 d)) sum_{c not bypassed} q_c^2 s_{g(c),t}^2.
 
 §3 output propagation and §4.2 "Value side and the joint event": with
 rho^v_t = ||v^_t - v_t||, ||y - y^|| <= 2 TV max_t ||v_t|| + sum_t p~_t rho^v_t;
@@ -122,6 +124,21 @@ def tier_b_bound(q, s, ctx_len, delta_loc):
     d = q.shape[-1]
     s = np.asarray(s, dtype=np.float64)
     var = np.sum(q * q, axis=-1)[..., None] * s * s / (12.0 * d)
+    return np.sqrt(2.0 * var * np.log(2.0 * ctx_len / delta_loc))
+
+
+def tier_b_bound_grouped(q, s_groups, group, excluded, ctx_len, delta_loc):
+    """u_t with grouped scales and bypassed channels (exact, no error).
+
+    q: [d]; s_groups: [S, d / group] stored fp16 group scales; excluded: the
+    bypassed dims; returns [S].
+    """
+    q = np.asarray(q, dtype=np.float64).copy()
+    d = q.shape[-1]
+    q[np.asarray(excluded, dtype=np.int64)] = 0.0
+    qn2 = np.sum((q * q).reshape(d // group, group), axis=-1)            # [G]
+    sg = np.asarray(s_groups, dtype=np.float64)
+    var = (sg * sg) @ qn2 / (12.0 * d)
     return np.sqrt(2.0 * var * np.log(2.0 * ctx_len / delta_loc))
 
 

@@ -10,6 +10,11 @@ P = page_size; per layer the arrays are
   k_scale, v_scale  [num_pages, Hkv, P]      fp16 (dither scheme only)
   k_witness         [num_pages, Hkv, P, B]   fp16
 
+and for the grouped scheme (§6.2.3) k_scale, v_scale [num_pages, Hkv, P, d/G_c]
+(one per channel group), k_bypass [num_pages, Hkv, P, 2m] fp16 (the exact
+values of the m bypassed RoPE pairs, pair by pair) and bypass_pairs [Hkv, m],
+the layer's fixed pair set per KV head.
+
 The meter loop (§6 box): write path quantizes k -> k^ and stores the
 witness; the read path computes the compressed attention and
 A = sum_t p~_t e^{c_t}; meter = min(1, 1/2 (A^2 - 1)); the gate compares it
@@ -26,6 +31,7 @@ from . import fp, philox, quantizer
 
 SCHEME_DITHER_INT8 = 0
 SCHEME_FP8_E4M3 = 1
+SCHEME_DITHER_INT8_G32 = 2     # grouped scales + fixed-channel outlier bypass (§6.2.3)
 
 
 @dataclass
@@ -40,11 +46,13 @@ class Desc:
     rope_layout: int = quantizer.ROPE_HALF
     dither_bits: int = 8
     seed: int = 0
+    group_channels: int = 32      # G_c, grouped scheme
+    num_bypass_pairs: int = 0     # m, grouped scheme
 
 
 def empty_cache(desc):
     shp = (desc.num_pages, desc.num_kv_heads, desc.page_size)
-    code_t = np.int8 if desc.scheme == SCHEME_DITHER_INT8 else np.uint8
+    code_t = np.uint8 if desc.scheme == SCHEME_FP8_E4M3 else np.int8
     cache = {
         "k_codes": np.zeros(shp + (desc.head_dim,), code_t),
         "v_codes": np.zeros(shp + (desc.head_dim,), code_t),
@@ -54,14 +62,41 @@ def empty_cache(desc):
     if desc.scheme == SCHEME_DITHER_INT8:
         cache["k_scale"] = np.zeros(shp, np.float16)
         cache["v_scale"] = np.zeros(shp, np.float16)
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        ng = desc.head_dim // desc.group_channels
+        cache["k_scale"] = np.zeros(shp + (ng,), np.float16)
+        cache["v_scale"] = np.zeros(shp + (ng,), np.float16)
+        cache["k_bypass"] = np.zeros(shp + (2 * desc.num_bypass_pairs,), np.float16)
+        cache["bypass_pairs"] = np.zeros((desc.num_kv_heads, desc.num_bypass_pairs), np.int64)
     return cache
 
 
-def quantize_rows(desc, layer, kv_head, rows16, slots, tag):
+def _excluded(desc, cache, kv_head, tag):
+    """Bypassed dims of a KV head: keys only (tag 0)."""
+    if tag != 0 or desc.num_bypass_pairs == 0:
+        return np.zeros(0, np.int64)
+    return quantizer.bypass_dims(cache["bypass_pairs"][kv_head], desc.head_dim, desc.rope_layout)
+
+
+def quantize_rows(desc, layer, kv_head, rows16, slots, tag, excluded=()):
     """Quantize fp16 rows [n, d] written to ``slots``.
 
-    Returns (codes, scale or None, reconstruction float64 [n, d]).
+    Returns (codes, scale or None, reconstruction float64 [n, d]); ``excluded``
+    are the bypassed dims of the grouped scheme (exact, code 0).
     """
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        G = desc.group_channels
+        s = quantizer.group_scales(rows16, G, excluded)
+        s_chan = np.repeat(s, G, axis=-1)
+        j = philox.dither_integers(desc.seed, layer, kv_head, slots, tag,
+                                   desc.head_dim, desc.dither_bits)
+        xi = philox.dither_values(j, desc.dither_bits)
+        code = quantizer.dither_code(rows16, s_chan, xi)
+        rec = quantizer.dither_reconstruct(code, s_chan, xi)
+        if len(excluded):
+            code[:, excluded] = 0
+            rec[:, excluded] = np.asarray(rows16, dtype=np.float16)[:, excluded].astype(np.float64)
+        return code, s, rec
     if desc.scheme == SCHEME_DITHER_INT8:
         s = quantizer.int8_scale(rows16)
         j = philox.dither_integers(desc.seed, layer, kv_head, slots, tag,
@@ -73,8 +108,15 @@ def quantize_rows(desc, layer, kv_head, rows16, slots, tag):
     return code, None, rec
 
 
-def write_tokens(desc, layer, k16, v16, slot_mapping, cache):
-    """kv_quantize_witness: k16, v16 [n_tok, Hkv, d] fp16; slot < 0 skips."""
+def write_tokens(desc, layer, k16, v16, slot_mapping, cache, bypass_pairs=None):
+    """kv_quantize_witness: k16, v16 [n_tok, Hkv, d] fp16; slot < 0 skips.
+
+    Grouped scheme: ``bypass_pairs`` [Hkv, m] is the layer's fixed pair set
+    (kept in the cache for the read side).
+    """
+    if desc.scheme == SCHEME_DITHER_INT8_G32 and desc.num_bypass_pairs:
+        cache["bypass_pairs"][...] = np.asarray(bypass_pairs, dtype=np.int64).reshape(
+            desc.num_kv_heads, desc.num_bypass_pairs)
     slot_mapping = np.asarray(slot_mapping, dtype=np.int64)
     live = slot_mapping >= 0
     slots = slot_mapping[live]
@@ -82,8 +124,11 @@ def write_tokens(desc, layer, k16, v16, slot_mapping, cache):
     for h in range(desc.num_kv_heads):
         kr = np.asarray(k16)[live, h, :]
         vr = np.asarray(v16)[live, h, :]
-        kc, ks, khat = quantize_rows(desc, layer, h, kr, slots, 0)
+        excl = _excluded(desc, cache, h, 0) if desc.scheme == SCHEME_DITHER_INT8_G32 else ()
+        kc, ks, khat = quantize_rows(desc, layer, h, kr, slots, 0, excl)
         vc, vs, vhat = quantize_rows(desc, layer, h, vr, slots, 1)
+        if len(excl):
+            cache["k_bypass"][page, h, off] = kr[:, excl]
         cache["k_codes"][page, h, off] = kc
         cache["v_codes"][page, h, off] = vc
         if ks is not None:
@@ -105,7 +150,18 @@ def reconstruct(desc, layer, kv_head, slots, cache):
     page, off = slots // desc.page_size, slots % desc.page_size
     kc = cache["k_codes"][page, kv_head, off]
     vc = cache["v_codes"][page, kv_head, off]
-    if desc.scheme == SCHEME_DITHER_INT8:
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        G = desc.group_channels
+        xk = philox.dither_values(philox.dither_integers(
+            desc.seed, layer, kv_head, slots, 0, desc.head_dim, desc.dither_bits), desc.dither_bits)
+        xv = philox.dither_values(philox.dither_integers(
+            desc.seed, layer, kv_head, slots, 1, desc.head_dim, desc.dither_bits), desc.dither_bits)
+        khat = quantizer.dither_reconstruct(kc, np.repeat(cache["k_scale"][page, kv_head, off], G, axis=-1), xk)
+        vhat = quantizer.dither_reconstruct(vc, np.repeat(cache["v_scale"][page, kv_head, off], G, axis=-1), xv)
+        excl = _excluded(desc, cache, kv_head, 0)
+        if len(excl):
+            khat[:, excl] = cache["k_bypass"][page, kv_head, off].astype(np.float64)
+    elif desc.scheme == SCHEME_DITHER_INT8:
         xk = philox.dither_values(philox.dither_integers(
             desc.seed, layer, kv_head, slots, 0, desc.head_dim, desc.dither_bits), desc.dither_bits)
         xv = philox.dither_values(philox.dither_integers(
@@ -141,7 +197,7 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
     if repair_tau is not None:
         res["contrib"] = np.zeros((desc.num_q_heads, n_pages))
         res["repair"] = [None] * desc.num_q_heads
-    if tier_b and desc.scheme != SCHEME_DITHER_INT8:
+    if tier_b and desc.scheme == SCHEME_FP8_E4M3:
         raise ValueError("Tier B needs the dithered INT8 cache (a controlled quantizer)")
     page, off = slots // desc.page_size, slots % desc.page_size
     for h in range(desc.num_kv_heads):
@@ -160,7 +216,11 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
             res["value_term"][hq] = M.value_term(p_tilde, vw[:, 0])
             res["v_max"][hq] = np.max(vw[:, 1]) if ctx_len else 0.0
             res["out_bound"][hq] = M.output_bound(res["meter"][hq], res["v_max"][hq], res["value_term"][hq])
-            if tier_b:
+            if tier_b and desc.scheme == SCHEME_DITHER_INT8_G32:
+                u = M.tier_b_bound_grouped(q, cache["k_scale"][page, h, off], desc.group_channels,
+                                           _excluded(desc, cache, h, 0), ctx_len, delta_loc)
+                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
+            elif tier_b:
                 u = M.tier_b_bound(q, cache["k_scale"][page, h, off].astype(np.float64), ctx_len, delta_loc)
                 res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
             if k_exact is not None:

@@ -20,6 +20,16 @@ the even integer; s that rounds to 0 while amax > 0 is raised to the least
 fp16 subnormal 2^-24 (then clipping can occur, and the witness, being the
 actual residual, stays sound); amax = 0 gives s = 0, code 0, x^ = 0.
 
+Grouped scales with a fixed-channel outlier bypass (§6.2.3 "Storage side",
+Table "granularity"; "Fixed-channel outlier bypass", Tables "amax" and
+"bypassbudget"): one fp16 scale per token and group of G_c contiguous
+channels (G_c = 32 by default), s_g = fp16_rn(fp32(amax_g) / 126.5f) by the
+rule above, where amax_g leaves out the bypassed channels; the bypassed
+channels are the 2m dims of m RoPE pairs fixed per (layer, KV head), stored
+exactly as fp16 (x^ = x there) with code 0.  Readings: the bypass is a key
+side device (RoPE pairs), values use the grouped scales only; a group whose
+channels are all bypassed gets s = 0.
+
 Raw-cast fp8-e4m3 (the black-box fp8 scheme of Fig. f5): code = e4m3(x),
 x^ = decode(code), no scale, no dither.
 
@@ -45,7 +55,12 @@ SCALE_DIVISOR = np.float32(126.5)
 def int8_scale(x16):
     """Per-row fp16 scale from fp16 rows x16 [..., d] (returns float16 [...])."""
     x = np.asarray(x16, dtype=np.float16).astype(np.float64)
-    amax = np.max(np.abs(x), axis=-1)
+    return scale_of_amax(np.max(np.abs(x), axis=-1))
+
+
+def scale_of_amax(amax):
+    """fp16_rn(fp32(amax) / 126.5f), raised to 2^-24 when it rounds to 0."""
+    amax = np.asarray(amax, dtype=np.float64)
     s = (amax.astype(np.float32) / SCALE_DIVISOR).astype(np.float16)
     raise_to_min = (s == 0) & (amax > 0)
     s = np.where(raise_to_min, np.float16(fp.FP16_MIN_SUBNORMAL), s)
@@ -55,12 +70,15 @@ def int8_scale(x16):
 def dither_code(x16, s16, xi):
     """Exact round-half-even of x/s + xi, clamped to [-127, 127].
 
-    x16: fp16 [..., d]; s16: fp16 [...]; xi: float64 [..., d] on the grid
+    x16: fp16 [..., d]; s16: fp16 [...] (one scale per row) or [..., d] (one per
+    channel); xi: float64 [..., d] on the grid
     (odd integer) / 2^(bits+1).  All products below are exact in float64:
     s has 11 significant bits and k + 1/2 - xi has at most 20 for |k| <= 255.
     """
     x = np.asarray(x16, dtype=np.float16).astype(np.float64)
-    s = np.asarray(s16, dtype=np.float16).astype(np.float64)[..., None]
+    s = np.asarray(s16, dtype=np.float16).astype(np.float64)
+    if s.ndim < x.ndim:
+        s = s[..., None]
     xi = np.asarray(xi, dtype=np.float64)
     s_b = np.broadcast_to(s, x.shape)
     zero = s_b == 0
@@ -92,9 +110,48 @@ def dither_code_fraction(x, s, xi):
 
 
 def dither_reconstruct(code, s16, xi):
-    """x^ = s (code - xi), exact in float64."""
-    s = np.asarray(s16, dtype=np.float16).astype(np.float64)[..., None]
+    """x^ = s (code - xi), exact in float64 (s per row, or per channel)."""
+    s = np.asarray(s16, dtype=np.float16).astype(np.float64)
+    if s.ndim < np.ndim(code):
+        s = s[..., None]
     return s * (np.asarray(code, dtype=np.float64) - np.asarray(xi, dtype=np.float64))
+
+
+def bypass_dims(pairs, head_dim, rope_layout):
+    """Dims of the bypassed RoPE pairs, pair by pair: [a_0, b_0, a_1, b_1, ...]."""
+    pairs = np.asarray(pairs, dtype=np.int64).reshape(-1)
+    half = head_dim // 2
+    if rope_layout == ROPE_HALF:
+        a, b = pairs, pairs + half
+    elif rope_layout == ROPE_INTERLEAVED:
+        a, b = 2 * pairs, 2 * pairs + 1
+    else:
+        raise ValueError("unknown rope layout")
+    return np.stack([a, b], axis=1).reshape(-1)
+
+
+def group_scales(x16, group, excluded=(), exclude_from_amax=True):
+    """fp16 scale per row and channel group [..., d / group]; the excluded
+    (bypassed) channels leave the group amax unless exclude_from_amax is False
+    (the "amax unchanged" control of Table "amax")."""
+    x = np.abs(np.asarray(x16, dtype=np.float16).astype(np.float64))
+    if exclude_from_amax and len(excluded):
+        x = x.copy()
+        x[..., np.asarray(excluded, dtype=np.int64)] = 0.0
+    d = x.shape[-1]
+    return scale_of_amax(np.max(x.reshape(x.shape[:-1] + (d // group, group)), axis=-1))
+
+
+def select_bypass_pairs(k16, m, rope_layout):
+    """The m RoPE pairs of largest energy sum_t (x_a^2 + x_b^2) over the rows
+    k16 [n, d] (ties to the lower pair), in increasing pair order."""
+    x = np.asarray(k16, dtype=np.float16).astype(np.float64)
+    d = x.shape[-1]
+    pairs = np.arange(d // 2)
+    dims = bypass_dims(pairs, d, rope_layout).reshape(-1, 2)
+    energy = np.sum(x[:, dims[:, 0]] ** 2 + x[:, dims[:, 1]] ** 2, axis=0)
+    order = sorted(pairs, key=lambda j: (-energy[j], j))
+    return np.sort(np.asarray(order[:m], dtype=np.int64))
 
 
 def fp8_quantize(x16):
