@@ -15,6 +15,17 @@ and for the grouped scheme (§6.2.3) k_scale, v_scale [num_pages, Hkv, P, d/G_c]
 values of the m bypassed RoPE pairs, pair by pair) and bypass_pairs [Hkv, m],
 the layer's fixed pair set per KV head.
 
+Reading (storage order, grouped scheme): the paper fixes neither the byte
+order of a stored row nor which dither word serves which channel.  The
+grouped scheme stores a row's channels in a fixed permuted order and draws
+the dither by storage position (byte i of the Philox call with channel-group
+index n serves storage position 16 n + i, the same rule as the per-token
+scheme's identity order).  Storage position p holds channel
+  K:  16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3)
+  V:  16 ((p >> 1) & 7) + 8 (p & 1) + (p >> 4)
+(the order in which the decode's matrix-multiply fragments consume them, so
+that each fragment step meets one channel group).
+
 The meter loop (§6 box): write path quantizes k -> k^ and stores the
 witness; the read path computes the compressed attention and
 A = sum_t p~_t e^{c_t}; meter = min(1, 1/2 (A^2 - 1)); the gate compares it
@@ -71,6 +82,23 @@ def empty_cache(desc):
     return cache
 
 
+def storage_order(head_dim, tag):
+    """Channel held by each storage position of a grouped-scheme row (K: tag 0, V: tag 1)."""
+    p = np.arange(head_dim)
+    if tag == 0:
+        return 16 * ((p >> 2) & 7) + 4 * (p >> 5) + (p & 3)
+    return 16 * ((p >> 1) & 7) + 8 * (p & 1) + (p >> 4)
+
+
+def _grouped_dither(desc, layer, kv_head, slots, tag):
+    """xi [n, d] by channel: the storage-position dither moved to its channels."""
+    xi_pos = philox.dither_values(philox.dither_integers(
+        desc.seed, layer, kv_head, slots, tag, desc.head_dim, desc.dither_bits), desc.dither_bits)
+    xi = np.empty_like(xi_pos)
+    xi[:, storage_order(desc.head_dim, tag)] = xi_pos
+    return xi
+
+
 def _excluded(desc, cache, kv_head, tag):
     """Bypassed dims of a KV head: keys only (tag 0)."""
     if tag != 0 or desc.num_bypass_pairs == 0:
@@ -81,16 +109,14 @@ def _excluded(desc, cache, kv_head, tag):
 def quantize_rows(desc, layer, kv_head, rows16, slots, tag, excluded=()):
     """Quantize fp16 rows [n, d] written to ``slots``.
 
-    Returns (codes, scale or None, reconstruction float64 [n, d]); ``excluded``
-    are the bypassed dims of the grouped scheme (exact, code 0).
+    Returns (codes by channel, scale or None, reconstruction float64 [n, d]);
+    ``excluded`` are the bypassed dims of the grouped scheme (exact, code 0).
     """
     if desc.scheme == SCHEME_DITHER_INT8_G32:
         G = desc.group_channels
         s = quantizer.group_scales(rows16, G, excluded)
         s_chan = np.repeat(s, G, axis=-1)
-        j = philox.dither_integers(desc.seed, layer, kv_head, slots, tag,
-                                   desc.head_dim, desc.dither_bits)
-        xi = philox.dither_values(j, desc.dither_bits)
+        xi = _grouped_dither(desc, layer, kv_head, slots, tag)
         code = quantizer.dither_code(rows16, s_chan, xi)
         rec = quantizer.dither_reconstruct(code, s_chan, xi)
         if len(excluded):
@@ -129,6 +155,8 @@ def write_tokens(desc, layer, k16, v16, slot_mapping, cache, bypass_pairs=None):
         vc, vs, vhat = quantize_rows(desc, layer, h, vr, slots, 1)
         if len(excl):
             cache["k_bypass"][page, h, off] = kr[:, excl]
+        if desc.scheme == SCHEME_DITHER_INT8_G32:     # storage order
+            kc, vc = kc[:, storage_order(desc.head_dim, 0)], vc[:, storage_order(desc.head_dim, 1)]
         cache["k_codes"][page, h, off] = kc
         cache["v_codes"][page, h, off] = vc
         if ks is not None:
@@ -152,10 +180,11 @@ def reconstruct(desc, layer, kv_head, slots, cache):
     vc = cache["v_codes"][page, kv_head, off]
     if desc.scheme == SCHEME_DITHER_INT8_G32:
         G = desc.group_channels
-        xk = philox.dither_values(philox.dither_integers(
-            desc.seed, layer, kv_head, slots, 0, desc.head_dim, desc.dither_bits), desc.dither_bits)
-        xv = philox.dither_values(philox.dither_integers(
-            desc.seed, layer, kv_head, slots, 1, desc.head_dim, desc.dither_bits), desc.dither_bits)
+        xk = _grouped_dither(desc, layer, kv_head, slots, 0)
+        xv = _grouped_dither(desc, layer, kv_head, slots, 1)
+        kc, vc = np.empty_like(kc), np.empty_like(vc)              # back to channel order
+        kc[:, storage_order(desc.head_dim, 0)] = cache["k_codes"][page, kv_head, off]
+        vc[:, storage_order(desc.head_dim, 1)] = cache["v_codes"][page, kv_head, off]
         khat = quantizer.dither_reconstruct(kc, np.repeat(cache["k_scale"][page, kv_head, off], G, axis=-1), xk)
         vhat = quantizer.dither_reconstruct(vc, np.repeat(cache["v_scale"][page, kv_head, off], G, axis=-1), xv)
         excl = _excluded(desc, cache, kv_head, 0)

@@ -53,16 +53,48 @@ def _cache(scheme, k, v, slots, m=0, G=32, pairs=None, seed=9, layout=0, exclude
     return od, c
 
 
-def test_one_group_without_bypass_is_the_per_token_scheme():
+def _xi_storage_order(seed, layer, kv_head, slots, tag):
+    """The dither by channel of the grouped scheme, built independently: the
+    Philox bytes in storage order, moved to the channel each position holds."""
+    xi_pos = philox.dither_values(philox.dither_integers(seed, layer, kv_head, slots, tag, 128, 8), 8)
+    xi = np.zeros_like(xi_pos)
+    for p in range(128):
+        if tag == 0:
+            c, ks, j = p // 32, (p // 4) % 8, p % 4
+            xi[:, 16 * ks + 4 * c + j] = xi_pos[:, p]
+        else:
+            g, mt, e = p // 16, (p // 2) % 8, p % 2
+            xi[:, 16 * mt + 8 * e + g] = xi_pos[:, p]
+    return xi
+
+
+def test_storage_orders_are_permutations_with_whole_groups_per_fragment_step():
+    for tag in (0, 1):
+        o = OP.storage_order(128, tag)
+        assert sorted(o) == list(range(128))
+    ok, ov = OP.storage_order(128, 0), OP.storage_order(128, 1)
+    for ks in range(8):       # K: positions 32c + 4ks + j (c, j = 0..3) are one QK k-step
+        assert len({ok[32 * c + 4 * ks + j] // 32 for c in range(4) for j in range(4)}) == 1
+    for mt in range(8):       # V: positions 16g + 2mt + e (g = 0..7, e = 0, 1) are one PV m-tile
+        assert {ov[16 * g + 2 * mt + e] for g in range(8) for e in range(2)} == set(range(16 * mt, 16 * mt + 16))
+
+
+def test_one_group_without_bypass_is_the_per_token_quantizer():
     rng = np.random.default_rng(0)
     k, v = _rows(rng, 40 * 2).reshape(40, 2, 128), _rows(rng, 40 * 2).reshape(40, 2, 128)
     slots = rng.permutation(64)[:40]
-    _, a = _cache(OP.SCHEME_DITHER_INT8, k, v, slots)
-    _, b = _cache(OP.SCHEME_DITHER_INT8_G32, k, v, slots, G=128)
-    for name in ("k_codes", "v_codes", "k_witness", "v_witness"):
-        assert np.array_equal(a[name], b[name]), name
-    for name in ("k_scale", "v_scale"):
-        assert np.array_equal(a[name], b[name][..., 0]), name
+    od, b = _cache(OP.SCHEME_DITHER_INT8_G32, k, v, slots, G=128)
+    page, off = slots // 16, slots % 16
+    for h in range(2):
+        for tag, x, name in ((0, k, "k"), (1, v, "v")):
+            s = Q.int8_scale(x[:, h])
+            xi = _xi_storage_order(od.seed, 0, h, slots, tag)
+            code = Q.dither_code(x[:, h], s, xi)
+            assert np.array_equal(b[name + "_scale"][page, h, off][:, 0], s)
+            assert np.array_equal(b[name + "_codes"][page, h, off], code[:, OP.storage_order(128, tag)])
+            if tag == 0:
+                r = Q.dither_reconstruct(code, s, xi) - x[:, h].astype(np.float64)
+                assert np.array_equal(b["k_witness"][page, h, off], Q.witness(r, 8, 0))
 
 
 def test_each_group_is_the_per_token_quantizer_on_its_channels():
@@ -73,7 +105,7 @@ def test_each_group_is_the_per_token_quantizer_on_its_channels():
     slots = np.arange(50) + 100
     desc = OP.Desc(scheme=OP.SCHEME_DITHER_INT8_G32)
     code, s, rec = OP.quantize_rows(desc, 2, 1, x, slots, 0)
-    xi = philox.dither_values(philox.dither_integers(desc.seed, 2, 1, slots, 0, 128, 8), 8)
+    xi = _xi_storage_order(desc.seed, 2, 1, slots, 0)
     for g in range(4):
         sl = slice(32 * g, 32 * g + 32)
         s_ref = Q.int8_scale(x[:, sl])
@@ -226,3 +258,21 @@ def test_meter_sound_on_grouped_caches(m):
             r = OP.decode_sequence(od, 0, q[b] * scale, bt[b], S, cache, k[offs[b]:offs[b] + S],
                                    v.numpy()[offs[b]:offs[b] + S])
             assert np.all(r["tv"] <= r["meter_raw"] * (1 + 1e-12))
+
+
+def test_storage_round_trip():
+    """reconstruct() of a written grouped cache gives back the quantizer's
+    channel-order reconstruction exactly (keys with the bypass, values)."""
+    rng = np.random.default_rng(7)
+    n = 37
+    k = np.stack([_rows(rng, n), _rows(rng, n)], axis=1)
+    v = np.stack([_rows(rng, n), _rows(rng, n)], axis=1)
+    slots = rng.permutation(80)[:n]
+    pairs = np.array([[1, 2, 30, 63], [4, 5, 6, 7]])
+    od, c = _cache(OP.SCHEME_DITHER_INT8_G32, k, v, slots, m=4, pairs=pairs)
+    for h in range(2):
+        dims = Q.bypass_dims(pairs[h], 128, Q.ROPE_HALF)
+        _, _, krec = OP.quantize_rows(od, 0, h, k[:, h], slots, 0, dims)
+        _, _, vrec = OP.quantize_rows(od, 0, h, v[:, h], slots, 1)
+        khat, vhat, _ = OP.reconstruct(od, 0, h, slots, c)
+        assert np.array_equal(khat, krec) and np.array_equal(vhat, vrec)
