@@ -33,6 +33,18 @@
  *   k_witness        [num_pages][Hkv][16][8]    fp16, per-band residual norms
  *   v_witness        [num_pages][Hkv][16][2]    fp16 (||v^ - v||, ||v||) rounded up;
  *                                               optional, for the value side only
+ * The grouped scheme (WC_SCHEME_DITHER_INT8_G32) instead holds
+ *   k_scale, v_scale [num_pages][Hkv][16][4]    fp16, one per 32-channel group
+ *   k_bypass         [num_pages][Hkv][16][2m]   fp16 exact values of the bypassed
+ *                                               pairs, pair by pair (dims a, b)
+ * and stores each row's 128 codes in a permuted channel order, with the
+ * dither drawn by storage position (byte i of the Philox call for channel
+ * group n serves storage position 16 n + i); storage position p holds channel
+ *   K:  16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3)
+ *   V:  16 ((p >> 1) & 7) + 8 (p & 1) + (p >> 4)
+ * (a bypassed key channel holds code 0).  The bypass pairs of a layer,
+ * bypass_pairs [Hkv][m] int32 in [0, 64), are RoPE pair indices: pair j is
+ * dims (j, j + 64) for WC_ROPE_HALF and (2j, 2j + 1) for WC_ROPE_INTERLEAVED.
  */
 #ifndef WITCERT_H
 #define WITCERT_H
@@ -59,7 +71,8 @@ enum {
     WC_DEV_BAD_SLOT = 1u,     /* write: slot >= num_pages * 16; token skipped    */
     WC_DEV_BAD_PAGE = 2u,     /* decode: block-table page outside [0, num_pages)  */
     WC_DEV_BAD_CTX = 4u,      /* decode: context length < 0 or > max_pages * 16   */
-    WC_DEV_TIMEOUT = 8u       /* decode: a bounded wait for staged data gave up   */
+    WC_DEV_TIMEOUT = 8u,      /* decode: a bounded wait for staged data gave up   */
+    WC_DEV_BAD_PAIR = 16u     /* grouped scheme: a bypass pair outside [0, 64) is ignored */
 };
 
 typedef enum {
@@ -69,7 +82,12 @@ typedef enum {
     WC_SCHEME_DITHER_INT8 = 0,
     /* Black-box raw cast to fp8 e4m3fn (round to nearest even, saturating
      * finite overflow to +-448), no scale, no dither (§4.1, Fig. f5). */
-    WC_SCHEME_FP8_E4M3 = 1
+    WC_SCHEME_FP8_E4M3 = 1,
+    /* Subtractive-dither INT8 with one fp16 scale per token and 32-channel
+     * group and a fixed per-(layer, KV head) set of m key RoPE pairs stored
+     * exactly ("outlier bypass", left out of the group amax); §6.2.3.  8-bit
+     * dither only; written and read by the _g32 entry points. */
+    WC_SCHEME_DITHER_INT8_G32 = 2
 } wc_scheme;
 
 typedef enum {
@@ -325,6 +343,59 @@ wc_status wc_repair_select(const float* page_terms, const float* softmax_norm,
                            int32_t max_pages, const uint8_t* keep_q, float tau,
                            float* contrib, int32_t* repair_pages, int32_t* n_repair,
                            float* d_after, uint32_t* dev_status, void* stream);
+
+/*
+ * Write path of the grouped scheme (§6.2.3 "Storage side", "Fixed-channel
+ * outlier bypass"): as wc_kv_quantize_witness, with for each row and group g
+ * of 32 channels s_g = fp16_rn(fp32(amax_g) / 126.5f), amax_g over the
+ * group's channels that are not bypassed (a key row's bypassed channels, the
+ * 2m dims of bypass_pairs[h], are stored exactly in k_bypass with code 0;
+ * value rows have no bypass).  The K witness covers the residual of every
+ * channel (0 on the bypassed ones).
+ *   desc->scheme    WC_SCHEME_DITHER_INT8_G32 with dither_bits 8
+ *   k_scale, v_scale, k_bypass, bypass_pairs  as in the layout above
+ *   num_bypass_pairs  m in [0, 16]; k_bypass and bypass_pairs may be NULL if 0
+ *   dev_status      optional device uint32: WC_DEV_BAD_SLOT, WC_DEV_BAD_PAIR
+ */
+wc_status wc_kv_quantize_witness_g32(const wc_cache_desc* desc, int32_t layer, const void* k,
+                                     const void* v, const int32_t* slot_mapping, int32_t n_tok,
+                                     void* k_codes, void* v_codes, void* k_scale, void* v_scale,
+                                     void* k_witness, void* k_bypass, const int32_t* bypass_pairs,
+                                     int32_t num_bypass_pairs, uint32_t* dev_status, void* stream);
+
+/*
+ * Metered decode attention over a grouped-scheme cache: the same outputs as
+ * wc_metered_decode_attention, from k^_c = s_{g(c)} (code_c - xi_c) (exact
+ * fp16 values on the bypassed key channels) and v^ likewise.  With meter_b
+ * and meter_b_raw not NULL also the Tier-B meter (§4.2) with the grouped proxy
+ *   varsigma_t^2 = (1 / (12 * 128)) sum_{c not bypassed} q_c^2 s_{g(c),t}^2
+ * (delta_loc in (0, 1)); both NULL: not computed.
+ */
+wc_status wc_metered_decode_attention_g32(const wc_cache_desc* desc, int32_t layer,
+                                          const void* q, const int32_t* block_table,
+                                          int32_t max_pages, const int32_t* ctx_lens,
+                                          int32_t batch,
+                                          const void* k_codes, const void* v_codes,
+                                          const void* k_scale, const void* v_scale,
+                                          const void* k_witness, const void* k_bypass,
+                                          const int32_t* bypass_pairs, int32_t num_bypass_pairs,
+                                          double delta_loc,
+                                          float* out, float* meter, float* meter_raw,
+                                          float* meter_b, float* meter_b_raw,
+                                          void* workspace, size_t workspace_bytes, void* stream);
+
+/*
+ * Bypass-pair calibration (§6.2.3 "Fixed-channel outlier bypass": the
+ * massive-activation RoPE pairs are stable across tokens, so a fixed set per
+ * (layer, KV head) chosen from a prefix suffices).  For each KV head h,
+ * pairs[h][0 .. m-1] = the m RoPE pairs of largest energy
+ * sum_t (k[t][h][a]^2 + k[t][h][b]^2) over the n_tok rows (fp32 sums; ties to
+ * the lower pair), in increasing pair order.
+ *   k      [n_tok][Hkv][128] fp16 post-RoPE keys, device, 16-byte aligned
+ *   m      in [0, 16]; pairs [Hkv][m] int32, device
+ */
+wc_status wc_select_bypass_pairs(const void* k, int32_t n_tok, int32_t num_kv_heads,
+                                 int32_t rope_layout, int32_t m, int32_t* pairs, void* stream);
 
 /*
  * Gate (§6 meter-loop box; certified tau < 1 vs risk-ranked tau >= 1, §4.3).

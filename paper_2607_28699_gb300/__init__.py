@@ -27,13 +27,15 @@ LIB_PATH = os.path.join(_HERE, "_lib", "libwitcert.so")
 
 SCHEME_DITHER_INT8 = 0
 SCHEME_FP8_E4M3 = 1
+SCHEME_DITHER_INT8_G32 = 2
 ROPE_HALF = 0
 ROPE_INTERLEAVED = 1
-DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT = 1, 2, 4, 8
+DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT, DEV_BAD_PAIR = 1, 2, 4, 8, 16
 EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
            "wc_metered_decode_attention_tier_b", "wc_metered_decode_attention_noalloc",
            "wc_kv_quantize_witness_v", "wc_metered_decode_attention_v", "wc_gate_joint",
            "wc_metered_decode_attention_repair", "wc_repair_select",
+           "wc_kv_quantize_witness_g32", "wc_metered_decode_attention_g32", "wc_select_bypass_pairs",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -74,6 +76,13 @@ def _load():
     lib.wc_metered_decode_attention_repair.restype = ctypes.c_int
     lib.wc_repair_select.argtypes = [vp, vp, vp, i32, i32, i32, vp, ctypes.c_float, vp, vp, vp, vp, vp, vp]
     lib.wc_repair_select.restype = ctypes.c_int
+    lib.wc_kv_quantize_witness_g32.argtypes = [vp, i32, vp, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, i32, vp, vp]
+    lib.wc_kv_quantize_witness_g32.restype = ctypes.c_int
+    lib.wc_metered_decode_attention_g32.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp, vp, vp, i32,
+                                                    ctypes.c_double, vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.wc_metered_decode_attention_g32.restype = ctypes.c_int
+    lib.wc_select_bypass_pairs.argtypes = [vp, i32, i32, i32, i32, vp, vp]
+    lib.wc_select_bypass_pairs.restype = ctypes.c_int
     lib.wc_read_status.argtypes = [vp, i32, vp, vp]
     lib.wc_read_status.restype = ctypes.c_int
     lib.wc_last_error.argtypes = []
@@ -146,23 +155,35 @@ class LayerCache:
     v_scale: Optional[torch.Tensor]
     k_witness: torch.Tensor
     v_witness: Optional[torch.Tensor] = None   # (||v^ - v||, ||v||) per slot, value side only
+    k_bypass: Optional[torch.Tensor] = None    # grouped scheme: exact bypassed key values [.., 16, 2m]
+    bypass_pairs: Optional[torch.Tensor] = None   # grouped scheme: int32 [Hkv, m] RoPE pair set
 
     @staticmethod
-    def empty(desc: CacheDesc, device="cuda", value_witness=False):
+    def empty(desc: CacheDesc, device="cuda", value_witness=False, num_bypass_pairs=0):
         shp = (desc.num_pages, desc.num_kv_heads, desc.page_size)
-        code_t = torch.int8 if desc.scheme == SCHEME_DITHER_INT8 else torch.uint8
-        dither = desc.scheme == SCHEME_DITHER_INT8
+        code_t = torch.uint8 if desc.scheme == SCHEME_FP8_E4M3 else torch.int8
+        grouped = desc.scheme == SCHEME_DITHER_INT8_G32
+        sshp = shp + (desc.head_dim // 32,) if grouped else shp
+        dither = desc.scheme != SCHEME_FP8_E4M3
+        m = num_bypass_pairs if grouped else 0
         return LayerCache(
             torch.zeros(shp + (desc.head_dim,), dtype=code_t, device=device),
             torch.zeros(shp + (desc.head_dim,), dtype=code_t, device=device),
-            torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
-            torch.zeros(shp, dtype=torch.float16, device=device) if dither else None,
+            torch.zeros(sshp, dtype=torch.float16, device=device) if dither else None,
+            torch.zeros(sshp, dtype=torch.float16, device=device) if dither else None,
             torch.zeros(shp + (desc.num_bands,), dtype=torch.float16, device=device),
-            torch.zeros(shp + (2,), dtype=torch.float16, device=device) if value_witness else None)
+            torch.zeros(shp + (2,), dtype=torch.float16, device=device) if value_witness else None,
+            torch.zeros(shp + (2 * m,), dtype=torch.float16, device=device) if m else None,
+            torch.zeros(desc.num_kv_heads, m, dtype=torch.int32, device=device) if grouped else None)
+
+    @property
+    def num_bypass_pairs(self):
+        return 0 if self.bypass_pairs is None else int(self.bypass_pairs.shape[1])
 
     def nbytes(self):
         return sum(t.numel() * t.element_size() for t in
-                   (self.k_codes, self.v_codes, self.k_scale, self.v_scale, self.k_witness, self.v_witness)
+                   (self.k_codes, self.v_codes, self.k_scale, self.v_scale, self.k_witness, self.v_witness,
+                    self.k_bypass)
                    if t is not None)
 
 
@@ -172,7 +193,13 @@ def kv_quantize_witness(desc: CacheDesc, layer: int, k: torch.Tensor, v: torch.T
     """``wc_kv_quantize_witness`` (``_v`` when the cache holds a value witness):
     k, v fp16 [n_tok, Hkv, 128]; slots int32 [n_tok]."""
     d = desc.c()
-    if cache.v_witness is None:
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        _check(lib.wc_kv_quantize_witness_g32(
+            ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
+            _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+            _ptr(cache.k_witness), _ptr(cache.k_bypass), _ptr(cache.bypass_pairs), cache.num_bypass_pairs,
+            _ptr(dev_status), _stream(stream)))
+    elif cache.v_witness is None:
         _check(lib.wc_kv_quantize_witness(
             ctypes.byref(d), layer, _ptr(k), _ptr(v), _ptr(slot_mapping), int(slot_mapping.numel()),
             _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
@@ -218,12 +245,36 @@ def metered_decode_attention(desc: CacheDesc, layer: int, q: torch.Tensor, block
     if meter_raw is None:
         meter_raw = torch.empty(batch, desc.num_q_heads, dtype=torch.float32, device=dev)
     d = desc.c()
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        _decode_g32(d, layer, q, block_table, ctx_lens, cache, ws, 0.0, out, meter, meter_raw, None, None, stream)
+        return out, meter, meter_raw
     _check(lib.wc_metered_decode_attention(
         ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
         _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
         _ptr(cache.k_witness), _ptr(out), _ptr(meter), _ptr(meter_raw), ws.ptr(), ws.nbytes,
         _stream(stream)))
     return out, meter, meter_raw
+
+
+def _decode_g32(d, layer, q, block_table, ctx_lens, cache, ws, delta_loc, out, meter, meter_raw, meter_b,
+                meter_b_raw, stream):
+    """``wc_metered_decode_attention_g32`` (grouped-scale cache with the outlier bypass)."""
+    batch, max_pages = block_table.shape
+    _check(lib.wc_metered_decode_attention_g32(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(cache.k_bypass), _ptr(cache.bypass_pairs), cache.num_bypass_pairs,
+        float(delta_loc), _ptr(out), _ptr(meter), _ptr(meter_raw), _ptr(meter_b), _ptr(meter_b_raw),
+        ws.ptr(), ws.nbytes, _stream(stream)))
+
+
+def select_bypass_pairs(k: torch.Tensor, m: int, rope_layout: int = ROPE_HALF, pairs=None, stream=None):
+    """``wc_select_bypass_pairs``: k fp16 [n_tok, Hkv, 128] -> int32 [Hkv, m], the m RoPE pairs of
+    largest energy per KV head in increasing order."""
+    n_tok, hkv = k.shape[0], k.shape[1]
+    pairs = torch.empty(hkv, m, dtype=torch.int32, device=k.device) if pairs is None else pairs
+    _check(lib.wc_select_bypass_pairs(_ptr(k), n_tok, hkv, rope_layout, m, _ptr(pairs), _stream(stream)))
+    return pairs
 
 
 def metered_decode_attention_tier_b(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
@@ -240,6 +291,10 @@ def metered_decode_attention_tier_b(desc: CacheDesc, layer: int, q: torch.Tensor
     meter_b = torch.empty(cells, dtype=torch.float32, device=dev) if meter_b is None else meter_b
     meter_b_raw = torch.empty(cells, dtype=torch.float32, device=dev) if meter_b_raw is None else meter_b_raw
     d = desc.c()
+    if desc.scheme == SCHEME_DITHER_INT8_G32:
+        _decode_g32(d, layer, q, block_table, ctx_lens, cache, ws, delta_loc, out, meter, meter_raw, meter_b,
+                    meter_b_raw, stream)
+        return out, meter, meter_raw, meter_b, meter_b_raw
     _check(lib.wc_metered_decode_attention_tier_b(
         ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
         _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),

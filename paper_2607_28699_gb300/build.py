@@ -14,7 +14,8 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 OUT_DIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(OUT_DIR, "libwitcert.so")
-SOURCES = ["api.cu", "write_kernel.cu", "decode_kernel.cu", "gate_kernel.cu", "repair_kernel.cu"]
+SOURCES = ["api.cu", "write_kernel.cu", "decode_kernel.cu", "gate_kernel.cu", "repair_kernel.cu",
+           "decode_g32_kernel.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-O2"]
 

@@ -29,7 +29,9 @@ wc_status cuda_fail(cudaError_t e, const char* what) {
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-wc_status check_desc(const wc_cache_desc* d) {
+// allow_grouped: the grouped scheme is accepted only by its own (_g32) entry
+// points and the workspace query; every other entry point rejects it.
+wc_status check_desc(const wc_cache_desc* d, bool allow_grouped = false) {
     if (!d) return fail(WC_ERR_INVALID_ARG, "desc is NULL");
     if (d->head_dim != wc::kHeadDim) return fail(WC_ERR_UNSUPPORTED, "head_dim must be 128 (got %d)", d->head_dim);
     if (d->page_size != wc::kPage) return fail(WC_ERR_UNSUPPORTED, "page_size must be 16 (got %d)", d->page_size);
@@ -45,8 +47,13 @@ wc_status check_desc(const wc_cache_desc* d) {
     if (d->num_pages < 1) return fail(WC_ERR_INVALID_ARG, "num_pages must be positive (got %d)", d->num_pages);
     if ((long long)d->num_pages * wc::kPage > 0x7FFFFFFFLL)
         return fail(WC_ERR_UNSUPPORTED, "num_pages * 16 must fit in int32");
-    if (d->scheme != WC_SCHEME_DITHER_INT8 && d->scheme != WC_SCHEME_FP8_E4M3)
+    if (d->scheme == WC_SCHEME_DITHER_INT8_G32) {
+        if (!allow_grouped)
+            return fail(WC_ERR_UNSUPPORTED, "the grouped scheme is written and read by the _g32 entry points");
+        if (d->dither_bits != 8) return fail(WC_ERR_UNSUPPORTED, "the grouped scheme uses the 8-bit dither");
+    } else if (d->scheme != WC_SCHEME_DITHER_INT8 && d->scheme != WC_SCHEME_FP8_E4M3) {
         return fail(WC_ERR_UNSUPPORTED, "unknown scheme %d", d->scheme);
+    }
     if (d->rope_layout != WC_ROPE_HALF && d->rope_layout != WC_ROPE_INTERLEAVED)
         return fail(WC_ERR_UNSUPPORTED, "unknown rope_layout %d", d->rope_layout);
     if (d->scheme == WC_SCHEME_DITHER_INT8 && d->dither_bits != 8 && d->dither_bits != 10)
@@ -60,7 +67,7 @@ wc_status check_cache(const wc_cache_desc* d, const void* kc, const void* vc, co
     if (!kc || !vc || !kw) return fail(WC_ERR_INVALID_ARG, "cache pointers must not be NULL");
     if (!aligned16(kc) || !aligned16(vc) || !aligned16(kw))
         return fail(WC_ERR_INVALID_ARG, "cache arrays must be 16-byte aligned");
-    if (d->scheme == WC_SCHEME_DITHER_INT8) {
+    if (d->scheme == WC_SCHEME_DITHER_INT8 || d->scheme == WC_SCHEME_DITHER_INT8_G32) {
         if (!ks || !vs) return fail(WC_ERR_INVALID_ARG, "k_scale/v_scale are required by the dither scheme");
         if (!aligned16(ks) || !aligned16(vs)) return fail(WC_ERR_INVALID_ARG, "scale arrays must be 16-byte aligned");
     } else if (ks || vs) {
@@ -84,11 +91,27 @@ int32_t wc_version(void) { return (1 << 16) | 0; }
 
 const char* wc_last_error(void) { return g_last_error.c_str(); }
 
+// Bypass arguments of the grouped scheme: m in [0, 16]; the pair list and the
+// exact-value array are required when m > 0.
+static wc_status check_bypass(const void* k_bypass, const int32_t* bypass_pairs, int32_t m) {
+    if (m < 0 || m > 16) return fail(WC_ERR_INVALID_ARG, "num_bypass_pairs must be in [0, 16] (got %d)", m);
+    if (m > 0 && (!k_bypass || !bypass_pairs))
+        return fail(WC_ERR_INVALID_ARG, "k_bypass and bypass_pairs must not be NULL when num_bypass_pairs > 0");
+    if (m > 0 && !aligned16(k_bypass)) return fail(WC_ERR_INVALID_ARG, "k_bypass must be 16-byte aligned");
+    return WC_OK;
+}
+
 static wc_status write_tokens(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
                               const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
                               void* k_scale, void* v_scale, void* k_witness, void* v_witness,
-                              uint32_t* dev_status, void* stream) {
-    if (wc_status st = check_desc(desc)) return st;
+                              uint32_t* dev_status, void* stream, bool grouped = false, void* k_bypass = nullptr,
+                              const int32_t* bypass_pairs = nullptr, int32_t num_bypass = 0) {
+    if (wc_status st = check_desc(desc, grouped)) return st;
+    if (grouped) {
+        if (desc->scheme != WC_SCHEME_DITHER_INT8_G32)
+            return fail(WC_ERR_INVALID_ARG, "the _g32 entry points need desc->scheme = WC_SCHEME_DITHER_INT8_G32");
+        if (wc_status st = check_bypass(k_bypass, bypass_pairs, num_bypass)) return st;
+    }
     if (layer < 0 || layer > 65535) return fail(WC_ERR_INVALID_ARG, "layer must be in [0, 65535] (got %d)", layer);
     if (n_tok < 0) return fail(WC_ERR_INVALID_ARG, "n_tok must be >= 0 (got %d)", n_tok);
     if ((long long)n_tok * desc->num_kv_heads > 0x7FFFFFFFLL - 8)
@@ -108,6 +131,9 @@ static wc_status write_tokens(const wc_cache_desc* desc, int32_t layer, const vo
     p.v_scale = static_cast<__half*>(v_scale);
     p.k_witness = static_cast<__half*>(k_witness);
     p.v_witness = static_cast<__half*>(v_witness);
+    p.k_bypass = static_cast<__half*>(k_bypass);
+    p.bypass_pairs = bypass_pairs;
+    p.num_bypass = num_bypass;
     p.dev_status = dev_status;
     p.n_tok = n_tok;
     p.num_kv_heads = desc->num_kv_heads;
@@ -136,8 +162,32 @@ wc_status wc_kv_quantize_witness_v(const wc_cache_desc* desc, int32_t layer, con
                         v_witness, dev_status, stream);
 }
 
+wc_status wc_kv_quantize_witness_g32(const wc_cache_desc* desc, int32_t layer, const void* k, const void* v,
+                                     const int32_t* slot_mapping, int32_t n_tok, void* k_codes, void* v_codes,
+                                     void* k_scale, void* v_scale, void* k_witness, void* k_bypass,
+                                     const int32_t* bypass_pairs, int32_t num_bypass_pairs, uint32_t* dev_status,
+                                     void* stream) {
+    return write_tokens(desc, layer, k, v, slot_mapping, n_tok, k_codes, v_codes, k_scale, v_scale, k_witness,
+                        nullptr, dev_status, stream, true, k_bypass, bypass_pairs, num_bypass_pairs);
+}
+
+wc_status wc_select_bypass_pairs(const void* k, int32_t n_tok, int32_t num_kv_heads, int32_t rope_layout, int32_t m,
+                                 int32_t* pairs, void* stream) {
+    if (n_tok < 0) return fail(WC_ERR_INVALID_ARG, "n_tok must be >= 0 (got %d)", n_tok);
+    if (num_kv_heads < 1 || num_kv_heads > 65535)
+        return fail(WC_ERR_INVALID_ARG, "num_kv_heads must be in [1, 65535] (got %d)", num_kv_heads);
+    if (rope_layout != WC_ROPE_HALF && rope_layout != WC_ROPE_INTERLEAVED)
+        return fail(WC_ERR_UNSUPPORTED, "unknown rope_layout %d", rope_layout);
+    if (m < 0 || m > 16) return fail(WC_ERR_INVALID_ARG, "m must be in [0, 16] (got %d)", m);
+    if (m == 0) return WC_OK;
+    if (!pairs || (n_tok > 0 && !k)) return fail(WC_ERR_INVALID_ARG, "k and pairs must not be NULL");
+    cudaError_t e = wc::launch_select_pairs(static_cast<const __half*>(k), n_tok, num_kv_heads, rope_layout, m, pairs,
+                                            static_cast<cudaStream_t>(stream));
+    return e == cudaSuccess ? WC_OK : cuda_fail(e, "pair selection kernel launch");
+}
+
 size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_pages) {
-    if (check_desc(desc) != WC_OK) return 0;
+    if (check_desc(desc, true) != WC_OK) return 0;
     if (batch < 1 || max_pages < 1) {
         fail(WC_ERR_INVALID_ARG, "batch and max_pages must be positive");
         return 0;
@@ -160,8 +210,14 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
                                        float* meter_b_raw, double delta_loc, const void* v_witness,
                                        float* value_term, float* v_max, float* out_bound, float* page_terms,
                                        float* softmax_norm, void* workspace, size_t workspace_bytes,
-                                       void* stream) {
-    if (wc_status st = check_desc(desc)) return st;
+                                       void* stream, bool grouped = false, const void* k_bypass = nullptr,
+                                       const int32_t* bypass_pairs = nullptr, int32_t num_bypass = 0) {
+    if (wc_status st = check_desc(desc, grouped)) return st;
+    if (grouped) {
+        if (desc->scheme != WC_SCHEME_DITHER_INT8_G32)
+            return fail(WC_ERR_INVALID_ARG, "the _g32 entry points need desc->scheme = WC_SCHEME_DITHER_INT8_G32");
+        if (wc_status st = check_bypass(k_bypass, bypass_pairs, num_bypass)) return st;
+    }
     if (page_terms || softmax_norm) {
         if (!page_terms || !softmax_norm)
             return fail(WC_ERR_INVALID_ARG, "page_terms and softmax_norm must not be NULL");
@@ -177,7 +233,7 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
         if (meter_b) return fail(WC_ERR_UNSUPPORTED, "Tier B and the value side are separate calls");
     }
     if (meter_b || meter_b_raw) {
-        if (desc->scheme != WC_SCHEME_DITHER_INT8)
+        if (desc->scheme == WC_SCHEME_FP8_E4M3)
             return fail(WC_ERR_UNSUPPORTED, "Tier B needs the dithered INT8 cache (a controlled quantizer)");
         if (!meter_b || !meter_b_raw) return fail(WC_ERR_INVALID_ARG, "meter_b and meter_b_raw must not be NULL");
         if (!(delta_loc > 0.0 && delta_loc < 1.0))
@@ -221,6 +277,9 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.out_bound = out_bound;
     p.page_terms = reinterpret_cast<float2*>(page_terms);
     p.softmax_norm = reinterpret_cast<float2*>(softmax_norm);
+    p.k_bypass = static_cast<const __half*>(k_bypass);
+    p.bypass_pairs = bypass_pairs;
+    p.num_bypass = num_bypass;
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
@@ -290,6 +349,20 @@ wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t 
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
                                  nullptr, nullptr, page_terms, softmax_norm, workspace, workspace_bytes, stream);
+}
+
+wc_status wc_metered_decode_attention_g32(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                          const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                          int32_t batch, const void* k_codes, const void* v_codes,
+                                          const void* k_scale, const void* v_scale, const void* k_witness,
+                                          const void* k_bypass, const int32_t* bypass_pairs,
+                                          int32_t num_bypass_pairs, double delta_loc, float* out, float* meter,
+                                          float* meter_raw, float* meter_b, float* meter_b_raw, void* workspace,
+                                          size_t workspace_bytes, void* stream) {
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, meter_b, meter_b_raw, delta_loc, nullptr,
+                                 nullptr, nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream, true,
+                                 k_bypass, bypass_pairs, num_bypass_pairs);
 }
 
 wc_status wc_repair_select(const float* page_terms, const float* softmax_norm, const int32_t* ctx_lens,

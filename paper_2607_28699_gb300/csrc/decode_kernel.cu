@@ -26,7 +26,7 @@
 #include <climits>
 #include <mutex>
 
-#include "wc_kernels.cuh"
+#include "decode_common.cuh"
 
 namespace wc {
 
@@ -41,50 +41,6 @@ constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
 constexpr int kOffVw = 4416;             // value witness [16][2] fp16 (value side)
 constexpr int kStageStride = 4480;       // stage buffer size
 constexpr int kSmemBytes = kWarps * kStages * kStageStride + kWarps * kStages * 8;
-
-// Extra outputs compiled into a decode kernel (template bit mask).
-constexpr int kXTierB = 1;   // Tier-B meter (§4.2)
-constexpr int kXValue = 2;   // value-side witness terms and output bound (§3, §4.2)
-constexpr int kXRepair = 4;  // per-page meter terms for block-level repair selection (§6.4)
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kRsd = 0.08838834764831845f;                      // 1/sqrt(128)
-constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;
-
-constexpr uint32_t kSel01 = 0x4140u, kSel23 = 0x4342u;   // [x0,K,x1,K], [x2,K,x3,K]
-
-__device__ __forceinline__ uint32_t sel_interleave(int p) {  // [a_p, b_p, a_p+1, b_p+1]
-    return p == 0 ? 0x5140u : 0x7362u;
-}
-
-template <int kBits>
-struct DitherConst;
-template <>
-struct DitherConst<8> {  // xi = (j + 1/2)/256 - 1/2 = h' - kappa, h' = 4 + j/256
-    static constexpr float kappa = 4.498046875f;
-};
-template <>
-struct DitherConst<10> {  // xi = (j + 1/2)/1024 - 1/2 = h' - kappa, h' = 1 + j/1024
-    static constexpr float kappa = 1.49951171875f;
-};
-
-// h' pair (fp16) for two 8-bit dithers: bytes of x at the selector.
-__device__ __forceinline__ uint32_t h8(uint32_t x, uint32_t sel) { return prmt(x, 0x44444444u, sel); }
-// h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
-__device__ __forceinline__ uint32_t h10(uint32_t x) { return (x & 0x03FF03FFu) | 0x3C003C00u; }
-
-// 2^n for -126 <= n <= 127.
-__device__ __forceinline__ float pow2(int n) { return __int_as_float((127 + n) << 23); }
-
-__device__ __forceinline__ uint32_t word_of(const uint4& v, int i) {
-    return i == 0 ? v.x : i == 1 ? v.y : i == 2 ? v.z : v.w;
-}
-
-// Transpose of an 8x8 b16 matrix held in the mma fragment layout.
-__device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
-    uint32_t y;
-    asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
-    return y;
-}
 
 // §6.4 "Block-level paging": the share of D of logical page lp for this
 // thread's softmax heads 2c, 2c+1, kept against the running maximum it was
@@ -1351,6 +1307,12 @@ static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
     return launch_pdl(merge_kernel<kX>, grid, dim3(32 * kMergeWarps), smem, stream, p);
 }
 
+cudaError_t launch_merge_x(const DecodeParams& p, int x, cudaStream_t stream) {
+    return x == kXTierB ? launch_merge<kXTierB>(p, stream)
+         : x == kXValue ? launch_merge<kXValue>(p, stream)
+         : x == kXRepair ? launch_merge<kXRepair>(p, stream) : launch_merge<0>(p, stream);
+}
+
 template <int kScheme, int kBits, int kX>
 static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;   // per process; the attributes are per function
@@ -1429,6 +1391,7 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.batch == 0) return cudaSuccess;
+    if (scheme == WC_SCHEME_DITHER_INT8_G32) return launch_decode_g32(p, stream);
     // Tier B (dithered INT8 only), the value side and the repair terms are
     // requested by separate entry points, never together (checked by the caller)
     const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0) | (p.page_terms ? kXRepair : 0);

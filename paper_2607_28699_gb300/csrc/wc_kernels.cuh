@@ -17,6 +17,9 @@ struct WriteParams {
     __half* v_scale;
     __half* k_witness;
     __half* v_witness;    // [slot][2] (rho^v, ||v||) rounded up, nullptr: not stored
+    __half* k_bypass = nullptr;              // grouped scheme: [slot][2m] exact bypassed values
+    const int32_t* bypass_pairs = nullptr;   // grouped scheme: [Hkv][m] RoPE pair indices
+    int32_t num_bypass = 0;                  // m
     uint32_t* dev_status;
     int32_t n_tok, num_kv_heads, num_pages, layer, rope_layout;
     PhiloxKeys keys;
@@ -47,6 +50,10 @@ struct DecodeParams {
     // per (sequence, query head): (M, L), the final log2-domain maximum and sum.
     float2* page_terms = nullptr;     // [batch][Hq][max_pages]
     float2* softmax_norm = nullptr;   // [batch][Hq]
+    // grouped scheme: exact bypassed key values [slot][2m] and the pair set [Hkv][m]
+    const __half* k_bypass = nullptr;
+    const int32_t* bypass_pairs = nullptr;
+    int32_t num_bypass = 0;
     uint32_t* status;     // workspace word
     uint32_t* counters;   // [batch * Hkv], zero between calls
     float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
@@ -108,7 +115,10 @@ constexpr int kRepairMaxPages = 16384;
 
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
+cudaError_t launch_decode_g32(const DecodeParams& p, cudaStream_t stream);
 cudaError_t launch_repair_select(const RepairParams& p, cudaStream_t stream);
+cudaError_t launch_select_pairs(const __half* k, int n_tok, int num_kv_heads, int rope_layout, int m, int32_t* pairs,
+                                cudaStream_t stream);
 cudaError_t launch_gate(const float* meter_raw, const float* value_term, const float* v_max, int n_cells, int group,
                         float tau, float tau_v, uint8_t* keep_q, uint8_t* keep_kv, int32_t* n_kept,
                         cudaStream_t stream);

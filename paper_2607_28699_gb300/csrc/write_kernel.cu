@@ -5,8 +5,20 @@
 // A CTA of 4 warps handles eight (token, KV head) units: warps 0 and 2 the K
 // rows, warps 1 and 3 the V rows, 8 lanes per row.  Each lane owns 16
 // consecutive channels, so it loads 32 B of fp16, stores 16 B of codes, and
-// (for the dither scheme) consumes exactly one Philox4x32-10 call per 16
+// (for the dither schemes) consumes exactly one Philox4x32-10 call per 16
 // channels.
+//
+// Grouped scheme (§6.2.3 "Storage side" and "Fixed-channel outlier bypass"):
+// one fp16 scale per 32-channel group (a lane pair), the group amax leaving
+// out the bypassed channels of the KV head's fixed RoPE pairs, which are
+// stored exactly (fp16, code 0).  A row is stored in a permuted channel order
+// with the dither drawn by storage position; storage position p holds channel
+//   K:  16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3)
+//   V:  16 ((p >> 1) & 7) + 8 (p & 1) + (p >> 4)
+// (the decode's fragment order: each QK k-step and each PV m-tile then meets
+// one group).  The lane's Philox call covers storage positions 16 sub .. +15;
+// dither bytes and codes move between storage and channel order through a
+// 128-byte shared row per unit, so quantization runs in channel order.
 #include <type_traits>
 
 #include "wc_kernels.cuh"
@@ -64,10 +76,21 @@ constexpr float kBias = 12582912.0f;
 // Dither word byte (i % 4) placed as the float 1 + j/2^15 (bits 0x3F80jj00).
 __device__ __forceinline__ uint32_t xi_sel(int i) { return 0x7604u | ((uint32_t)(i & 3) << 4); }
 
+// x[i] for a lane-uniform runtime index i in [0, 16), without local memory.
+__device__ __forceinline__ float pick16(const float (&x)[16], int i) {
+    float v = x[0];
+#pragma unroll
+    for (int k = 1; k < 16; ++k) v = (i == k) ? x[k] : v;
+    return v;
+}
+
 // One row (K or V) of one (token, KV head): 8 lanes, 16 channels each.
+// xrow: the unit's 128-byte shared row (grouped scheme only).
 template <int kScheme, int kBits>
 __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2], int slot, bool live_unit, int h,
-                                          int row, int sub) {
+                                          int row, int sub, uint8_t* xrow) {
+    constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
+    constexpr bool kDither = kScheme != WC_SCHEME_FP8_E4M3;
     const bool bad = slot >= p.num_pages * kPage;
     const bool active = live_unit && slot >= 0 && !bad;
     if (live_unit && bad && sub == 0 && row == 0 && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_SLOT);
@@ -89,12 +112,30 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
     float lo = 0.0f, hi = 0.0f;
     const bool resid = row == 0 || p.v_witness != nullptr;   // warp-uniform
     float s = 0.0f;
-    if constexpr (kScheme == WC_SCHEME_DITHER_INT8) {
+    uint32_t bmask = 0;   // grouped K rows: bypassed channels among 16 sub .. 16 sub + 15
+    if constexpr (kGrouped) {
+        if (row == 0) {
+            const int32_t* pr = p.bypass_pairs + (size_t)h * p.num_bypass;
+            for (int t = 0; t < p.num_bypass; ++t) {
+                const int j = __ldg(pr + t);
+                if (j < 0 || j >= kHeadDim / 2) {
+                    if (live_unit && sub == 0 && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_PAIR);
+                    continue;
+                }
+                const int a = p.rope_layout == WC_ROPE_HALF ? j : 2 * j;
+                const int b = p.rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+                if ((a >> 4) == sub) bmask |= 1u << (a & 15);
+                if ((b >> 4) == sub) bmask |= 1u << (b & 15);
+            }
+        }
+    }
+    if constexpr (kDither) {
         float amax = 0.0f;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) amax = fmaxf(amax, fabsf(x[i]));
+        for (int i = 0; i < 16; ++i) amax = fmaxf(amax, ((bmask >> i) & 1u) ? 0.0f : fabsf(x[i]));
+        // the row (8 lanes) or the 32-channel group (a lane pair)
 #pragma unroll
-        for (int o = 1; o < 8; o <<= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
+        for (int o = 1; o < (kGrouped ? 2 : 8); o <<= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
         __half sh = __float2half_rn(__fdiv_rn(amax, 126.5f));
         if (__half_as_ushort(sh) == 0 && amax > 0.0f) sh = __ushort_as_half((unsigned short)1);
         s = __half2float(sh);
@@ -107,6 +148,26 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         if constexpr (kBits == 8) {
             const uint4 w = philox(slot_u, c1, (uint32_t)sub, (uint32_t)row, p.keys);
             dw[0] = w.x; dw[1] = w.y; dw[2] = w.z; dw[3] = w.w;
+            if constexpr (kGrouped) {
+                // storage-position bytes -> this lane's channels 16 sub + i
+                __syncwarp();
+                *reinterpret_cast<uint4*>(xrow + 16 * sub) = w;
+                __syncwarp();
+                if (row == 0) {   // channel 16 sub + 4q + j is at position 32q + 4 sub + j
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) dw[q] = *reinterpret_cast<const uint32_t*>(xrow + 32 * q + 4 * sub);
+                } else {          // channel 16 sub + 8e + g is at position 16g + 2 sub + e
+                    uint32_t u[8];
+#pragma unroll
+                    for (int g = 0; g < 8; ++g) u[g] = *reinterpret_cast<const uint16_t*>(xrow + 16 * g + 2 * sub);
+                    const uint32_t t01 = u[0] | (u[1] << 16), t23 = u[2] | (u[3] << 16);
+                    const uint32_t t45 = u[4] | (u[5] << 16), t67 = u[6] | (u[7] << 16);
+                    dw[0] = prmt(t01, t23, 0x6420u);   // e = 0, g = 0..3
+                    dw[1] = prmt(t45, t67, 0x6420u);   // e = 0, g = 4..7
+                    dw[2] = prmt(t01, t23, 0x7531u);   // e = 1, g = 0..3
+                    dw[3] = prmt(t45, t67, 0x7531u);   // e = 1, g = 4..7
+                }
+            }
         } else {
 #pragma unroll
             for (int gi = 0; gi < 2; ++gi) {
@@ -143,14 +204,15 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
             float dev = 0.0f;
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
+                const bool byp = kGrouped && ((bmask >> i) & 1u);   // exact channel: code 0, no residual
                 const float xi = xi_of(i);
-                const float est = fmaf(x[i], inv_s, xi);   // s = 0: x = 0, est = xi, k = 0
+                const float est = byp ? 0.0f : fmaf(x[i], inv_s, xi);   // s = 0: x = 0, est = xi, k = 0
                 const float t = est + kBias;
                 const float k = t - kBias;
                 dev = fmaxf(dev, fabsf(est - k));
                 tb[i] = __float_as_uint(t);
                 if constexpr (decltype(with_residual)::value) {
-                    const float r = fmaf(s, k - xi, -x[i]);   // x^ - x, one rounding
+                    const float r = byp ? 0.0f : fmaf(s, k - xi, -x[i]);   // x^ - x, one rounding
                     if (i < 8) lo = fmaf(r, r, lo);
                     else hi = fmaf(r, r, hi);
                 }
@@ -166,12 +228,13 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
             lo = hi = 0.0f;
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
+                const bool byp = kGrouped && ((bmask >> i) & 1u);
                 const float xi = xi_of(i);
                 const float est = fminf(127.0f, fmaxf(-127.0f, fmaf(x[i], inv_s, xi)));
-                const float k = exact_round(x[i], s, xi, (est + kBias) - kBias);
+                const float k = byp ? 0.0f : exact_round(x[i], s, xi, (est + kBias) - kBias);
                 tb[i] = __float_as_uint(k + kBias);
                 if (resid) {
-                    const float r = fmaf(s, k - xi, -x[i]);
+                    const float r = byp ? 0.0f : fmaf(s, k - xi, -x[i]);
                     if (i < 8) lo = fmaf(r, r, lo);
                     else hi = fmaf(r, r, hi);
                 }
@@ -181,6 +244,21 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         for (int i = 0; i < 4; ++i)
             codes[i] = prmt(prmt(tb[4 * i], tb[4 * i + 1], 0x0040u), prmt(tb[4 * i + 2], tb[4 * i + 3], 0x0040u),
                             0x5410u);
+        if constexpr (kGrouped) {   // channel order -> storage order
+            __syncwarp();
+            if (row == 0) {
+#pragma unroll
+                for (int q = 0; q < 4; ++q) *reinterpret_cast<uint32_t*>(xrow + 32 * q + 4 * sub) = codes[q];
+            } else {
+#pragma unroll
+                for (int g = 0; g < 8; ++g)   // bytes of channels 16 sub + g and 16 sub + 8 + g
+                    *reinterpret_cast<uint16_t*>(xrow + 16 * g + 2 * sub) =
+                        (uint16_t)((tb[g] & 0xFFu) | ((tb[8 + g] & 0xFFu) << 8));
+            }
+            __syncwarp();
+            const uint4 st = *reinterpret_cast<const uint4*>(xrow + 16 * sub);
+            codes[0] = st.x; codes[1] = st.y; codes[2] = st.z; codes[3] = st.w;
+        }
     } else {
         const uint32_t* hw = reinterpret_cast<const uint32_t*>(raw);
 #pragma unroll
@@ -208,6 +286,24 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         *reinterpret_cast<uint4*>(dst) = make_uint4(codes[0], codes[1], codes[2], codes[3]);
         if constexpr (kScheme == WC_SCHEME_DITHER_INT8) {
             if (sub == 0) (row == 0 ? p.k_scale : p.v_scale)[rowidx] = __float2half_rn(s);
+        }
+        if constexpr (kGrouped) {
+            if ((sub & 1) == 0) (row == 0 ? p.k_scale : p.v_scale)[rowidx * 4 + (sub >> 1)] = __float2half_rn(s);
+            if (row == 0 && p.num_bypass > 0) {   // the exact values of the bypassed pairs, pair by pair
+                const int32_t* pr = p.bypass_pairs + (size_t)h * p.num_bypass;
+                __half* bdst = p.k_bypass + rowidx * (2 * p.num_bypass);
+                for (int t = 0; t < p.num_bypass; ++t) {
+                    const int j = __ldg(pr + t);
+                    if (j < 0 || j >= kHeadDim / 2) {   // an ignored pair stores zeros
+                        if (sub == 0) bdst[2 * t] = bdst[2 * t + 1] = __float2half_rn(0.0f);
+                        continue;
+                    }
+                    const int a = p.rope_layout == WC_ROPE_HALF ? j : 2 * j;
+                    const int b = p.rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+                    if ((a >> 4) == sub) bdst[2 * t] = __float2half_rn(pick16(x, a & 15));
+                    if ((b >> 4) == sub) bdst[2 * t + 1] = __float2half_rn(pick16(x, b & 15));
+                }
+            }
         }
     }
     if (row != 0) {   // warp-uniform
@@ -261,6 +357,8 @@ constexpr int kPerHeadMinTokens = 16;                     // per-head grid from 
 //            (decode steps, where every SM the next decode needs counts).
 template <int kScheme, int kBits, bool kPerHead>
 __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ WriteParams p) {
+    constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
+    __shared__ __align__(16) uint8_t xrows[kGrouped ? 4 * 4 * kHeadDim : 16];   // [warp][unit][128]
     grid_dep_launch();    // a dependent decode may be scheduled now: it waits for this whole grid
     grid_dep_wait();      // inputs may come from the preceding kernel
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -301,21 +399,66 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
 #pragma unroll
     for (int t = 0; t < kWriteTasks; ++t)
         if (__any_sync(0xffffffffu, live[t]))   // warp-uniform: a task past the end is skipped whole
-            write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub);
+            write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub,
+                                      kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kHeadDim : xrows);
+}
+
+// Bypass-pair calibration: one CTA per KV head; thread t sums pair t % 64
+// over every fourth token, the four partial sums are added in a fixed order,
+// and a pair is selected iff fewer than m pairs rank above it (larger energy,
+// or equal energy and a lower index).
+__global__ void __launch_bounds__(256) select_pairs_kernel(const __half* __restrict__ k, int n_tok, int num_kv_heads,
+                                                           int rope_layout, int m, int32_t* __restrict__ pairs) {
+    __shared__ float part[4][kHeadDim / 2];
+    __shared__ float energy[kHeadDim / 2];
+    __shared__ int chosen[kHeadDim / 2];
+    const int h = blockIdx.x, j = threadIdx.x & 63, stripe = threadIdx.x >> 6;
+    const int a = rope_layout == WC_ROPE_HALF ? j : 2 * j;
+    const int b = rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+    float acc = 0.0f;
+    for (int t = stripe; t < n_tok; t += 4) {
+        const __half* row = k + ((size_t)t * num_kv_heads + h) * kHeadDim;
+        const float xa = __half2float(row[a]), xb = __half2float(row[b]);
+        acc = fmaf(xa, xa, fmaf(xb, xb, acc));
+    }
+    part[stripe][j] = acc;
+    __syncthreads();
+    if (threadIdx.x < 64) energy[j] = ((part[0][j] + part[1][j]) + part[2][j]) + part[3][j];
+    __syncthreads();
+    if (threadIdx.x < 64) {
+        const float e = energy[j];
+        int rank = 0;
+        for (int i = 0; i < 64; ++i) rank += (energy[i] > e || (energy[i] == e && i < j)) ? 1 : 0;
+        chosen[j] = rank < m;
+    }
+    __syncthreads();
+    if (threadIdx.x < 64 && chosen[j]) {
+        int pos = 0;
+        for (int i = 0; i < j; ++i) pos += chosen[i];
+        pairs[(size_t)h * m + pos] = j;
+    }
 }
 
 }  // namespace
+
+cudaError_t launch_select_pairs(const __half* k, int n_tok, int num_kv_heads, int rope_layout, int m, int32_t* pairs,
+                                cudaStream_t stream) {
+    select_pairs_kernel<<<num_kv_heads, 256, 0, stream>>>(k, n_tok, num_kv_heads, rope_layout, m, pairs);
+    return cudaGetLastError();
+}
 
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream) {
     if (p.n_tok == 0) return cudaSuccess;
     static bool configured = false;   // same carveout as the decode kernels: no L1/shared reconfiguration
     if (!configured) {
-        const void* fns[6] = {(const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8, false>,
+        const void* fns[8] = {(const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8, false>,
                               (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8, false>,
                               (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10, false>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8_G32, 8, false>,
                               (const void*)write_kernel<WC_SCHEME_FP8_E4M3, 8, true>,
                               (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 8, true>,
-                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10, true>};
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8, 10, true>,
+                              (const void*)write_kernel<WC_SCHEME_DITHER_INT8_G32, 8, true>};
         for (const void* f : fns) {
             cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributePreferredSharedMemoryCarveout,
                                                  (int)cudaSharedmemCarveoutMaxShared);
@@ -329,6 +472,9 @@ cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_
     auto go = [&](auto kernel) { return launch_pdl(kernel, grid, dim3(128), 0, stream, p); };
     if (scheme == WC_SCHEME_FP8_E4M3)
         return per_head ? go(write_kernel<WC_SCHEME_FP8_E4M3, 8, true>) : go(write_kernel<WC_SCHEME_FP8_E4M3, 8, false>);
+    if (scheme == WC_SCHEME_DITHER_INT8_G32)
+        return per_head ? go(write_kernel<WC_SCHEME_DITHER_INT8_G32, 8, true>)
+                        : go(write_kernel<WC_SCHEME_DITHER_INT8_G32, 8, false>);
     if (bits == 8)
         return per_head ? go(write_kernel<WC_SCHEME_DITHER_INT8, 8, true>)
                         : go(write_kernel<WC_SCHEME_DITHER_INT8, 8, false>);

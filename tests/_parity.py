@@ -37,10 +37,10 @@ def assert_close(gpu, ref, what, rtol=RTOL, atol=ATOL):
                              f"gpu={g[tuple(idx.T)]} ref={r[tuple(idx.T)]}")
 
 
-def descs(n_q, n_kv, num_pages, scheme=0, bits=8, layout=0, seed=0):
+def descs(n_q, n_kv, num_pages, scheme=0, bits=8, layout=0, seed=0, num_bypass_pairs=0):
     import paper_2607_28699_gb300 as wc
     o = OP.Desc(num_q_heads=n_q, num_kv_heads=n_kv, num_pages=num_pages, scheme=scheme,
-                dither_bits=bits, rope_layout=layout, seed=seed)
+                dither_bits=bits, rope_layout=layout, seed=seed, num_bypass_pairs=num_bypass_pairs)
     g = wc.CacheDesc(num_q_heads=n_q, num_kv_heads=n_kv, num_pages=num_pages, scheme=scheme,
                      dither_bits=bits, rope_layout=layout, seed=seed)
     return o, g
@@ -54,12 +54,20 @@ def gpu_cache_to_numpy(cache):
         out["v_scale"] = cache.v_scale.cpu().numpy()
     if cache.v_witness is not None:
         out["v_witness"] = cache.v_witness.cpu().numpy()
+    if cache.k_bypass is not None:
+        out["k_bypass"] = cache.k_bypass.cpu().numpy()
+    if cache.bypass_pairs is not None:
+        out["bypass_pairs"] = cache.bypass_pairs.cpu().numpy().astype(np.int64)
     return out
 
 
 def numpy_cache_to_gpu(cache, desc_g, value_witness=False):
     import paper_2607_28699_gb300 as wc
-    c = wc.LayerCache.empty(desc_g, value_witness=value_witness)
+    m = cache["bypass_pairs"].shape[1] if "bypass_pairs" in cache else 0
+    c = wc.LayerCache.empty(desc_g, value_witness=value_witness, num_bypass_pairs=m)
+    if m:
+        c.k_bypass.copy_(torch.from_numpy(cache["k_bypass"]))
+        c.bypass_pairs.copy_(torch.from_numpy(cache["bypass_pairs"].astype(np.int32)))
     if value_witness:
         c.v_witness.copy_(torch.from_numpy(cache["v_witness"]))
     c.k_codes.copy_(torch.from_numpy(cache["k_codes"]))

@@ -14,7 +14,7 @@ HEADER = os.path.join(ROOT, "include", "witcert.h")
 def _declared():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"\b(wc_[a-z_]+)\s*\(", text)))
+    return sorted(set(re.findall(r"\b(wc_[a-z0-9_]+)\s*\(", text)))
 
 
 @pytest.fixture(scope="module")
@@ -103,3 +103,33 @@ def test_repair_host_validation_without_gpu(lib):
     assert sel(0, 8, 4) == 0                      # nothing to select, nothing launched
     assert sel(1, 8, 4, rp=None) == 1 and b"repair_pages" in lib.wc_last_error()
     assert sel(1, 8, 4, sn=vp(12)) == 1 and b"aligned" in lib.wc_last_error()
+
+
+def test_grouped_scheme_host_validation_without_gpu(lib):
+    import paper_2607_28699_gb300 as wc
+    vp = ctypes.c_void_p
+    d = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4, scheme=wc.SCHEME_DITHER_INT8_G32).c()
+    # the per-token entry points do not read a grouped cache
+    assert lib.wc_kv_quantize_witness(ctypes.byref(d), 0, vp(16), vp(16), vp(16), 1, vp(16), vp(16), vp(16),
+                                      vp(16), vp(16), None, None) == 2 and b"_g32" in lib.wc_last_error()
+    assert lib.wc_metered_decode_attention(ctypes.byref(d), 0, None, None, 1, None, 1, None, None, None,
+                                           None, None, None, None, None, None, 0, None) == 2
+    assert lib.wc_metered_decode_attention_noalloc(ctypes.byref(d), 0, None, None, 1, None, 1, None, None, None,
+                                                   None, None, None, None, None, None, None) == 2
+    g32 = lambda desc, m, kb=vp(16), pr=vp(16): lib.wc_kv_quantize_witness_g32(
+        ctypes.byref(desc), 0, vp(16), vp(16), vp(16), 0, vp(16), vp(16), vp(16), vp(16), vp(16), kb, pr, m,
+        None, None)
+    assert g32(d, 4) == 0                               # no tokens: nothing launched
+    assert g32(d, 17) == 1 and b"num_bypass_pairs" in lib.wc_last_error()
+    assert g32(d, 4, kb=None) == 1
+    assert g32(d, 4, kb=vp(8)) == 1 and b"aligned" in lib.wc_last_error()
+    assert g32(d, 0, kb=None, pr=None) == 0
+    d0 = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4).c()
+    assert g32(d0, 0) == 1 and b"WC_SCHEME_DITHER_INT8_G32" in lib.wc_last_error()
+    d10 = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4, scheme=2, dither_bits=10).c()
+    assert g32(d10, 0) == 2
+    lib.wc_workspace_size(ctypes.byref(d), 1, 8)      # accepted (without a GPU: no device to size for)
+    assert b"scheme" not in lib.wc_last_error() and b"_g32" not in lib.wc_last_error()
+    sel = lambda n, hkv, layout, m, pairs=vp(16): lib.wc_select_bypass_pairs(vp(16), n, hkv, layout, m, pairs, None)
+    assert sel(4, 2, 0, 0) == 0
+    assert sel(4, 2, 0, 17) == 1 and sel(4, 0, 0, 4) == 1 and sel(4, 2, 5, 4) == 2 and sel(4, 2, 0, 4, None) == 1
