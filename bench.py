@@ -168,7 +168,9 @@ class Setup:
         self.ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
         last = np.cumsum(wl.ctx_lens) - 1                       # index of each sequence's newest token
         self.new_slots = self.sm[torch.from_numpy(last).cuda()].contiguous()
-        self.caches, self.k_new, self.v_new, self.vcaches = [], [], [], []
+        self.caches, self.k_new, self.v_new, self.vcaches, self.gcaches = [], [], [], [], []
+        # the grouped-scale cache with the outlier-pair bypass (§6.2.3), pairs calibrated on the prefill
+        self.gdesc = dataclasses.replace(self.desc, scheme=wc.SCHEME_DITHER_INT8_G32, dither_bits=8)
         for layer in range(wl.n_layers):
             k, v = W.layer_kv(wl, layer, device="cuda")
             cache = wc.LayerCache.empty(self.desc)
@@ -179,6 +181,10 @@ class Setup:
                                                                   dtype=torch.float16, device="cuda"))
             wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, vc)
             self.vcaches.append(vc)
+            gc = wc.LayerCache.empty(self.gdesc, num_bypass_pairs=self.BYPASS_PAIRS)
+            wc.select_bypass_pairs(k, self.BYPASS_PAIRS, self.desc.rope_layout, pairs=gc.bypass_pairs)
+            wc.kv_quantize_witness(self.gdesc, layer, k, v, self.sm, gc)
+            self.gcaches.append(gc)
             li = torch.from_numpy(last).cuda()
             self.k_new.append(k[li].contiguous())
             self.v_new.append(v[li].contiguous())
@@ -202,6 +208,12 @@ class Setup:
         e.record()
         e.synchronize()
         self.write_v_call_s = s.elapsed_time(e) / 1e3 / reps
+        s.record()                                   # the grouped cache's write
+        for _ in range(reps):
+            wc.kv_quantize_witness(self.gdesc, wl.n_layers - 1, k, v, self.sm, self.gcaches[-1])
+        e.record()
+        e.synchronize()
+        self.write_g_call_s = s.elapsed_time(e) / 1e3 / reps
         del k, v
         self.q = torch.stack([W.layer_queries(wl, layer, device="cuda") for layer in range(wl.n_layers)])
         self.ws = wc.Workspace(self.desc, wl.batch, wl.max_pages)
@@ -242,6 +254,24 @@ class Setup:
                 value_term=self.vterm[layer], v_max=self.vmax[layer], out_bound=self.obound[layer])
 
     TIER_B_DELTA_REQ = 1e-2   # request-level budget, split over layers, query heads and one step
+    BYPASS_PAIRS = 4          # m, the paper's default budget (Table "bypassbudget")
+
+    def decode_all_grouped(self, tier_b=False):
+        """The same calls over the grouped-scale cache (meters into their own buffers)."""
+        wl = self.wl
+        if not hasattr(self, "g_raw"):
+            self.g_raw, self.g_meter, self.g_b, self.g_b_raw = (torch.empty_like(self.raw) for _ in range(4))
+        delta_loc = self.TIER_B_DELTA_REQ / (wl.n_layers * wl.n_q_heads)
+        for layer in range(wl.n_layers):
+            if tier_b:
+                self.wc.metered_decode_attention_tier_b(
+                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.ws, delta_loc,
+                    out=self.out[layer], meter=self.g_meter[layer], meter_raw=self.g_raw[layer],
+                    meter_b=self.g_b[layer], meter_b_raw=self.g_b_raw[layer])
+            else:
+                self.wc.metered_decode_attention(
+                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.ws,
+                    out=self.out[layer], meter=self.g_meter[layer], meter_raw=self.g_raw[layer])
 
     def decode_all_tier_b(self):
         """The same calls with the Tier-B certificate as well (§4.2; dithered INT8 only)."""
@@ -414,6 +444,17 @@ def run_ours(args, rank, world, local):
               "page_in_frac_vs_whole_head": float(nr.sum() / n_pages[flag].float().sum()) if nr.numel() else 0.0,
               "d_after_max": float(st.d_after[flag].max()) if nr.numel() else 0.0}
 
+    # ---- the grouped-scale cache with the outlier-pair bypass (§6.2.3) ----------
+    g_ms = graph_ms(st.decode_all_grouped, wl.n_layers)
+    gb_ms = graph_ms(lambda: st.decode_all_grouped(tier_b=True), wl.n_layers)
+    grouped = {"bypass_pairs": st.BYPASS_PAIRS, "decode_call_ms": g_ms, "overhead_vs_plain": g_ms / dec_avg_ms - 1.0,
+               "decode_tier_b_call_ms": gb_ms,
+               "write_ms_per_layer_prefill": st.write_g_call_s * 1e3,
+               "kept_frac_tier_a_at_tau": float((st.g_raw <= st.tau).float().mean()),
+               "kept_frac_tier_b_at_tau": float((st.g_b_raw <= st.tau).float().mean()),
+               "meter_raw_median": float(st.g_raw.median()), "meter_b_raw_median": float(st.g_b_raw.median()),
+               "bytes_per_token_head": st.gcaches[0].nbytes() / (wl.num_pages * 16 * wl.n_kv_heads)}
+
     kv_tokens_step = wl.kv_tokens
     value = kv_tokens_step * world / (ms / 1e3)
     algo_bytes = st.decode_bytes_per_launch()
@@ -452,6 +493,7 @@ def run_ours(args, rank, world, local):
         "tier_b": tier_b,
         "value_side": value_side,
         "repair": repair,
+        "grouped": grouped,
         "roofline": {"kernel": ("decode_ws_kernel" if wl.scheme == 0 and args.dither_bits == 8 else "decode_kernel")
                                + " + merge_kernel (one metered_decode_attention call)",
                      "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",

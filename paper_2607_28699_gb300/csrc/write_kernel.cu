@@ -435,7 +435,7 @@ __global__ void __launch_bounds__(256) select_pairs_kernel(const __half* __restr
     if (threadIdx.x < 64 && chosen[j]) {
         int pos = 0;
         for (int i = 0; i < j; ++i) pos += chosen[i];
-        pairs[(size_t)h * m + pos] = j;
+        if (pos < m) pairs[(size_t)h * m + pos] = j;   // NaN energies can make more than m ranks fall below m
     }
 }
 
