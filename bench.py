@@ -261,16 +261,17 @@ class Setup:
         wl = self.wl
         if not hasattr(self, "g_raw"):
             self.g_raw, self.g_meter, self.g_b, self.g_b_raw = (torch.empty_like(self.raw) for _ in range(4))
+            self.gws = self.wc.Workspace(self.gdesc, wl.batch, wl.max_pages)   # its own split plan
         delta_loc = self.TIER_B_DELTA_REQ / (wl.n_layers * wl.n_q_heads)
         for layer in range(wl.n_layers):
             if tier_b:
                 self.wc.metered_decode_attention_tier_b(
-                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.ws, delta_loc,
+                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.gws, delta_loc,
                     out=self.out[layer], meter=self.g_meter[layer], meter_raw=self.g_raw[layer],
                     meter_b=self.g_b[layer], meter_b_raw=self.g_b_raw[layer])
             else:
                 self.wc.metered_decode_attention(
-                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.ws,
+                    self.gdesc, layer, self.q[layer], self.bt, self.ctx, self.gcaches[layer], self.gws,
                     out=self.out[layer], meter=self.g_meter[layer], meter_raw=self.g_raw[layer])
 
     def decode_all_tier_b(self):
