@@ -1244,6 +1244,12 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
 
 static bool use_ws(int scheme, int bits) { return scheme == WC_SCHEME_DITHER_INT8 && bits == 8; }
 
+// Resident decode CTAs per SM: the warp-specialized kernel and the grouped
+// kernel take a whole SM, the per-token kernel two CTAs.
+static int ctas_per_sm(int scheme, int bits) {
+    return (use_ws(scheme, bits) || scheme == WC_SCHEME_DITHER_INT8_G32) ? 1 : kMinBlocks;
+}
+
 // Split plan.  A CTA's 8 page streams (warps or warp pairs) each take every
 // 8th page of its split, so a split of P pages costs ceil(P / 8) page steps,
 // and a wave of resident CTAs adds a fixed prologue / epilogue of about one
@@ -1254,7 +1260,7 @@ static bool use_ws(int scheme, int bits) { return scheme == WC_SCHEME_DITHER_INT
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits) {
     DecodePlan pl;
     const long units = (long)batch * num_kv_heads;
-    const long slots = std::max<long>(1, (long)num_sms * (use_ws(scheme, bits) ? 1 : kMinBlocks));
+    const long slots = std::max<long>(1, (long)num_sms * ctas_per_sm(scheme, bits));
     constexpr long kStreams = 8;      // page streams per CTA
     constexpr long kWaveCost2 = 3;    // per-wave fixed cost, in half page steps
     const long max_splits = std::max<long>(1, std::min<long>(max_pages / kStreams, 4 * slots));
