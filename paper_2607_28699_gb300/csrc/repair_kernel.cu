@@ -79,14 +79,19 @@ __global__ void __launch_bounds__(kSelThreads) repair_select_kernel(const __grid
 
     // ---- descending bitonic sort (skipped for kept cells: nothing is paged in) ----
     if (!kept) {
+        // exchange layout: position i lives at word i ^ sw(i / KPT), sw(t) a permutation of
+        // the thread's KPT words that gives the 16 lanes of a half-warp 16 distinct bank
+        // pairs; a partner i ^ j (j >= 32 KPT) flips only bits >= 5 of the thread index,
+        // which sw does not read, so loads use the same sw
+        const int sw = KPT >= 16 ? (tid & 15) : (((tid * KPT) >> 4) & (KPT - 1));
         for (int k = 2; k <= N; k <<= 1) {
             for (int j = k >> 1; j >= W; j >>= 1) {   // partner in another warp
                 const bool tm = bitonic_takes_max(base, j, k);
 #pragma unroll
-                for (int r = 0; r < KPT; ++r) xs[base + r] = key[r];
+                for (int r = 0; r < KPT; ++r) xs[(base + r) ^ sw] = key[r];
                 __syncthreads();
 #pragma unroll
-                for (int r = 0; r < KPT; ++r) key[r] = pick(tm, key[r], xs[(base + r) ^ j]);
+                for (int r = 0; r < KPT; ++r) key[r] = pick(tm, key[r], xs[((base + r) ^ j) ^ sw]);
                 __syncthreads();
             }
             for (int j = min(k >> 1, W >> 1); j >= KPT; j >>= 1) {   // partner in this warp
