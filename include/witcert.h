@@ -72,7 +72,8 @@ enum {
     WC_DEV_BAD_PAGE = 2u,     /* decode: block-table page outside [0, num_pages)  */
     WC_DEV_BAD_CTX = 4u,      /* decode: context length < 0 or > max_pages * 16   */
     WC_DEV_TIMEOUT = 8u,      /* decode: a bounded wait for staged data gave up   */
-    WC_DEV_BAD_PAIR = 16u     /* grouped scheme: a bypass pair outside [0, 64) is ignored */
+    WC_DEV_BAD_PAIR = 16u     /* grouped scheme: a bypass pair outside [0, 64), or listed
+                                 again, is ignored (its two stored values are 0) */
 };
 
 typedef enum {
@@ -354,7 +355,9 @@ wc_status wc_repair_select(const float* page_terms, const float* softmax_norm,
  * channel (0 on the bypassed ones).
  *   desc->scheme    WC_SCHEME_DITHER_INT8_G32 with dither_bits 8
  *   k_scale, v_scale, k_bypass, bypass_pairs  as in the layout above
- *   num_bypass_pairs  m in [0, 16]; k_bypass and bypass_pairs may be NULL if 0
+ *   num_bypass_pairs  m in [0, 16]; k_bypass and bypass_pairs may be NULL if 0.
+ *                   The pairs of a head should be distinct: an index outside [0, 64)
+ *                   or repeated is ignored (its entries store 0, WC_DEV_BAD_PAIR).
  *   dev_status      optional device uint32: WC_DEV_BAD_SLOT, WC_DEV_BAD_PAIR
  */
 wc_status wc_kv_quantize_witness_g32(const wc_cache_desc* desc, int32_t layer, const void* k,

@@ -120,12 +120,16 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
     const int32_t* prs = p.bypass_pairs + (size_t)h * m;
     uint32_t nmask = 0, pmask = 0, pvalid = 0;   // pvalid: bit t for a pair index in range
     uint32_t qb[4] = {0u, 0u, 0u, 0u};
+    uint32_t seen_lo = 0u, seen_hi = 0u;   // pair indices met so far: a repeated pair is ignored
     for (int t = 0; t < m; ++t) {
         const int j = __ldg(prs + t);
-        if (j < 0 || j >= kHeadDim / 2) {
+        const bool again = j >= 0 && j < kHeadDim / 2 && (((j < 32 ? seen_lo : seen_hi) >> (j & 31)) & 1u);
+        if (j < 0 || j >= kHeadDim / 2 || again) {
             if (threadIdx.x == 0 && split == 0) atomicOr(p.status, WC_DEV_BAD_PAIR);
             continue;
         }
+        if (j < 32) seen_lo |= 1u << j;
+        else seen_hi |= 1u << (j - 32);
         pvalid |= 1u << t;
         const int da = p.rope_layout == WC_ROPE_HALF ? j : 2 * j;
         const int db = p.rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;

@@ -84,11 +84,25 @@ __device__ __forceinline__ float pick16(const float (&x)[16], int i) {
     return v;
 }
 
+// Bypass set of one KV head in shared memory (grouped scheme, per-head grid):
+// the bypassed channels as a 128-bit mask, the k_bypass entry of each channel
+// (-1: not bypassed), and the pairs whose index is out of range.
+struct BypassTable {
+    uint32_t mask[4];
+    uint32_t bad;
+    int8_t entry[kHeadDim];
+};
+
+// Row stride of the grouped scheme's shared rows: 160 bytes puts the four
+// units of a warp on distinct bank groups.
+constexpr int kXRowStride = 160;
+
 // One row (K or V) of one (token, KV head): 8 lanes, 16 channels each.
-// xrow: the unit's 128-byte shared row (grouped scheme only).
+// xrow: the unit's shared row (grouped scheme only); tab: the head's bypass
+// table, or nullptr (then each K row reads the pair list itself).
 template <int kScheme, int kBits>
 __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2], int slot, bool live_unit, int h,
-                                          int row, int sub, uint8_t* xrow) {
+                                          int row, int sub, uint8_t* xrow, const BypassTable* tab) {
     constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
     constexpr bool kDither = kScheme != WC_SCHEME_FP8_E4M3;
     const bool bad = slot >= p.num_pages * kPage;
@@ -114,7 +128,9 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
     float s = 0.0f;
     uint32_t bmask = 0;   // grouped K rows: bypassed channels among 16 sub .. 16 sub + 15
     if constexpr (kGrouped) {
-        if (row == 0) {
+        if (row == 0 && tab != nullptr) {
+            bmask = (tab->mask[sub >> 1] >> (16 * (sub & 1))) & 0xFFFFu;
+        } else if (row == 0) {
             const int32_t* pr = p.bypass_pairs + (size_t)h * p.num_bypass;
             for (int t = 0; t < p.num_bypass; ++t) {
                 const int j = __ldg(pr + t);
@@ -289,9 +305,20 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         }
         if constexpr (kGrouped) {
             if ((sub & 1) == 0) (row == 0 ? p.k_scale : p.v_scale)[rowidx * 4 + (sub >> 1)] = __float2half_rn(s);
-            if (row == 0 && p.num_bypass > 0) {   // the exact values of the bypassed pairs, pair by pair
+            if (row == 0 && p.num_bypass > 0 && tab != nullptr) {
+                __half* bdst = p.k_bypass + rowidx * (2 * p.num_bypass);
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    if ((bmask >> i) & 1u) bdst[tab->entry[16 * sub + i]] = __float2half_rn(x[i]);
+                if (sub == 0)   // an ignored pair stores zeros
+                    for (uint32_t bad = tab->bad; bad != 0u; bad &= bad - 1u) {
+                        const int t = __ffs(bad) - 1;
+                        bdst[2 * t] = bdst[2 * t + 1] = __float2half_rn(0.0f);
+                    }
+            } else if (row == 0 && p.num_bypass > 0) {   // the exact values of the bypassed pairs, pair by pair
                 const int32_t* pr = p.bypass_pairs + (size_t)h * p.num_bypass;
                 __half* bdst = p.k_bypass + rowidx * (2 * p.num_bypass);
+                uint32_t seen = 0;   // this lane's channels stored already: a repeated pair stores zeros
                 for (int t = 0; t < p.num_bypass; ++t) {
                     const int j = __ldg(pr + t);
                     if (j < 0 || j >= kHeadDim / 2) {   // an ignored pair stores zeros
@@ -300,8 +327,17 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
                     }
                     const int a = p.rope_layout == WC_ROPE_HALF ? j : 2 * j;
                     const int b = p.rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
-                    if ((a >> 4) == sub) bdst[2 * t] = __float2half_rn(pick16(x, a & 15));
-                    if ((b >> 4) == sub) bdst[2 * t + 1] = __float2half_rn(pick16(x, b & 15));
+                    if ((a >> 4) == sub) {
+                        const bool again = (seen >> (a & 15)) & 1u;
+                        bdst[2 * t] = __float2half_rn(again ? 0.0f : pick16(x, a & 15));
+                        if (again && live_unit && p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_PAIR);
+                        seen |= 1u << (a & 15);
+                    }
+                    if ((b >> 4) == sub) {
+                        const bool again = (seen >> (b & 15)) & 1u;
+                        bdst[2 * t + 1] = __float2half_rn(again ? 0.0f : pick16(x, b & 15));
+                        seen |= 1u << (b & 15);
+                    }
                 }
             }
         }
@@ -358,10 +394,38 @@ constexpr int kPerHeadMinTokens = 16;                     // per-head grid from 
 template <int kScheme, int kBits, bool kPerHead>
 __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ WriteParams p) {
     constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
-    __shared__ __align__(16) uint8_t xrows[kGrouped ? 4 * 4 * kHeadDim : 16];   // [warp][unit][128]
+    __shared__ __align__(16) uint8_t xrows[kGrouped ? 4 * 4 * kXRowStride : 16];   // [warp][unit][row]
+    __shared__ BypassTable btab;
     grid_dep_launch();    // a dependent decode may be scheduled now: it waits for this whole grid
     grid_dep_wait();      // inputs may come from the preceding kernel
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const BypassTable* tab = nullptr;
+    if constexpr (kGrouped && kPerHead) {   // one KV head per CTA: its bypass set, once
+        if (threadIdx.x < kHeadDim) btab.entry[threadIdx.x] = -1;
+        if (threadIdx.x < 4) btab.mask[threadIdx.x] = 0u;
+        if (threadIdx.x == 0) btab.bad = 0u;
+        __syncthreads();
+        if (threadIdx.x < p.num_bypass) {
+            const int t = threadIdx.x;
+            const int32_t* pr = p.bypass_pairs + (size_t)blockIdx.y * p.num_bypass;
+            const int j = __ldg(pr + t);
+            bool dup = false;   // a pair listed again is ignored after its first occurrence
+            for (int u = 0; u < t; ++u) dup = dup || __ldg(pr + u) == j;
+            if (j < 0 || j >= kHeadDim / 2 || dup) {
+                atomicOr(&btab.bad, 1u << t);
+                if (p.dev_status) atomicOr(p.dev_status, WC_DEV_BAD_PAIR);
+            } else {
+                const int a = p.rope_layout == WC_ROPE_HALF ? j : 2 * j;
+                const int b = p.rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+                btab.entry[a] = (int8_t)(2 * t);
+                btab.entry[b] = (int8_t)(2 * t + 1);
+                atomicOr(&btab.mask[a >> 5], 1u << (a & 31));
+                atomicOr(&btab.mask[b >> 5], 1u << (b & 31));
+            }
+        }
+        __syncthreads();
+        tab = &btab;
+    }
     // Warps 0, 2 take the K rows and warps 1, 3 the V rows of the same units,
     // so the residual and witness work stays in whole warps; lanes 8i .. 8i+7
     // own unit i of a 4-unit task.
@@ -400,7 +464,7 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
     for (int t = 0; t < kWriteTasks; ++t)
         if (__any_sync(0xffffffffu, live[t]))   // warp-uniform: a task past the end is skipped whole
             write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub,
-                                      kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kHeadDim : xrows);
+                                      kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab);
 }
 
 // Bypass-pair calibration: one CTA per KV head; thread t sums pair t % 64

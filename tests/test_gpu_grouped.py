@@ -177,3 +177,33 @@ def test_out_of_range_pair_is_reported_and_ignored():
     torch.cuda.synchronize()
     assert wc.read_status(ws) & wc.DEV_BAD_PAIR
     assert torch.isfinite(out).all() and torch.isfinite(raw).all()
+
+
+def test_repeated_pair_is_ignored_like_an_out_of_range_one():
+    """A pair listed twice counts once: its second occurrence is reported and
+    stores zeros, exactly like an out-of-range index in its place."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("gr", 1, 8, 2, [300, 20], shuffle_pages=True, seed=73)
+    bt, sm, k, v, q = make_inputs(wl, 0)
+    k = _massive(k.numpy(), np.array([[5, 11], [7, 8]]), Q.ROPE_HALF)
+    gd = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=wl.num_pages, scheme=wc.SCHEME_DITHER_INT8_G32)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    res = []
+    for pairs in ([[5, 11, 5], [7, 8, 8]], [[5, 11, -1], [7, 8, 64]]):
+        for n_split in (None, 3):   # the per-head grid (all tokens) and the one-index grid (3 tokens at a time)
+            cache = wc.LayerCache.empty(gd, num_bypass_pairs=3)
+            cache.bypass_pairs.copy_(torch.tensor(pairs, dtype=torch.int32))
+            status = torch.zeros(1, dtype=torch.int32, device="cuda")
+            kd, vd, sd = torch.from_numpy(k).cuda(), v.cuda(), torch.from_numpy(sm).cuda()
+            chunks = [slice(0, len(sm))] if n_split is None else [slice(i, i + n_split) for i in range(0, len(sm), n_split)]
+            for ch in chunks:
+                wc.kv_quantize_witness(gd, 0, kd[ch].contiguous(), vd[ch].contiguous(), sd[ch].contiguous(), cache,
+                                       dev_status=status)
+            ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+            out, meter, raw = wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx, cache, ws)
+            torch.cuda.synchronize()
+            assert int(status.item()) & wc.DEV_BAD_PAIR and wc.read_status(ws) & wc.DEV_BAD_PAIR
+            res.append((cache.k_codes.clone(), cache.k_bypass.clone(), out, raw))
+    for other in res[1:]:
+        for a, b in zip(res[0], other):
+            assert torch.equal(a, b)
