@@ -2,6 +2,8 @@
 // mma.sync m16n8k16 / m16n8k8 and the exact int8 / dither -> fp16 operands).
 #pragma once
 
+#include <cuda.h>
+
 #include <climits>
 
 #include "wc_kernels.cuh"
@@ -54,7 +56,25 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
     return y;
 }
 
+// Byte offset of 16-byte chunk q of token row t in a tile written with the
+// 128-byte swizzle (tile 1024-byte aligned): chunk q of row t sits at chunk
+// q ^ (t & 7), so the 8 rows a warp touches per instruction hit distinct banks.
+__device__ __forceinline__ int swz(int t, int q) { return t * kHeadDim + 16 * (q ^ (t & 7)); }
+
+__device__ __forceinline__ void tma_page(void* dst, const CUtensorMap* map, int z, uint64_t* bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
+        "[%5];" ::"r"(smem_addr(dst)),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(z), "r"(smem_addr(bar))
+        : "memory");
+}
+
 }  // namespace
+
+// One layer's code array [num_pages][Hkv][16][128] bytes as a 3-D tensor map
+// (channel, slot, page * Hkv + head) whose box is one page of one head,
+// written to shared memory with the 128-byte swizzle (swz above).
+bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, int num_kv_heads);
 
 // The split-K merge for the extra outputs in the bit mask x (0, kXTierB,
 // kXValue or kXRepair), launched as a programmatic dependent of the decode.

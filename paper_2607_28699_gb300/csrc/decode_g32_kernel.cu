@@ -1,8 +1,9 @@
 // Metered decode attention over the grouped-scale cache (§6.2.3 "Storage
 // side" and "Fixed-channel outlier bypass"): one fp16 scale per token and
 // 32-channel group, and the m key RoPE pairs of a (layer, KV head) stored
-// exactly.  The structure is the per-token kernel's (8 warps, a bulk-copy
-// ring per warp, the same split-K partials and merge); what differs:
+// exactly.  The structure is the per-token kernel's (8 warps, a copy ring per
+// warp, the same split-K partials and merge; code tiles by tensor-map TMA with
+// the 128-byte swizzle as in the warp-specialized kernel); what differs:
 //
 //  - A row is stored in the order the mma fragments consume it (storage
 //    position p of K holds channel 16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3),
@@ -31,16 +32,25 @@ constexpr int kGMinBlocks = 1;   // one CTA per SM: the kernel needs ~205 regist
 // stage: K codes | V codes | K scales [16][4] | V scales [16][4] | witness [16][8] | bypass [16][2m]
 constexpr int kGOffV = 2048, kGOffKs = 4096, kGOffVs = 4224, kGOffW = 4352, kGOffB = 4608;
 constexpr int kGMaxBypass = 16;
-constexpr int kGStageStride = kGOffB + 16 * 2 * kGMaxBypass * 2;
-constexpr int kGSmemBytes = kGWarps * kGStages * kGStageStride + kGWarps * kGStages * 8;
+constexpr int kGStageStride = 6144;   // 1024-aligned: the code tiles land with the 128-byte swizzle
+static_assert(kGOffB + 16 * 2 * kGMaxBypass * 2 <= kGStageStride, "stage layout");
+constexpr int kGSmemBytes = kGWarps * kGStages * kGStageStride + kGWarps * kGStages * 8 + 1024;   // + alignment
+
+struct G32Params {
+    CUtensorMap k_map;   // k_codes as [num_pages * Hkv][16][128] bytes, box = one page of one head
+    CUtensorMap v_map;
+    DecodeParams p;
+};
 static_assert(kGWarps * kMaxGroup * kPartialStride * 4 <= kGWarps * kGStages * kGStageStride, "merge buffer");
 static_assert(kGSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
 
 template <int kX>
-__global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(const __grid_constant__ DecodeParams p) {
+__global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(const __grid_constant__ G32Params gparams) {
     constexpr bool kTierB = (kX & kXTierB) != 0;
     constexpr float kKappa = DitherConst<8>::kappa;
-    extern __shared__ __align__(128) uint8_t smem[];
+    const DecodeParams& p = gparams.p;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
     const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
@@ -102,8 +112,8 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
         uint8_t* st = my_stages + (k % kGStages) * kGStageStride;
         const size_t ph = (size_t)phys * p.num_kv_heads + h;
         mbar_arrive_expect_tx(bar, (uint32_t)(kGOffB + 64 * m));
-        bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, bar);
-        bulk_g2s(st + kGOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, bar);
+        tma_page(st, &gparams.k_map, (int)ph, bar);
+        tma_page(st + kGOffV, &gparams.v_map, (int)ph, bar);
         bulk_g2s(st + kGOffKs, p.k_scale + ph * (kPage * 4), 128, bar);
         bulk_g2s(st + kGOffVs, p.v_scale + ph * (kPage * 4), 128, bar);
         bulk_g2s(st + kGOffW, p.k_witness + ph * (kPage * kBands), 256, bar);
@@ -259,8 +269,8 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             float raw[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {   // storage positions 32c + 16gp .. +15: k-steps 4gp .. 4gp+3
-                const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + 32 * c + 16 * gp);
-                const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + 32 * c + 16 * gp);
+                const uint4 ka = *reinterpret_cast<const uint4*>(st + swz(g, 2 * c + gp));
+                const uint4 kb = *reinterpret_cast<const uint4*>(st + swz(g + 8, 2 * c + gp));
                 const uint4 da = philox(slot0 + g, c1, (uint32_t)(2 * c + gp), 0u, p.keys);
                 const uint4 db = philox(slot0 + g + 8, c1, (uint32_t)(2 * c + gp), 0u, p.keys);
                 float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
@@ -380,7 +390,7 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             uint4 vq[4], dv[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                vq[j] = *reinterpret_cast<const uint4*>(st + kGOffV + tv[j] * kHeadDim + 16 * g);
+                vq[j] = *reinterpret_cast<const uint4*>(st + kGOffV + swz(tv[j], g));
                 dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
             }
 #pragma unroll
@@ -523,8 +533,13 @@ cudaError_t launch_g32(const DecodeParams& p, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
+    G32Params gp;
+    gp.p = p;
+    if (!encode_page_map(&gp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
+        !encode_page_map(&gp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
+        return cudaErrorInvalidValue;
     const dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_g32_kernel<kX>, grid, dim3(kGThreads), kGSmemBytes, stream, p);
+    cudaError_t e = launch_pdl(decode_g32_kernel<kX>, grid, dim3(kGThreads), kGSmemBytes, stream, gp);
     if (e != cudaSuccess) return e;
     return launch_merge_x(p, kX, stream);
 }

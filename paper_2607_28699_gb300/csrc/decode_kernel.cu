@@ -617,19 +617,6 @@ struct WsParams {
     DecodeParams p;
 };
 
-// Byte offset of 16-byte chunk q of token row t in a tile written with the
-// 128-byte swizzle (tile 1024-byte aligned): chunk q of row t sits at chunk
-// q ^ (t & 7), so the 8 rows a warp touches per instruction hit distinct banks.
-__device__ __forceinline__ int swz(int t, int q) { return t * kHeadDim + 16 * (q ^ (t & 7)); }
-
-__device__ __forceinline__ void tma_page(void* dst, const CUtensorMap* map, int z, uint64_t* bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], "
-        "[%5];" ::"r"(smem_addr(dst)),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(0), "r"(0), "r"(z), "r"(smem_addr(bar))
-        : "memory");
-}
-
 __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
 }
@@ -1360,7 +1347,7 @@ static PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
 // One layer's code array [num_pages][Hkv][16][128] bytes as a 3-D tensor
 // (channel, slot, page * Hkv + head); a box is one page of one head, written
 // to shared memory with the 128-byte swizzle.
-static bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, int num_kv_heads) {
+bool encode_page_map(CUtensorMap* map, const void* codes, int num_pages, int num_kv_heads) {
     PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
     if (!enc) return false;
     const cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)kPage, (cuuint64_t)num_pages * num_kv_heads};
