@@ -231,12 +231,23 @@ class Setup:
                                          self.ws, out=self.out[layer], meter=self.meter[layer],
                                          meter_raw=self.raw[layer])
 
+    @property
+    def fused_append(self):
+        """The step writes each new token inside the decode (dithered INT8, 8-bit dither)."""
+        return self.wl.scheme == 0 and self.desc.dither_bits == 8
+
     def step(self):
         wc, wl = self.wc, self.wl
         for layer in range(wl.n_layers):
-            wc.kv_quantize_witness(self.desc, layer, self.k_new[layer], self.v_new[layer], self.new_slots,
-                                   self.caches[layer])
-            self.decode(layer)
+            if self.fused_append:
+                wc.metered_decode_attention_append(
+                    self.desc, layer, self.q[layer], self.bt, self.ctx, self.caches[layer], self.ws,
+                    self.k_new[layer], self.v_new[layer], self.new_slots, out=self.out[layer],
+                    meter=self.meter[layer], meter_raw=self.raw[layer])
+            else:
+                wc.kv_quantize_witness(self.desc, layer, self.k_new[layer], self.v_new[layer], self.new_slots,
+                                       self.caches[layer])
+                self.decode(layer)
         wc.gate(self.raw.reshape(-1), wl.group, self.tau, self.keep_q, self.keep_kv, self.n_kept)
 
     def decode_all(self):
@@ -320,8 +331,9 @@ class Setup:
                               d_after=self.d_after.view(L * B, Hq))
 
     def launches_per_step(self):
-        # per layer: write kernel, decode kernel, merge kernel; then one gate
-        return 3 * self.wl.n_layers + 1
+        # per layer: decode kernel (with the new token's write fused) and merge kernel,
+        # or write, decode and merge kernels; then one gate
+        return (2 if self.fused_append else 3) * self.wl.n_layers + 1
 
     def decode_bytes_per_launch(self):
         return sum(self.wl.ctx_lens) * self.wl.n_kv_heads * BYTES_PER_TOKEN_HEAD[self.wl.scheme]
@@ -488,6 +500,8 @@ def run_ours(args, rank, world, local):
                    "kv_heads": wl.n_kv_heads, "head_dim": 128, "batch": wl.batch,
                    "ctx_tokens": sum(wl.ctx_lens), "page": 16, "dither_bits": args.dither_bits,
                    "tau": st.tau, "parallelism": f"replica-per-gpu x{world}",
+                   "step": "write of each new token fused into its decode" if st.fused_append
+                           else "write kernel, then decode",
                    "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step > 129 MB L2; no flush"},
         "hbm_gbs_step": step_gbs,
         "decode_call_ms": dec_avg_ms,

@@ -72,8 +72,10 @@ enum {
     WC_DEV_BAD_PAGE = 2u,     /* decode: block-table page outside [0, num_pages)  */
     WC_DEV_BAD_CTX = 4u,      /* decode: context length < 0 or > max_pages * 16   */
     WC_DEV_TIMEOUT = 8u,      /* decode: a bounded wait for staged data gave up   */
-    WC_DEV_BAD_PAIR = 16u     /* grouped scheme: a bypass pair outside [0, 64), or listed
+    WC_DEV_BAD_PAIR = 16u,    /* grouped scheme: a bypass pair outside [0, 64), or listed
                                  again, is ignored (its two stored values are 0) */
+    WC_DEV_BAD_APPEND = 32u   /* append: slot_new[b] is not the slot of the context's last
+                                 token; the token is not written */
 };
 
 typedef enum {
@@ -286,6 +288,33 @@ wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t
                                               const void* k_witness,
                                               float* out, float* meter, float* meter_raw,
                                               uint32_t* dev_status, void* stream);
+
+/*
+ * One decode step with the write of its new token fused in: the effect of
+ * wc_kv_quantize_witness for the tokens k_new[b], v_new[b] at slots
+ * slot_new[b] (codes, scales, K witness; no value witness), followed by
+ * wc_metered_decode_attention, in one pair of launches.  The new token of
+ * sequence b is the last of its context: slot_new[b] must be the slot of
+ * logical position ctx_lens[b] - 1 (block_table[b][(ctx - 1) / 16] * 16 +
+ * (ctx - 1) % 16); otherwise it is not written and WC_DEV_BAD_APPEND is set.
+ * slot_new[b] < 0: no new token for sequence b.  The token is quantized by
+ * the CTA that reads the sequence's last page, before it reads it.
+ *   k_new, v_new  [batch][Hkv][128] fp16 post-RoPE, device, 16-byte aligned
+ *   slot_new      [batch] int32, device
+ * The cache arrays are written, hence not const.  WC_ERR_UNSUPPORTED for any
+ * scheme but WC_SCHEME_DITHER_INT8 with dither_bits 8 (write, then decode).
+ */
+wc_status wc_metered_decode_attention_append(const wc_cache_desc* desc, int32_t layer,
+                                             const void* q, const int32_t* block_table,
+                                             int32_t max_pages, const int32_t* ctx_lens,
+                                             int32_t batch,
+                                             void* k_codes, void* v_codes,
+                                             void* k_scale, void* v_scale, void* k_witness,
+                                             const void* k_new, const void* v_new,
+                                             const int32_t* slot_new,
+                                             float* out, float* meter, float* meter_raw,
+                                             void* workspace, size_t workspace_bytes,
+                                             void* stream);
 
 /*
  * Metered decode attention with the per-page terms of block-level repair

@@ -30,12 +30,13 @@ SCHEME_FP8_E4M3 = 1
 SCHEME_DITHER_INT8_G32 = 2
 ROPE_HALF = 0
 ROPE_INTERLEAVED = 1
-DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT, DEV_BAD_PAIR = 1, 2, 4, 8, 16
+DEV_BAD_SLOT, DEV_BAD_PAGE, DEV_BAD_CTX, DEV_TIMEOUT, DEV_BAD_PAIR, DEV_BAD_APPEND = 1, 2, 4, 8, 16, 32
 EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_attention",
            "wc_metered_decode_attention_tier_b", "wc_metered_decode_attention_noalloc",
            "wc_kv_quantize_witness_v", "wc_metered_decode_attention_v", "wc_gate_joint",
            "wc_metered_decode_attention_repair", "wc_repair_select",
            "wc_kv_quantize_witness_g32", "wc_metered_decode_attention_g32", "wc_select_bypass_pairs",
+           "wc_metered_decode_attention_append",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -83,6 +84,9 @@ def _load():
     lib.wc_metered_decode_attention_g32.restype = ctypes.c_int
     lib.wc_select_bypass_pairs.argtypes = [vp, i32, i32, i32, i32, vp, vp]
     lib.wc_select_bypass_pairs.restype = ctypes.c_int
+    lib.wc_metered_decode_attention_append.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp, vp, vp,
+                                                       vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    lib.wc_metered_decode_attention_append.restype = ctypes.c_int
     lib.wc_read_status.argtypes = [vp, i32, vp, vp]
     lib.wc_read_status.restype = ctypes.c_int
     lib.wc_last_error.argtypes = []
@@ -253,6 +257,28 @@ def metered_decode_attention(desc: CacheDesc, layer: int, q: torch.Tensor, block
         _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
         _ptr(cache.k_witness), _ptr(out), _ptr(meter), _ptr(meter_raw), ws.ptr(), ws.nbytes,
         _stream(stream)))
+    return out, meter, meter_raw
+
+
+def metered_decode_attention_append(desc: CacheDesc, layer: int, q: torch.Tensor, block_table: torch.Tensor,
+                                    ctx_lens: torch.Tensor, cache: LayerCache, ws: Workspace, k_new: torch.Tensor,
+                                    v_new: torch.Tensor, slot_new: torch.Tensor, out=None, meter=None,
+                                    meter_raw=None, stream=None):
+    """``wc_metered_decode_attention_append``: writes each sequence's new token (k_new, v_new fp16
+    [B, Hkv, 128] at slot_new int32 [B], the last of its context) and decodes, in one step;
+    returns (out, meter, meter_raw)."""
+    batch, max_pages = block_table.shape
+    dev = q.device
+    cells = (batch, desc.num_q_heads)
+    out = torch.empty(batch, desc.num_q_heads, desc.head_dim, dtype=torch.float32, device=dev) if out is None else out
+    meter = torch.empty(cells, dtype=torch.float32, device=dev) if meter is None else meter
+    meter_raw = torch.empty(cells, dtype=torch.float32, device=dev) if meter_raw is None else meter_raw
+    d = desc.c()
+    _check(lib.wc_metered_decode_attention_append(
+        ctypes.byref(d), layer, _ptr(q), _ptr(block_table), max_pages, _ptr(ctx_lens), batch,
+        _ptr(cache.k_codes), _ptr(cache.v_codes), _ptr(cache.k_scale), _ptr(cache.v_scale),
+        _ptr(cache.k_witness), _ptr(k_new), _ptr(v_new), _ptr(slot_new), _ptr(out), _ptr(meter), _ptr(meter_raw),
+        ws.ptr(), ws.nbytes, _stream(stream)))
     return out, meter, meter_raw
 
 

@@ -211,8 +211,21 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
                                        float* value_term, float* v_max, float* out_bound, float* page_terms,
                                        float* softmax_norm, void* workspace, size_t workspace_bytes,
                                        void* stream, bool grouped = false, const void* k_bypass = nullptr,
-                                       const int32_t* bypass_pairs = nullptr, int32_t num_bypass = 0) {
+                                       const int32_t* bypass_pairs = nullptr, int32_t num_bypass = 0,
+                                       const void* k_new = nullptr, const void* v_new = nullptr,
+                                       const int32_t* slot_new = nullptr) {
     if (wc_status st = check_desc(desc, grouped)) return st;
+    if (k_new || v_new || slot_new) {
+        if (!k_new || !v_new || !slot_new)
+            return fail(WC_ERR_INVALID_ARG, "k_new, v_new and slot_new must not be NULL");
+        if (!aligned16(k_new) || !aligned16(v_new))
+            return fail(WC_ERR_INVALID_ARG, "k_new and v_new must be 16-byte aligned");
+        if (desc->scheme != WC_SCHEME_DITHER_INT8 || desc->dither_bits != 8)
+            return fail(WC_ERR_UNSUPPORTED,
+                        "the fused append is implemented for the dithered INT8 cache with the 8-bit dither");
+        if (meter_b || value_term || page_terms)
+            return fail(WC_ERR_UNSUPPORTED, "the append, Tier B, the value side and the repair terms are separate calls");
+    }
     if (grouped) {
         if (desc->scheme != WC_SCHEME_DITHER_INT8_G32)
             return fail(WC_ERR_INVALID_ARG, "the _g32 entry points need desc->scheme = WC_SCHEME_DITHER_INT8_G32");
@@ -280,6 +293,9 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.k_bypass = static_cast<const __half*>(k_bypass);
     p.bypass_pairs = bypass_pairs;
     p.num_bypass = num_bypass;
+    p.k_new = static_cast<const __half*>(k_new);
+    p.v_new = static_cast<const __half*>(v_new);
+    p.slot_new = slot_new;
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
@@ -349,6 +365,20 @@ wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t 
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
                                  nullptr, nullptr, page_terms, softmax_norm, workspace, workspace_bytes, stream);
+}
+
+wc_status wc_metered_decode_attention_append(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                             const int32_t* block_table, int32_t max_pages,
+                                             const int32_t* ctx_lens, int32_t batch, void* k_codes, void* v_codes,
+                                             void* k_scale, void* v_scale, void* k_witness, const void* k_new,
+                                             const void* v_new, const int32_t* slot_new, float* out, float* meter,
+                                             float* meter_raw, void* workspace, size_t workspace_bytes,
+                                             void* stream) {
+    if (!k_new || !v_new || !slot_new) return fail(WC_ERR_INVALID_ARG, "k_new, v_new and slot_new must not be NULL");
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
+                                 nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream, false,
+                                 nullptr, nullptr, 0, k_new, v_new, slot_new);
 }
 
 wc_status wc_metered_decode_attention_g32(const wc_cache_desc* desc, int32_t layer, const void* q,

@@ -27,6 +27,7 @@
 #include <mutex>
 
 #include "decode_common.cuh"
+#include "write_row.cuh"
 
 namespace wc {
 
@@ -615,7 +616,38 @@ struct WsParams {
     CUtensorMap k_map;   // k_codes as [num_pages * Hkv][16][128] bytes, box = one page of one head
     CUtensorMap v_map;
     DecodeParams p;
+    WriteParams w;       // the cache as the write path sees it (append variant)
 };
+
+// Append (kXAppend): the step's new token of sequence b, the last of its
+// context, is quantized and stored by the producer warp that stages the
+// sequence's last page, before that page's copies are issued.  Its slot must
+// be that of the context's last token (else WC_DEV_BAD_APPEND, not written),
+// so no other CTA reads it.  Lanes 0-7 hold the row (write path layout); the
+// generic-proxy stores are fenced against the async-proxy copies that follow.
+__device__ __forceinline__ void append_new_token(const WsParams& wp, int b, int h, int phys, int ctx, int lane) {
+    const DecodeParams& p = wp.p;
+    const int slot = __ldg(p.slot_new + b);
+    if (slot < 0) return;   // warp-uniform: no new token for this sequence
+    if (slot != phys * kPage + (ctx - 1) % kPage) {
+        if (lane == 0) atomicOr(p.status, WC_DEV_BAD_APPEND);
+        return;
+    }
+    const bool live = lane < 8;
+    const int sub = lane & 7;
+    const size_t off = ((size_t)b * p.num_kv_heads + h) * kHeadDim + sub * 16;
+    uint4 rk[2] = {make_uint4(0, 0, 0, 0), make_uint4(0, 0, 0, 0)}, rv[2] = {rk[0], rk[1]};
+    if (live) {
+        rk[0] = __ldg(reinterpret_cast<const uint4*>(p.k_new + off));
+        rk[1] = __ldg(reinterpret_cast<const uint4*>(p.k_new + off) + 1);
+        rv[0] = __ldg(reinterpret_cast<const uint4*>(p.v_new + off));
+        rv[1] = __ldg(reinterpret_cast<const uint4*>(p.v_new + off) + 1);
+    }
+    write_row<WC_SCHEME_DITHER_INT8, 8>(wp.w, rk, slot, live, h, 0, sub, nullptr, nullptr);
+    write_row<WC_SCHEME_DITHER_INT8, 8>(wp.w, rv, slot, live, h, 1, sub, nullptr, nullptr);
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+    __syncwarp();
+}
 
 __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
@@ -637,6 +669,7 @@ __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h,
 template <int kX>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
     constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
+    constexpr bool kAppend = (kX & kXAppend) != 0;
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -716,6 +749,9 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             if (k + 1 < n_my) phys_next = __ldg(bt_row + p0 + pw + kWsPairs * (k + 1));
             const bool ok = phys >= 0 && phys < p.num_pages;
             uint8_t* st = stages + s * kWsStageBytes;
+            if constexpr (kAppend) {   // the sequence's last page: store the new token first
+                if (ok && p0 + pw + kWsPairs * k == npages - 1) append_new_token(wp, b, h, phys, ctx, lane);
+            }
             if (lane == 0) {
                 *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
                 if (ok) {
@@ -1373,13 +1409,31 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     }
     WsParams wp;
     wp.p = p;
+    if constexpr ((kX & kXAppend) != 0) {   // the cache as the write path sees it
+        WriteParams& w = wp.w;
+        w.k = w.v = nullptr;
+        w.slot_mapping = p.slot_new;
+        w.k_codes = const_cast<uint8_t*>(p.k_codes);
+        w.v_codes = const_cast<uint8_t*>(p.v_codes);
+        w.k_scale = const_cast<__half*>(p.k_scale);
+        w.v_scale = const_cast<__half*>(p.v_scale);
+        w.k_witness = const_cast<__half*>(p.k_witness);
+        w.v_witness = nullptr;
+        w.dev_status = p.status;
+        w.n_tok = p.batch;
+        w.num_kv_heads = p.num_kv_heads;
+        w.num_pages = p.num_pages;
+        w.layer = p.layer;
+        w.rope_layout = p.rope_layout;
+        w.keys = p.keys;
+    }
     if (!encode_page_map(&wp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
         !encode_page_map(&wp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
     cudaError_t e = launch_pdl(decode_ws_kernel<kX>, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
-    return launch_merge<kX>(p, stream);
+    return launch_merge<kX & ~kXAppend>(p, stream);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
@@ -1387,7 +1441,8 @@ cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStrea
     if (scheme == WC_SCHEME_DITHER_INT8_G32) return launch_decode_g32(p, stream);
     // Tier B (dithered INT8 only), the value side and the repair terms are
     // requested by separate entry points, never together (checked by the caller)
-    const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0) | (p.page_terms ? kXRepair : 0);
+    const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0) | (p.page_terms ? kXRepair : 0) |
+                  (p.k_new ? kXAppend : 0);
     if (scheme == WC_SCHEME_FP8_E4M3)
         return x == kXValue  ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
              : x == kXRepair ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXRepair>(p, stream)
@@ -1395,7 +1450,8 @@ cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStrea
     if (use_ws(scheme, bits))
         return x == kXTierB  ? launch_ws<kXTierB>(p, stream)
              : x == kXValue  ? launch_ws<kXValue>(p, stream)
-             : x == kXRepair ? launch_ws<kXRepair>(p, stream) : launch_ws<0>(p, stream);
+             : x == kXRepair ? launch_ws<kXRepair>(p, stream)
+             : x == kXAppend ? launch_ws<kXAppend>(p, stream) : launch_ws<0>(p, stream);
     return x == kXTierB  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
          : x == kXValue  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
          : x == kXRepair ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXRepair>(p, stream)

@@ -50,6 +50,11 @@ struct DecodeParams {
     // per (sequence, query head): (M, L), the final log2-domain maximum and sum.
     float2* page_terms = nullptr;     // [batch][Hq][max_pages]
     float2* softmax_norm = nullptr;   // [batch][Hq]
+    // append: the step's new token of each sequence, quantized and stored by the
+    // decode itself before it reads it (nullptr: none)
+    const __half* k_new = nullptr;     // [batch][Hkv][128] fp16
+    const __half* v_new = nullptr;
+    const int32_t* slot_new = nullptr;   // [batch], < 0: no new token
     // grouped scheme: exact bypassed key values [slot][2m] and the pair set [Hkv][m]
     const __half* k_bypass = nullptr;
     const int32_t* bypass_pairs = nullptr;

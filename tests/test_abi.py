@@ -133,3 +133,18 @@ def test_grouped_scheme_host_validation_without_gpu(lib):
     sel = lambda n, hkv, layout, m, pairs=vp(16): lib.wc_select_bypass_pairs(vp(16), n, hkv, layout, m, pairs, None)
     assert sel(4, 2, 0, 0) == 0
     assert sel(4, 2, 0, 17) == 1 and sel(4, 0, 0, 4) == 1 and sel(4, 2, 5, 4) == 2 and sel(4, 2, 0, 4, None) == 1
+
+
+def test_append_host_validation_without_gpu(lib):
+    import paper_2607_28699_gb300 as wc
+    vp = ctypes.c_void_p
+    call = lambda desc, kn=vp(16), vn=vp(16), sn=vp(16): lib.wc_metered_decode_attention_append(
+        ctypes.byref(desc), 0, vp(16), vp(16), 1, vp(16), 1, vp(16), vp(16), vp(16), vp(16), vp(16), kn, vn, sn,
+        vp(16), vp(16), vp(16), vp(256), 1 << 20, None)
+    d = wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4).c()
+    assert call(d, sn=None) == 1 and b"slot_new" in lib.wc_last_error()
+    assert call(d, kn=vp(8)) == 1 and b"aligned" in lib.wc_last_error()
+    for other in (wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4, scheme=wc.SCHEME_FP8_E4M3),
+                  wc.CacheDesc(num_q_heads=8, num_kv_heads=2, num_pages=4, dither_bits=10)):
+        o = other.c()
+        assert call(o) == 2 and b"append" in lib.wc_last_error()
