@@ -215,6 +215,9 @@ class Setup:
         e.synchronize()
         self.write_g_call_s = s.elapsed_time(e) / 1e3 / reps
         del k, v
+        # the step's new tokens as one stacked tensor per side (one copy in the end-to-end step)
+        self.k_new_all, self.v_new_all = torch.stack(self.k_new), torch.stack(self.v_new)
+        self.k_new, self.v_new = list(self.k_new_all), list(self.v_new_all)
         self.q = torch.stack([W.layer_queries(wl, layer, device="cuda") for layer in range(wl.n_layers)])
         self.ws = wc.Workspace(self.desc, wl.batch, wl.max_pages)
         L, B, Hq = wl.n_layers, wl.batch, wl.n_q_heads
@@ -535,11 +538,9 @@ def run_e2e(st, args, world):
     """Same step with inputs copied from pinned host memory and results read back."""
     wl = st.wl
     host_q = st.q.cpu().pin_memory()
-    host_k = torch.stack(st.k_new).cpu().pin_memory()
-    host_v = torch.stack(st.v_new).cpu().pin_memory()
+    host_k = st.k_new_all.cpu().pin_memory()
+    host_v = st.v_new_all.cpu().pin_memory()
     host_ctx = st.ctx.cpu().pin_memory()
-    dev_k = torch.stack(st.k_new)
-    dev_v = torch.stack(st.v_new)
     out_h = torch.empty_like(st.out, device="cpu").pin_memory()
     raw_h = torch.empty_like(st.raw, device="cpu").pin_memory()
     meter_h = torch.empty_like(st.meter, device="cpu").pin_memory()
@@ -548,12 +549,9 @@ def run_e2e(st, args, world):
 
     def e2e_step():
         st.q.copy_(host_q, non_blocking=True)
-        dev_k.copy_(host_k, non_blocking=True)
-        dev_v.copy_(host_v, non_blocking=True)
+        st.k_new_all.copy_(host_k, non_blocking=True)   # the per-layer tensors are views of these
+        st.v_new_all.copy_(host_v, non_blocking=True)
         st.ctx.copy_(host_ctx, non_blocking=True)
-        for layer in range(wl.n_layers):
-            st.k_new[layer].copy_(dev_k[layer], non_blocking=True)
-            st.v_new[layer].copy_(dev_v[layer], non_blocking=True)
         st.step()
         out_h.copy_(st.out, non_blocking=True)
         raw_h.copy_(st.raw, non_blocking=True)

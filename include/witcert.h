@@ -180,7 +180,8 @@ size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_p
  *   meter[b][hq]    = min(1, meter_raw)
  * The context is split across CTAs; partial softmax, output and A
  * accumulators are merged under log-sum-exp weights (A is a p~-weighted mean,
- * §6.2.2), by the last CTA of each (sequence, KV head).  A sequence with
+ * §6.2.2) by a second kernel, launched as a programmatic dependent of the
+ * first (two launches per call).  A sequence with
  * ctx_len 0 gets out = 0 and meter = meter_raw = 0.
  *
  *   q            [batch][Hq][128] fp16 post-RoPE queries, device

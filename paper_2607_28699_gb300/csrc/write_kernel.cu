@@ -114,36 +114,57 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
                                       kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab);
 }
 
-// Bypass-pair calibration: one CTA per KV head; thread t sums pair t % 64
-// over every fourth token, the four partial sums are added in a fixed order,
-// and a pair is selected iff fewer than m pairs rank above it (larger energy,
-// or equal energy and a lower index).
-__global__ void __launch_bounds__(256) select_pairs_kernel(const __half* __restrict__ k, int n_tok, int num_kv_heads,
-                                                           int rope_layout, int m, int32_t* __restrict__ pairs) {
-    __shared__ float part[4][kHeadDim / 2];
+// Bypass-pair calibration: one CTA of 32 warps per KV head.  Warp w sums
+// rows w, w + 32, ...: one 256-byte row per warp load, lane l squaring channels
+// 4l .. 4l + 3.  The 32 warps' sums are added in a fixed order, channels are
+// added into pairs, and a pair is selected iff fewer than m pairs rank above
+// it (larger energy, or equal energy and a lower index).
+constexpr int kSelPairThreads = 1024;
+
+__global__ void __launch_bounds__(kSelPairThreads) select_pairs_kernel(const __half* __restrict__ k, int n_tok,
+                                                                       int num_kv_heads, int rope_layout, int m,
+                                                                       int32_t* __restrict__ pairs) {
+    __shared__ float part[kSelPairThreads / 32][kHeadDim];
     __shared__ float energy[kHeadDim / 2];
     __shared__ int chosen[kHeadDim / 2];
-    const int h = blockIdx.x, j = threadIdx.x & 63, stripe = threadIdx.x >> 6;
-    const int a = rope_layout == WC_ROPE_HALF ? j : 2 * j;
-    const int b = rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
-    float acc = 0.0f;
-    for (int t = stripe; t < n_tok; t += 4) {
-        const __half* row = k + ((size_t)t * num_kv_heads + h) * kHeadDim;
-        const float xa = __half2float(row[a]), xb = __half2float(row[b]);
-        acc = fmaf(xa, xa, fmaf(xb, xb, acc));
+    const int h = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 4
+    for (int t = warp; t < n_tok; t += kSelPairThreads / 32) {
+        const uint2 w = __ldg(reinterpret_cast<const uint2*>(k + ((size_t)t * num_kv_heads + h) * kHeadDim) + lane);
+        const float2 f01 = __half22float2(*reinterpret_cast<const __half2*>(&w.x));
+        const float2 f23 = __half22float2(*reinterpret_cast<const __half2*>(&w.y));
+        a0 = fmaf(f01.x, f01.x, a0);
+        a1 = fmaf(f01.y, f01.y, a1);
+        a2 = fmaf(f23.x, f23.x, a2);
+        a3 = fmaf(f23.y, f23.y, a3);
     }
-    part[stripe][j] = acc;
+    part[warp][4 * lane] = a0;
+    part[warp][4 * lane + 1] = a1;
+    part[warp][4 * lane + 2] = a2;
+    part[warp][4 * lane + 3] = a3;
     __syncthreads();
-    if (threadIdx.x < 64) energy[j] = ((part[0][j] + part[1][j]) + part[2][j]) + part[3][j];
+    if (tid < kHeadDim) {   // channel sums in a fixed order (each thread its own column)
+        float e = 0.f;
+        for (int w = 0; w < kSelPairThreads / 32; ++w) e += part[w][tid];
+        part[0][tid] = e;
+    }
     __syncthreads();
-    if (threadIdx.x < 64) {
+    const int j = tid;
+    if (j < kHeadDim / 2) {
+        const int a = rope_layout == WC_ROPE_HALF ? j : 2 * j;
+        const int b = rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+        energy[j] = part[0][a] + part[0][b];
+    }
+    __syncthreads();
+    if (j < kHeadDim / 2) {
         const float e = energy[j];
         int rank = 0;
-        for (int i = 0; i < 64; ++i) rank += (energy[i] > e || (energy[i] == e && i < j)) ? 1 : 0;
+        for (int i = 0; i < kHeadDim / 2; ++i) rank += (energy[i] > e || (energy[i] == e && i < j)) ? 1 : 0;
         chosen[j] = rank < m;
     }
     __syncthreads();
-    if (threadIdx.x < 64 && chosen[j]) {
+    if (j < kHeadDim / 2 && chosen[j]) {
         int pos = 0;
         for (int i = 0; i < j; ++i) pos += chosen[i];
         if (pos < m) pairs[(size_t)h * m + pos] = j;   // NaN energies can make more than m ranks fall below m
@@ -154,7 +175,7 @@ __global__ void __launch_bounds__(256) select_pairs_kernel(const __half* __restr
 
 cudaError_t launch_select_pairs(const __half* k, int n_tok, int num_kv_heads, int rope_layout, int m, int32_t* pairs,
                                 cudaStream_t stream) {
-    select_pairs_kernel<<<num_kv_heads, 256, 0, stream>>>(k, n_tok, num_kv_heads, rope_layout, m, pairs);
+    select_pairs_kernel<<<num_kv_heads, kSelPairThreads, 0, stream>>>(k, n_tok, num_kv_heads, rope_layout, m, pairs);
     return cudaGetLastError();
 }
 
