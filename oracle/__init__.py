@@ -15,14 +15,19 @@ philox     Philox4x32-10 (Salmon et al., SC'11) and the dither derived from it
            (§6.2.1 "Research kernels": Philox dither from a slot-keyed counter;
            §6.2.3 storage side: counter uses the slot, not the position).
 quantizer  subtractive-dither INT8 quantizer (§4.2 "Subtractive dither"),
-           raw-cast fp8, residual band-norm witness (§4.1 Eq. witness).
+           raw-cast fp8, residual band-norm witness (§4.1 Eq. witness),
+           value witness (§3 output bound), grouped scales with the
+           fixed-channel outlier-pair bypass and its calibration (§6.2.3).
 meter      exact / compressed attention, total variation (§3 setup), the
            flawed dispersion certificate (§3 Eq. flawed, regression guard),
            Tier-A logit bound (§4.1 Thm. "Sound black-box logit bound"),
-           the e-form meter (§3 Thm. "Sound replacement"), gate (§6 meter
-           loop box).
-pipeline   the write path over a paged cache and the metered decode step,
-           composed from the functions above.
+           Tier-B sub-Gaussian bound, per-token and grouped (§4.2), the
+           e-form meter (§3 Thm. "Sound replacement"), the value term,
+           output bound and joint gate (§3, §4.2), block-level repair
+           selection (§6.4), gate (§6 meter loop box).
+pipeline   the write path over a paged cache (per-token, fp8 and grouped
+           schemes) and the metered decode step, composed from the
+           functions above.
 
 Every function is pinned by ``tests/test_oracle_*.py`` against something
 other than itself (paper-printed values, library routines, exact rational
