@@ -19,7 +19,11 @@
 // one group).  The lane's Philox call covers storage positions 16 sub .. +15;
 // dither bytes and codes move between storage and channel order through a
 // 128-byte shared row per unit, so quantization runs in channel order.
+#include <cooperative_groups.h>
+
 #include "write_row.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace wc {
 
@@ -114,23 +118,28 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
                                       kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab);
 }
 
-// Bypass-pair calibration: one CTA of 32 warps per KV head.  Warp w sums
-// rows w, w + 32, ...: one 256-byte row per warp load, lane l squaring channels
-// 4l .. 4l + 3.  The 32 warps' sums are added in a fixed order, channels are
-// added into pairs, and a pair is selected iff fewer than m pairs rank above
-// it (larger energy, or equal energy and a lower index).
+// Bypass-pair calibration: a cluster of 8 CTAs of 32 warps per KV head.  Warp
+// w of cluster rank r sums rows 32 r + w + 256 i: one 256-byte row per warp load,
+// lane l squaring channels 4l .. 4l + 3.  Each CTA adds its warps' sums in a
+// fixed order; rank 0 adds the 8 CTAs' sums (distributed shared memory, rank
+// order), adds channels into pairs, and selects a pair iff fewer than m pairs
+// rank above it (larger energy, or equal energy and a lower index).
 constexpr int kSelPairThreads = 1024;
+constexpr int kSelPairCluster = 8;
 
-__global__ void __launch_bounds__(kSelPairThreads) select_pairs_kernel(const __half* __restrict__ k, int n_tok,
-                                                                       int num_kv_heads, int rope_layout, int m,
-                                                                       int32_t* __restrict__ pairs) {
+__global__ void __cluster_dims__(kSelPairCluster, 1, 1) __launch_bounds__(kSelPairThreads)
+    select_pairs_kernel(const __half* __restrict__ k, int n_tok, int num_kv_heads, int rope_layout, int m,
+                        int32_t* __restrict__ pairs) {
     __shared__ float part[kSelPairThreads / 32][kHeadDim];
     __shared__ float energy[kHeadDim / 2];
     __shared__ int chosen[kHeadDim / 2];
-    const int h = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int h = blockIdx.y, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int kWarpsPerHead = kSelPairCluster * kSelPairThreads / 32;
     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll 4
-    for (int t = warp; t < n_tok; t += kSelPairThreads / 32) {
+    for (int t = rank * (kSelPairThreads / 32) + warp; t < n_tok; t += kWarpsPerHead) {
         const uint2 w = __ldg(reinterpret_cast<const uint2*>(k + ((size_t)t * num_kv_heads + h) * kHeadDim) + lane);
         const float2 f01 = __half22float2(*reinterpret_cast<const __half2*>(&w.x));
         const float2 f23 = __half22float2(*reinterpret_cast<const __half2*>(&w.y));
@@ -144,38 +153,48 @@ __global__ void __launch_bounds__(kSelPairThreads) select_pairs_kernel(const __h
     part[warp][4 * lane + 2] = a2;
     part[warp][4 * lane + 3] = a3;
     __syncthreads();
-    if (tid < kHeadDim) {   // channel sums in a fixed order (each thread its own column)
+    if (tid < kHeadDim) {   // this CTA's channel sums in a fixed order (each thread its own column)
         float e = 0.f;
         for (int w = 0; w < kSelPairThreads / 32; ++w) e += part[w][tid];
         part[0][tid] = e;
     }
-    __syncthreads();
-    const int j = tid;
-    if (j < kHeadDim / 2) {
-        const int a = rope_layout == WC_ROPE_HALF ? j : 2 * j;
-        const int b = rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
-        energy[j] = part[0][a] + part[0][b];
+    cluster.sync();   // every CTA's sums are in its row 0
+    if (rank == 0) {
+        if (tid < kHeadDim) {
+            float e = 0.f;
+            for (int r = 0; r < kSelPairCluster; ++r) e += cluster.map_shared_rank(&part[0][0], r)[tid];
+            part[1][tid] = e;
+        }
+        __syncthreads();
+        const int j = tid;
+        if (j < kHeadDim / 2) {
+            const int a = rope_layout == WC_ROPE_HALF ? j : 2 * j;
+            const int b = rope_layout == WC_ROPE_HALF ? j + kHeadDim / 2 : 2 * j + 1;
+            energy[j] = part[1][a] + part[1][b];
+        }
+        __syncthreads();
+        if (j < kHeadDim / 2) {
+            const float e = energy[j];
+            int rnk = 0;
+            for (int i = 0; i < kHeadDim / 2; ++i) rnk += (energy[i] > e || (energy[i] == e && i < j)) ? 1 : 0;
+            chosen[j] = rnk < m;
+        }
+        __syncthreads();
+        if (j < kHeadDim / 2 && chosen[j]) {
+            int pos = 0;
+            for (int i = 0; i < j; ++i) pos += chosen[i];
+            if (pos < m) pairs[(size_t)h * m + pos] = j;   // NaN energies can make more than m ranks fall below m
+        }
     }
-    __syncthreads();
-    if (j < kHeadDim / 2) {
-        const float e = energy[j];
-        int rank = 0;
-        for (int i = 0; i < kHeadDim / 2; ++i) rank += (energy[i] > e || (energy[i] == e && i < j)) ? 1 : 0;
-        chosen[j] = rank < m;
-    }
-    __syncthreads();
-    if (j < kHeadDim / 2 && chosen[j]) {
-        int pos = 0;
-        for (int i = 0; i < j; ++i) pos += chosen[i];
-        if (pos < m) pairs[(size_t)h * m + pos] = j;   // NaN energies can make more than m ranks fall below m
-    }
+    cluster.sync();   // the other CTAs' shared memory stays alive until rank 0 has read it
 }
 
 }  // namespace
 
 cudaError_t launch_select_pairs(const __half* k, int n_tok, int num_kv_heads, int rope_layout, int m, int32_t* pairs,
                                 cudaStream_t stream) {
-    select_pairs_kernel<<<num_kv_heads, kSelPairThreads, 0, stream>>>(k, n_tok, num_kv_heads, rope_layout, m, pairs);
+    select_pairs_kernel<<<dim3(kSelPairCluster, num_kv_heads), kSelPairThreads, 0, stream>>>(k, n_tok, num_kv_heads,
+                                                                                            rope_layout, m, pairs);
     return cudaGetLastError();
 }
 
