@@ -32,7 +32,12 @@ namespace {
 // Tasks of 4 tokens per warp whose loads are all issued before any is used:
 // more bytes in flight per SM (the kernel is otherwise bound by load latency).
 constexpr int kWriteTasks = 2;
-constexpr int kWriteUnitsPerCta = 2 * 4 * kWriteTasks;   // two warps per row type
+// The grouped scheme's row routine is much larger: one task per warp keeps the
+// kernel's code small enough for the instruction cache.
+__host__ __device__ constexpr int write_tasks(int scheme) {
+    return scheme == WC_SCHEME_DITHER_INT8_G32 ? 1 : kWriteTasks;
+}
+__host__ __device__ constexpr int write_units_per_cta(int scheme) { return 2 * 4 * write_tasks(scheme); }
 constexpr int kPerHeadMinTokens = 16;                     // per-head grid from this many tokens on
 
 // Two ways of cutting the units (token, KV head) into 4-unit tasks:
@@ -82,13 +87,14 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
     // own unit i of a 4-unit task.
     const int row = warp & 1;                                                  // 0 = K, 1 = V
     const int sub = lane & 7;                                                  // 16-channel chunk
-    const int first = (blockIdx.x * 2 + (warp >> 1)) * (4 * kWriteTasks) + (lane >> 3);
+    constexpr int kTasks = write_tasks(kScheme);
+    const int first = (blockIdx.x * 2 + (warp >> 1)) * (4 * kTasks) + (lane >> 3);
     const int n_first = kPerHead ? p.n_tok : p.n_tok * p.num_kv_heads;
-    bool live[kWriteTasks];
-    int slot[kWriteTasks], hs[kWriteTasks];
-    uint4 raw[kWriteTasks][2];
+    bool live[kTasks];
+    int slot[kTasks], hs[kTasks];
+    uint4 raw[kTasks][2];
 #pragma unroll
-    for (int t = 0; t < kWriteTasks; ++t) {
+    for (int t = 0; t < kTasks; ++t) {
         const int idx = first + 4 * t;   // a token (kPerHead) or a unit
         live[t] = idx < n_first;
         int tok = 0, h = 0;
@@ -112,7 +118,7 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
         }
     }
 #pragma unroll
-    for (int t = 0; t < kWriteTasks; ++t)
+    for (int t = 0; t < kTasks; ++t)
         if (__any_sync(0xffffffffu, live[t]))   // warp-uniform: a task past the end is skipped whole
             write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub,
                                       kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab);
@@ -218,8 +224,9 @@ cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_
         configured = true;
     }
     const bool per_head = p.n_tok >= kPerHeadMinTokens;
-    const dim3 grid = per_head ? dim3((p.n_tok + kWriteUnitsPerCta - 1) / kWriteUnitsPerCta, p.num_kv_heads)
-                               : dim3((p.n_tok * p.num_kv_heads + kWriteUnitsPerCta - 1) / kWriteUnitsPerCta);
+    const int upc = write_units_per_cta(scheme);
+    const dim3 grid = per_head ? dim3((p.n_tok + upc - 1) / upc, p.num_kv_heads)
+                               : dim3((p.n_tok * p.num_kv_heads + upc - 1) / upc);
     auto go = [&](auto kernel) { return launch_pdl(kernel, grid, dim3(128), 0, stream, p); };
     if (scheme == WC_SCHEME_FP8_E4M3)
         return per_head ? go(write_kernel<WC_SCHEME_FP8_E4M3, 8, true>) : go(write_kernel<WC_SCHEME_FP8_E4M3, 8, false>);
