@@ -299,7 +299,9 @@ wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t
  * logical position ctx_lens[b] - 1 (block_table[b][(ctx - 1) / 16] * 16 +
  * (ctx - 1) % 16); otherwise it is not written and WC_DEV_BAD_APPEND is set.
  * slot_new[b] < 0: no new token for sequence b.  The token is quantized by
- * the CTA that reads the sequence's last page, before it reads it.
+ * the CTA that reads the sequence's last page, before it reads it; that page
+ * must belong to sequence b alone (no other sequence of the call may map it,
+ * as with prefix sharing), since only that CTA is ordered after the write.
  *   k_new, v_new  [batch][Hkv][128] fp16 post-RoPE, device, 16-byte aligned
  *   slot_new      [batch] int32, device
  * The cache arrays are written, hence not const.  WC_ERR_UNSUPPORTED for any
