@@ -1,16 +1,21 @@
 // Metered decode attention over the grouped-scale cache (§6.2.3 "Storage
 // side" and "Fixed-channel outlier bypass"): one fp16 scale per token and
 // 32-channel group, and the m key RoPE pairs of a (layer, KV head) stored
-// exactly.  The structure is the per-token kernel's (8 warps, a copy ring per
-// warp, the same split-K partials and merge; code tiles by tensor-map TMA with
-// the 128-byte swizzle as in the warp-specialized kernel); what differs:
+// exactly.  Warp-specialized like the per-token kernel: 6 producer / 6 consumer
+// warp pairs per CTA, one CTA per SM (at 384 threads the consumer keeps its ~165
+// registers without spilling; 8 pairs with a producer -> consumer register
+// split measured slower).  A producer stages a page (code tiles by TMA with the
+// 128-byte swizzle; scales, witness and bypass values by bulk copy) and
+// regenerates its dither into swizzled byte tiles; its consumer runs the math
+// below with no Philox on its path.  The split-K partials and the merge are the
+// per-token kernel's.  What differs from the per-token math:
 //
 //  - A row is stored in the order the mma fragments consume it (storage
 //    position p of K holds channel 16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3),
 //    of V channel 16 ((p >> 1) & 7) + 8 (p & 1) + (p >> 4)), with the dither
-//    drawn by storage position.  So the code and dither loads and the two
-//    Philox calls per token are the per-token kernel's, while every QK
-//    k-step and every PV m-tile meets a single channel group.
+//    drawn by storage position.  So the code and dither tiles are the
+//    per-token kernel's, while every QK k-step and every PV m-tile meets a
+//    single channel group.
 //  - QK: the q operand is gathered in that order, with the bypassed channels
 //    zeroed; after the two k-steps of a group the accumulators are folded,
 //    raw += s_g (code.q - h'.q + kappa sum_g q), and the exact bypassed
@@ -25,56 +30,133 @@ namespace wc {
 
 namespace {
 
-constexpr int kGWarps = 8;
-constexpr int kGThreads = 32 * kGWarps;
-constexpr int kGStages = 2;
-constexpr int kGMinBlocks = 1;   // one CTA per SM: the kernel needs ~205 registers (two CTAs spilled: 1.3x slower)
-// stage: K codes | V codes | K scales [16][4] | V scales [16][4] | witness [16][8] | bypass [16][2m]
-constexpr int kGOffV = 2048, kGOffKs = 4096, kGOffVs = 4224, kGOffW = 4352, kGOffB = 4608;
 constexpr int kGMaxBypass = 16;
-constexpr int kGStageStride = 6144;   // 1024-aligned: the code tiles land with the 128-byte swizzle
-static_assert(kGOffB + 16 * 2 * kGMaxBypass * 2 <= kGStageStride, "stage layout");
-constexpr int kGSmemBytes = kGWarps * kGStages * kGStageStride + kGWarps * kGStages * 8 + 1024;   // + alignment
 
 struct G32Params {
     CUtensorMap k_map;   // k_codes as [num_pages * Hkv][16][128] bytes, box = one page of one head
     CUtensorMap v_map;
     DecodeParams p;
 };
-static_assert(kGWarps * kMaxGroup * kPartialStride * 4 <= kGWarps * kGStages * kGStageStride, "merge buffer");
-static_assert(kGSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
+
+constexpr int kGwPairs = kG32PageStreams;
+constexpr int kGwThreads = 64 * kGwPairs;
+constexpr int kGwStages = 2;
+// stage: K codes | V codes | K dither | V dither (16 x 128 bytes each, swizzled) |
+// K scales [16][4] | V scales [16][4] | witness [16][8] | bypass [16][2m] | header
+constexpr int kGwOffK = 0, kGwOffV = 2048, kGwOffKd = 4096, kGwOffVd = 6144;
+constexpr int kGwOffKs = 8192, kGwOffVs = 8320, kGwOffW = 8448, kGwOffB = 8704, kGwOffHdr = 9728;
+constexpr int kGwStageBytes = 10240;
+static_assert(kGwOffB + 16 * 2 * kGMaxBypass * 2 <= kGwOffHdr && kGwOffHdr + 16 <= kGwStageBytes, "stage layout");
+constexpr int kGwSmemBytes = kGwPairs * kGwStages * kGwStageBytes + kGwPairs * kGwStages * 2 * 8 + 1024;
+static_assert(kGwPairs * kMaxGroup * kPartialStride * 4 <= kGwPairs * kGwStages * kGwStageBytes, "merge buffer");
+static_assert(kGwSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
+
+__device__ __forceinline__ void gw_consumer_sync() {   // the consumer warps only
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kGwPairs) : "memory");
+}
 
 template <int kX>
-__global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(const __grid_constant__ G32Params gparams) {
+__global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __grid_constant__ G32Params gparams) {
     constexpr bool kTierB = (kX & kXTierB) != 0;
     constexpr float kKappa = DitherConst<8>::kappa;
     const DecodeParams& p = gparams.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const bool producer = warp >= kGwPairs;
+    const int pw = producer ? warp - kGwPairs : warp;
     const int g = lane >> 2, c = lane & 3;
     const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int G = p.group;
-    const int m = p.num_bypass, nb = 2 * m;   // bypassed pairs, dims
+    const int m = p.num_bypass, nb = 2 * m;
 
-    uint8_t* my_stages = smem + warp * kGStages * kGStageStride;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kGWarps * kGStages * kGStageStride) + warp * kGStages;
-    if (lane == 0)
-        for (int s = 0; s < kGStages; ++s) mbar_init(&bars[s], 1);
+    uint8_t* stages = smem + pw * kGwStages * kGwStageBytes;
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem + kGwPairs * kGwStages * kGwStageBytes) + pw * 2 * kGwStages;
+    uint64_t* empty = full + kGwStages;
+    if (producer && lane == 0)
+        for (int s = 0; s < kGwStages; ++s) {
+            mbar_init(&full[s], 2);
+            mbar_init(&empty[s], 1);
+        }
     fence_barrier_init();
-    grid_dep_launch();   // the dependent merge waits for this whole grid
-    grid_dep_wait();     // q, page tables and the cache may come from the preceding kernel
+    __syncthreads();   // every barrier is initialised before any warp waits on it
+    grid_dep_launch();
+    grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
     const int p0 = split * p.pages_per_split;
     const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
-    const int lim = min(p0 + p.pages_per_split, p.max_pages);
-    int ring[kGStages];   // physical pages of this warp's next kGStages pages
-#pragma unroll
-    for (int k = 0; k < kGStages; ++k) {
-        const int lp = p0 + warp + kGWarps * k;
-        ring[k] = lp < lim ? __ldg(bt_row + lp) : -1;
-    }
+    int phys_next = (producer && p.max_pages > 0) ? __ldg(bt_row + min(p0 + pw, p.max_pages - 1)) : -1;
     int ctx = __ldg(p.ctx_lens + b);
+    if (ctx < 0 || ctx > p.max_pages * kPage) {
+        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+        ctx = max(0, min(ctx, p.max_pages * kPage));
+    }
+    const int npages = (ctx + kPage - 1) / kPage;
+    const int p1 = min(p0 + p.pages_per_split, npages);
+    const int n_my = (p1 - p0 - pw > 0) ? (p1 - p0 - pw + kGwPairs - 1) / kGwPairs : 0;
+
+    if (producer) {
+        const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
+        const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+        int issued = 0;
+        for (int k = 0; k < n_my; ++k) {
+            const int s = k % kGwStages;
+            if (k >= kGwStages) {
+                const bool freed = mbar_wait_bounded(&empty[s], (uint32_t)(((k / kGwStages) - 1) & 1));
+                if (!__all_sync(0xffffffffu, freed)) {
+                    if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+                    break;
+                }
+            }
+            const int phys = phys_next;
+            if (k + 1 < n_my) phys_next = __ldg(bt_row + p0 + pw + kGwPairs * (k + 1));
+            const bool ok = phys >= 0 && phys < p.num_pages;
+            uint8_t* st = stages + s * kGwStageBytes;
+            if (lane == 0) {
+                *reinterpret_cast<int*>(st + kGwOffHdr) = ok ? phys : -1;
+                if (ok) {
+                    const int z = phys * p.num_kv_heads + h;
+                    const size_t ph = (size_t)z;
+                    mbar_arrive_expect_tx(&full[s], (uint32_t)(4096 + 128 + 128 + 256 + 64 * m));
+                    tma_page(st + kGwOffK, &gparams.k_map, z, &full[s]);
+                    tma_page(st + kGwOffV, &gparams.v_map, z, &full[s]);
+                    bulk_g2s(st + kGwOffKs, p.k_scale + ph * (kPage * 4), 128, &full[s]);
+                    bulk_g2s(st + kGwOffVs, p.v_scale + ph * (kPage * 4), 128, &full[s]);
+                    bulk_g2s(st + kGwOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
+                    if (m > 0) bulk_g2s(st + kGwOffB, p.k_bypass + ph * (kPage * nb), (uint32_t)(64 * m), &full[s]);
+                } else {
+                    atomicOr(p.status, WC_DEV_BAD_PAGE);
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+                }
+            }
+            issued = k + 1;
+            if (ok) {   // dither bytes j[token][storage position], swizzled like the code tiles
+                const uint32_t slot0 = (uint32_t)phys * kPage;
+                uint4 dk[4], dv[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x position chunks 2c, 2c+1
+                    dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
+#pragma unroll
+                for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x position chunk g
+                    dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+                    *reinterpret_cast<uint4*>(st + kGwOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
+#pragma unroll
+                for (int j = 0; j < 4; ++j)
+                    *reinterpret_cast<uint4*>(st + kGwOffVd + swz(tv[j], g)) = dv[j];
+            }
+            __syncwarp();
+            if (lane == 0)   // second arrival: dither tiles and header are written
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+        }
+        // copies still in flight must land before the CTA's smem is released
+        for (int k = max(0, issued - kGwStages); k < issued; ++k)
+            (void)mbar_wait_bounded(&full[k % kGwStages], (uint32_t)((k / kGwStages) & 1));
+        return;
+    }
+
+    // ---- consumer: dither read from the stage ------------------------------------------
     const bool row_valid = g < G;
     const __half* qrow = p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim;
     uint32_t qn[16];   // head g, channels 32c + 2i, +1 in word i (channel order: group c)
@@ -90,38 +172,6 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
         qw[2 * ks] = v.x;
         qw[2 * ks + 1] = v.y;
     }
-
-    if (ctx < 0 || ctx > p.max_pages * kPage) {
-        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
-        ctx = max(0, min(ctx, p.max_pages * kPage));
-    }
-    const int npages = (ctx + kPage - 1) / kPage;
-    const int p1 = min(p0 + p.pages_per_split, npages);
-    const int n_my = (p1 - p0 - warp > 0) ? (p1 - p0 - warp + kGWarps - 1) / kGWarps : 0;
-    const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
-
-    // ---- per-warp stage ring --------------------------------------------------
-    auto issue = [&](int k, int phys) {
-        if (k >= n_my || lane != 0) return;
-        uint64_t* bar = &bars[k % kGStages];
-        if (phys < 0 || phys >= p.num_pages) {
-            atomicOr(p.status, WC_DEV_BAD_PAGE);
-            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
-            return;
-        }
-        uint8_t* st = my_stages + (k % kGStages) * kGStageStride;
-        const size_t ph = (size_t)phys * p.num_kv_heads + h;
-        mbar_arrive_expect_tx(bar, (uint32_t)(kGOffB + 64 * m));
-        tma_page(st, &gparams.k_map, (int)ph, bar);
-        tma_page(st + kGOffV, &gparams.v_map, (int)ph, bar);
-        bulk_g2s(st + kGOffKs, p.k_scale + ph * (kPage * 4), 128, bar);
-        bulk_g2s(st + kGOffVs, p.v_scale + ph * (kPage * 4), 128, bar);
-        bulk_g2s(st + kGOffW, p.k_witness + ph * (kPage * kBands), 256, bar);
-        if (m > 0) bulk_g2s(st + kGOffB, p.k_bypass + ph * (kPage * nb), (uint32_t)(64 * m), bar);
-    };
-    __syncwarp();
-#pragma unroll
-    for (int k = 0; k < kGStages; ++k) issue(k, ring[k]);
 
     // ---- the bypassed key channels --------------------------------------------
     // nmask: bypassed channels of group c (bit d - 32c); pmask: bypassed slots of
@@ -219,34 +269,27 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
 #pragma unroll
     for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
     int lam_exp = INT_MIN;   // P s_g 2^lam_exp stays below 2^14 (fp16)
-    bool failed = false;
-    int consumed = 0;
     const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
 
     for (int k = 0; k < n_my; ++k) {
-        const int lp = p0 + warp + kGWarps * k;
-        const int phys = ring[0];
-        const int phys_issue = (k + kGStages < n_my) ? __ldg(bt_row + lp + kGWarps * kGStages) : -1;
-        const bool page_ok = phys >= 0 && phys < p.num_pages;
-        const bool landed = mbar_wait_bounded(&bars[k % kGStages], (uint32_t)((k / kGStages) & 1));
+        const int s = k % kGwStages;
+        const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kGwStages) & 1));
         if (!__all_sync(0xffffffffu, landed)) {   // warp-uniform decision
             if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
-            failed = true;
             break;
         }
-        consumed = k + 1;
-        if (page_ok) {
-            const uint8_t* st = my_stages + (k % kGStages) * kGStageStride;
-            const uint32_t slot0 = (uint32_t)phys * kPage;
+        const uint8_t* st = stages + s * kGwStageBytes;
+        const int lp = p0 + pw + kGwPairs * k;
+        if (*reinterpret_cast<const int*>(st + kGwOffHdr) >= 0) {
             const int nvalid = min(kPage, ctx - lp * kPage);
             const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
             // group scales of tokens g, g + 8
             float sk[2][4], sv[2][4];
             {
-                const uint2 ka = *reinterpret_cast<const uint2*>(st + kGOffKs + 8 * g);
-                const uint2 kb = *reinterpret_cast<const uint2*>(st + kGOffKs + 8 * (g + 8));
-                const uint2 va = *reinterpret_cast<const uint2*>(st + kGOffVs + 8 * g);
-                const uint2 vb = *reinterpret_cast<const uint2*>(st + kGOffVs + 8 * (g + 8));
+                const uint2 ka = *reinterpret_cast<const uint2*>(st + kGwOffKs + 8 * g);
+                const uint2 kb = *reinterpret_cast<const uint2*>(st + kGwOffKs + 8 * (g + 8));
+                const uint2 va = *reinterpret_cast<const uint2*>(st + kGwOffVs + 8 * g);
+                const uint2 vb = *reinterpret_cast<const uint2*>(st + kGwOffVs + 8 * (g + 8));
                 const uint32_t w[4][2] = {{ka.x, ka.y}, {kb.x, kb.y}, {va.x, va.y}, {vb.x, vb.y}};
 #pragma unroll
                 for (int r = 0; r < 2; ++r)
@@ -269,10 +312,10 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             float raw[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {   // storage positions 32c + 16gp .. +15: k-steps 4gp .. 4gp+3
-                const uint4 ka = *reinterpret_cast<const uint4*>(st + swz(g, 2 * c + gp));
-                const uint4 kb = *reinterpret_cast<const uint4*>(st + swz(g + 8, 2 * c + gp));
-                const uint4 da = philox(slot0 + g, c1, (uint32_t)(2 * c + gp), 0u, p.keys);
-                const uint4 db = philox(slot0 + g + 8, c1, (uint32_t)(2 * c + gp), 0u, p.keys);
+                const uint4 ka = *reinterpret_cast<const uint4*>(st + kGwOffK + swz(g, 2 * c + gp));
+                const uint4 kb = *reinterpret_cast<const uint4*>(st + kGwOffK + swz(g + 8, 2 * c + gp));
+                const uint4 da = *reinterpret_cast<const uint4*>(st + kGwOffKd + swz(g, 2 * c + gp));
+                const uint4 db = *reinterpret_cast<const uint4*>(st + kGwOffKd + swz(g + 8, 2 * c + gp));
                 float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
@@ -300,9 +343,9 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
                 if (t < nbt) {
                     const int e0 = 8 * t + 2 * c;   // entries e0, e0 + 1 = pair 4t + c
                     const bool use = e0 < nb && ((pvalid >> (4 * t + c)) & 1u);
-                    const uint32_t a0 = use ? *reinterpret_cast<const uint32_t*>(st + kGOffB + (g * nb + e0) * 2) : 0u;
+                    const uint32_t a0 = use ? *reinterpret_cast<const uint32_t*>(st + kGwOffB + (g * nb + e0) * 2) : 0u;
                     const uint32_t a1 =
-                        use ? *reinterpret_cast<const uint32_t*>(st + kGOffB + ((g + 8) * nb + e0) * 2) : 0u;
+                        use ? *reinterpret_cast<const uint32_t*>(st + kGwOffB + ((g + 8) * nb + e0) * 2) : 0u;
                     mma1688(raw, a0, a1, qb[t]);
                 }
             }
@@ -310,8 +353,8 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             // ---------------- logits, bound, softmax ------------------------------
             float cb[4] = {0.f, 0.f, 0.f, 0.f};
             {
-                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kGOffW + (g * kBands + 2 * c) * 2);
-                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kGOffW + ((g + 8) * kBands + 2 * c) * 2);
+                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kGwOffW + (g * kBands + 2 * c) * 2);
+                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kGwOffW + ((g + 8) * kBands + 2 * c) * 2);
                 mma1688(cb, wa, wb, a_hi);
                 mma1688(cb, wa, wb, a_lo);
             }
@@ -390,8 +433,8 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             uint4 vq[4], dv[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                vq[j] = *reinterpret_cast<const uint4*>(st + kGOffV + swz(tv[j], g));
-                dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
+                vq[j] = *reinterpret_cast<const uint4*>(st + kGwOffV + swz(tv[j], g));
+                dv[j] = *reinterpret_cast<const uint4*>(st + kGwOffVd + swz(tv[j], g));
             }
 #pragma unroll
             for (int gi = 0; gi < 4; ++gi) {
@@ -433,15 +476,8 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             }
         }
         __syncwarp();
-        issue(k + kGStages, phys_issue);
-#pragma unroll
-        for (int i = 0; i + 1 < kGStages; ++i) ring[i] = ring[i + 1];
-        ring[kGStages - 1] = phys_issue;
-    }
-    if (failed) {
-        // let copies still in flight land before the CTA's smem is released
-        for (int k = consumed; k < min(n_my, consumed + kGStages); ++k)
-            (void)mbar_wait_bounded(&bars[k % kGStages], (uint32_t)((k / kGStages) & 1));
+        if (lane == 0)   // release the stage to the producer
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&empty[s])) : "memory");
     }
 
     // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
@@ -457,11 +493,11 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
         }
     const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
 
-    // ---- CTA merge: warps -> shared, one partial per CTA -----------------------------
-    __syncthreads();   // stage buffers are reused below
+    // ---- CTA merge over the consumer warps: one partial per CTA ------------------------
+    gw_consumer_sync();   // all consumers are done with their stages (reused below)
     float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
     {
-        float* wb = mbuf + warp * kMaxGroup * kPartialStride;
+        float* wb = mbuf + pw * kMaxGroup * kPartialStride;
 #pragma unroll
         for (int e = 0; e < 2; ++e) {
             float* row = wb + (2 * c + e) * kPartialStride;
@@ -479,23 +515,23 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
             }
         }
     }
-    __syncthreads();
+    gw_consumer_sync();
     const size_t unit = (size_t)b * p.num_kv_heads + h;
     float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
     // thread -> (head, 4-dim chunk); chunk 32 carries (M, l, D, D_B)
-    for (int idx = threadIdx.x; idx < G * 33; idx += kGThreads) {
+    for (int idx = threadIdx.x; idx < G * 33; idx += 32 * kGwPairs) {
         const int hh = idx / 33, ch = idx % 33;
-        float mw[kGWarps];
+        float mw[kGwPairs];
         float M = -INFINITY;
 #pragma unroll
-        for (int w = 0; w < kGWarps; ++w) {
+        for (int w = 0; w < kGwPairs; ++w) {
             mw[w] = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
             M = fmaxf(M, mw[w]);
         }
         float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
         const int col = (ch < 32) ? 4 * ch : kHeadDim + 1;
 #pragma unroll
-        for (int w = 0; w < kGWarps; ++w) {
+        for (int w = 0; w < kGwPairs; ++w) {
             if (mw[w] == -INFINITY) continue;   // a warp without pages: its values are not read
             const float wt = fast_exp2(mw[w] - M);
             const float* src = mbuf + (w * kMaxGroup + hh) * kPartialStride + col;
@@ -522,13 +558,12 @@ __global__ void __launch_bounds__(kGThreads, kGMinBlocks) decode_g32_kernel(cons
 }
 
 template <int kX>
-cudaError_t launch_g32(const DecodeParams& p, cudaStream_t stream) {
+cudaError_t launch_g32_ws(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;   // per process; the attributes are per function
     if (!configured) {
-        cudaError_t e =
-            cudaFuncSetAttribute(decode_g32_kernel<kX>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmemBytes);
+        cudaError_t e = cudaFuncSetAttribute(decode_g32_ws_kernel<kX>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGwSmemBytes);
         if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(decode_g32_kernel<kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
+        e = cudaFuncSetAttribute(decode_g32_ws_kernel<kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
         if (e != cudaSuccess) return e;
         configured = true;
@@ -539,7 +574,7 @@ cudaError_t launch_g32(const DecodeParams& p, cudaStream_t stream) {
         !encode_page_map(&gp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
     const dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_g32_kernel<kX>, grid, dim3(kGThreads), kGSmemBytes, stream, gp);
+    cudaError_t e = launch_pdl(decode_g32_ws_kernel<kX>, grid, dim3(kGwThreads), kGwSmemBytes, stream, gp);
     if (e != cudaSuccess) return e;
     return launch_merge_x(p, kX, stream);
 }
@@ -547,7 +582,7 @@ cudaError_t launch_g32(const DecodeParams& p, cudaStream_t stream) {
 }  // namespace
 
 cudaError_t launch_decode_g32(const DecodeParams& p, cudaStream_t stream) {
-    return p.meter_b ? launch_g32<kXTierB>(p, stream) : launch_g32<0>(p, stream);
+    return p.meter_b ? launch_g32_ws<kXTierB>(p, stream) : launch_g32_ws<0>(p, stream);
 }
 
 }  // namespace wc

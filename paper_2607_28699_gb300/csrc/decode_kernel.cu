@@ -1273,18 +1273,21 @@ static int ctas_per_sm(int scheme, int bits) {
     return (use_ws(scheme, bits) || scheme == WC_SCHEME_DITHER_INT8_G32) ? 1 : kMinBlocks;
 }
 
-// Split plan.  A CTA's 8 page streams (warps or warp pairs) each take every
-// 8th page of its split, so a split of P pages costs ceil(P / 8) page steps,
-// and a wave of resident CTAs adds a fixed prologue / epilogue of about one
-// and a half page steps.  The split count minimises
-//     waves * (ceil(pages_per_split / 8) + 1.5),   waves = ceil(CTAs / resident CTAs),
+// Page streams per CTA: warps, or warp pairs.
+static long streams_per_cta(int scheme) { return scheme == WC_SCHEME_DITHER_INT8_G32 ? kG32PageStreams : 8; }
+
+// Split plan.  A CTA's n page streams each take every n-th page of its split,
+// so a split of P pages costs ceil(P / n) page steps, and a wave of resident
+// CTAs adds a fixed prologue / epilogue of about one and a half page steps.
+// The split count minimises
+//     waves * (ceil(pages_per_split / n) + 1.5),   waves = ceil(CTAs / resident CTAs),
 // so a grid never spills a small remainder into an extra wave; splits keep at
-// least 8 pages (one per stream).  Ties go to fewer splits (less to merge).
+// least n pages (one per stream).  Ties go to fewer splits (less to merge).
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits) {
     DecodePlan pl;
     const long units = (long)batch * num_kv_heads;
     const long slots = std::max<long>(1, (long)num_sms * ctas_per_sm(scheme, bits));
-    constexpr long kStreams = 8;      // page streams per CTA
+    const long kStreams = streams_per_cta(scheme);
     constexpr long kWaveCost2 = 3;    // per-wave fixed cost, in half page steps
     const long max_splits = std::max<long>(1, std::min<long>(max_pages / kStreams, 4 * slots));
     long best_pps = std::max(max_pages, 1), best_cost = -1;

@@ -117,6 +117,9 @@ struct RepairParams {
 // Largest block-table width the selection handles (its sort holds one cell's
 // pages in shared memory).
 constexpr int kRepairMaxPages = 16384;
+// Page streams (producer / consumer warp pairs) per CTA of the grouped-scheme
+// decode; the split planner sizes splits by it.
+constexpr int kG32PageStreams = 6;
 
 cudaError_t launch_write(const WriteParams& p, int scheme, int bits, cudaStream_t stream);
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream);
