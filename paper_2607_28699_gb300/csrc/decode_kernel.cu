@@ -609,6 +609,10 @@ constexpr int kWsStageBytes = 9216;
 static_assert(kWsOffVw + 64 <= kWsStageBytes && kWsStageBytes % 1024 == 0, "stage layout");
 constexpr int kWsBarBytes = kWsPairs * kWsStages * 2 * 8;
 constexpr int kWsSmemBytes = kWsPairs * kWsStages * kWsStageBytes + kWsBarBytes + 1024;   // + alignment slack
+// flattened plan: the CTA merge's own buffer after the barriers
+constexpr int kWsMergeOff = kWsPairs * kWsStages * kWsStageBytes + kWsBarBytes;
+constexpr int kWsSmemFlat = kWsSmemBytes + kWsPairs * kMaxGroup * kPartialStride * 4;
+static_assert(kWsMergeOff % 16 == 0 && kWsSmemFlat <= 232448, "flattened plan's shared memory");
 static_assert(kWsSmemBytes <= 232448, "exceeds the per-CTA shared memory limit");
 static_assert(kWsPairs * kMaxGroup * kPartialStride * 4 <= kWsPairs * kWsStages * kWsStageBytes, "merge buffer");
 
@@ -653,6 +657,143 @@ __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
 }
 
+// A CTA's work as segments: pages [a, e) of unit (b, h); page stream (warp
+// pair) w takes pages a + ((w - ph) & 7) + 8 i.  Split plan: one segment, the
+// CTA's split (possibly empty).  Flattened plan: CTA c serves KV head
+// h = c mod Hkv and takes share j = c / Hkv of the batch's pages laid end to
+// end (sequence after sequence), cut at sequence boundaries; the Hkv CTAs of a
+// share read the same pages together (the heads of a page are adjacent in the
+// cache).  ph keeps the streams' round robin running across the cuts, so
+// every stream gets ceil or floor of (hi - lo) / 8 pages.
+struct WsSeg {
+    int b, h, a, e, ph, ctx, np;
+    long long pos;      // flattened position of page a
+    long long lo, hi;   // the CTA's share
+};
+
+__device__ __forceinline__ int clamped_ctx(const DecodeParams& p, int b) {
+    return max(0, min(__ldg(p.ctx_lens + b), p.max_pages * kPage));
+}
+
+// First segment; called by every thread of the CTA (the flattened plan scans
+// the batch's page counts with two block barriers).  False: no pages.
+template <bool kFlat>
+__device__ __forceinline__ bool ws_first_segment(const DecodeParams& p, WsSeg& sg, int* s_wtot, long long* s_start) {
+    if constexpr (!kFlat) {
+        sg.b = blockIdx.z;
+        sg.h = blockIdx.y;
+        int ctx = __ldg(p.ctx_lens + sg.b);
+        if (ctx < 0 || ctx > p.max_pages * kPage) {
+            if (threadIdx.x == 0 && blockIdx.x == 0 && sg.h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+            ctx = max(0, min(ctx, p.max_pages * kPage));
+        }
+        sg.ctx = ctx;
+        sg.np = (ctx + kPage - 1) / kPage;
+        sg.a = blockIdx.x * p.pages_per_split;
+        sg.e = min(sg.a + p.pages_per_split, sg.np);
+        sg.ph = 0;
+        sg.pos = sg.lo = sg.hi = 0;
+        return true;
+    } else {
+        const int nt = blockDim.x, t = threadIdx.x, per = (p.batch + nt - 1) / nt;
+        int loc = 0;
+        bool bad = false;
+        for (int i = 0; i < per; ++i) {
+            const int bb = t * per + i;
+            if (bb < p.batch) {
+                const int cx = __ldg(p.ctx_lens + bb);
+                bad |= cx < 0 || cx > p.max_pages * kPage;
+                loc += (max(0, min(cx, p.max_pages * kPage)) + kPage - 1) / kPage;
+            }
+        }
+        if (bad && blockIdx.x == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+        int inc = loc;   // inclusive scan over the warp
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, inc, o);
+            if ((t & 31) >= o) inc += v;
+        }
+        if ((t & 31) == 31) s_wtot[t >> 5] = inc;
+        __syncthreads();
+        int before = 0, total = 0;
+        for (int w = 0; w < nt / 32; ++w) {
+            const int v = s_wtot[w];
+            total += v;
+            if (w < (t >> 5)) before += v;
+        }
+        const int excl = before + inc - loc;   // pages of the sequences before this thread's
+        const int hk = p.num_kv_heads, shares = max(1, p.splits / hk);
+        const long long R = max(1LL, ((long long)total + shares - 1) / shares);
+        const long long lo = (long long)(blockIdx.x / hk) * R, hi = min((long long)total, lo + R);
+        if (lo < hi && excl <= lo && lo < (long long)excl + loc) {
+            long long acc = excl;   // exactly one thread: the one whose sequences hold lo
+            for (int i = 0; i < per; ++i) {
+                const int bb = t * per + i;
+                if (bb >= p.batch) break;
+                const int np = (clamped_ctx(p, bb) + kPage - 1) / kPage;
+                if (lo < acc + np) {
+                    *s_start = ((long long)bb << 32) | (long long)(lo - acc);
+                    break;
+                }
+                acc += np;
+            }
+        }
+        __syncthreads();
+        if (lo >= hi) return false;
+        const long long st = *s_start;
+        sg.b = (int)(st >> 32);
+        sg.a = (int)(st & 0xffffffffLL);
+        sg.h = blockIdx.x % hk;
+        sg.ctx = clamped_ctx(p, sg.b);
+        sg.np = (sg.ctx + kPage - 1) / kPage;
+        sg.e = (int)min((long long)sg.np, sg.a + (hi - lo));
+        sg.ph = 0;
+        sg.pos = sg.lo = lo;
+        sg.hi = hi;
+        return true;
+    }
+}
+
+// Next segment of the flattened plan (the next sequence with pages); false
+// at the end of the CTA's share, and always in the split plan.
+template <bool kFlat>
+__device__ __forceinline__ bool ws_next_segment(const DecodeParams& p, WsSeg& sg) {
+    if constexpr (!kFlat) return false;
+    sg.pos += sg.e - sg.a;
+    if (sg.pos >= sg.hi) return false;
+    do {   // sequences without pages hold no part of the share
+        if (sg.b + 1 >= p.batch) return false;
+        ++sg.b;
+        sg.ctx = clamped_ctx(p, sg.b);
+        sg.np = (sg.ctx + kPage - 1) / kPage;
+    } while (sg.np == 0);
+    sg.a = 0;
+    sg.e = (int)min((long long)sg.np, sg.hi - sg.pos);
+    sg.ph = (int)((sg.pos - sg.lo) & (kWsPairs - 1));
+    return true;
+}
+
+static_assert((kWsPairs & (kWsPairs - 1)) == 0, "the page streams' round robin uses a mask");
+
+// Flattened plan: each warp's walker lives in a shared slot, so that only the
+// current segment's indices take registers in the page loop; lane 0 advances it.
+template <bool kFlat>
+__device__ __forceinline__ bool ws_step(const DecodeParams& p, WsSeg* slot, int lane) {
+    if constexpr (!kFlat) {
+        return false;
+    } else {
+        __syncwarp();
+        int more = 0;
+        if (lane == 0) more = ws_next_segment<true>(p, *slot);
+        __syncwarp();
+        return __shfl_sync(0xffffffffu, more, 0) != 0;
+    }
+}
+__device__ __forceinline__ int ws_seg_pages(const WsSeg& sg, int w, int& first) {
+    first = sg.a + ((w - sg.ph) & (kWsPairs - 1));
+    return first < sg.e ? (sg.e - first + kWsPairs - 1) / kWsPairs : 0;
+}
+
 // q fragment of the B operand (head g, channels 32c + 2i, +1 in word i).
 __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h, int G, int g, int c,
                                             uint32_t (&qw)[16]) {
@@ -670,6 +811,7 @@ template <int kX>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
     constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
     constexpr bool kAppend = (kX & kXAppend) != 0;
+    constexpr bool kFlat = (kX & kXFlat) != 0;   // flattened split plan (pages_per_split == 0)
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -677,7 +819,6 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     const bool producer = warp >= kWsPairs;
     const int pw = producer ? warp - kWsPairs : warp;     // pair index
     const int g = lane >> 2, c = lane & 3;
-    const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int G = p.group;
     constexpr float kKappa = DitherConst<8>::kappa;
 
@@ -695,14 +836,14 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     // (griddepcontrol.wait), and it launches only once every CTA of this grid
     // has started, so its CTAs never hold resources this grid still needs
     grid_dep_launch();
-    const int p0 = split * p.pages_per_split;
-    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
-    if (lane == 0 && p.max_pages > 0) {
-        // While the preceding kernel drains: warm L2 with this pair's first page
-        // and the CTA's query rows.  The context length and page-table entry read
-        // here may still be changing, so they serve only as prefetch addresses
-        // (clamped into the cache); the loads bypass L1, which therefore holds
-        // no copy that the reads after the wait could hit.
+    if (!kFlat && lane == 0 && p.max_pages > 0) {
+        // Split plan.  While the preceding kernel drains: warm L2 with this pair's
+        // first page and the CTA's query rows.  The context length and page-table
+        // entry read here may still be changing, so they serve only as prefetch
+        // addresses (clamped into the cache); the loads bypass L1, which therefore
+        // holds no copy that the reads after the wait could hit.
+        const int b = blockIdx.z, h = blockIdx.y, p0 = blockIdx.x * p.pages_per_split;
+        const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
         if (producer) {
             const int ctx_hint = __ldcg(p.ctx_lens + b);
             if (p0 + pw < p.max_pages && (p0 + pw) * kPage < ctx_hint) {
@@ -720,421 +861,457 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     }
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
-    // this pair's first page-table entry, loaded alongside the context length
-    // (in bounds whatever the length; used only if the pair has pages)
-    int phys_next = (producer && p.max_pages > 0) ? __ldg(bt_row + min(p0 + pw, p.max_pages - 1)) : -1;
-    int ctx = __ldg(p.ctx_lens + b);
-    if (ctx < 0 || ctx > p.max_pages * kPage) {
-        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
-        ctx = max(0, min(ctx, p.max_pages * kPage));
+    __shared__ int s_wtot[kWsThreads / 32];
+    __shared__ long long s_start;
+    __shared__ WsSeg s_seg[kWsThreads / 32];
+    // Split plan: this pair's first page-table entry and the consumer's query
+    // fragment are loaded alongside the context length (both in bounds
+    // whatever the length; used only if the pair has pages).
+    int phys_first = -1;
+    uint32_t qw[16];
+    if constexpr (!kFlat) {
+        if (producer && p.max_pages > 0)
+            phys_first = __ldg(p.block_table + (size_t)blockIdx.z * p.max_pages +
+                               min((int)blockIdx.x * p.pages_per_split + pw, p.max_pages - 1));
+        if (!producer) load_q_frag(p, blockIdx.z, blockIdx.y, G, g, c, qw);
     }
-    const int npages = (ctx + kPage - 1) / kPage;
-    const int p1 = min(p0 + p.pages_per_split, npages);
-    const int n_my = (p1 - p0 - pw > 0) ? (p1 - p0 - pw + kWsPairs - 1) / kWsPairs : 0;
+    WsSeg sg;
+    const bool have = ws_first_segment<kFlat>(p, sg, s_wtot, &s_start);
+    WsSeg* const my_seg = &s_seg[warp];
+    if constexpr (kFlat) {
+        if (lane == 0) *my_seg = sg;
+        __syncwarp();
+    }
 
     if (producer) {
-        const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
         const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
-        int issued = 0;
-        for (int k = 0; k < n_my; ++k) {
-            const int s = k % kWsStages;
-            if (k >= kWsStages) {
-                const bool freed = mbar_wait_bounded(&empty[s], (uint32_t)(((k / kWsStages) - 1) & 1));
-                if (!__all_sync(0xffffffffu, freed)) {
-                    if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
-                    break;
+        int k = 0, issued = 0;   // stage ring position, continued across segments
+        bool stop = false;
+        for (bool more = have; more && !stop; more = ws_step<kFlat>(p, my_seg, lane)) {
+            const WsSeg& cs = kFlat ? *my_seg : sg;
+            const int b = cs.b, h = cs.h, ctx = cs.ctx, npages = cs.np;
+            const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
+            const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
+            int first;
+            const int n_seg = ws_seg_pages(cs, pw, first);
+            int phys_next = kFlat ? (n_seg > 0 ? __ldg(bt_row + first) : -1) : phys_first;
+            for (int i = 0; i < n_seg; ++i, ++k) {
+                const int lp = first + kWsPairs * i;
+                const int s = k % kWsStages;
+                if (k >= kWsStages) {
+                    const bool freed = mbar_wait_bounded(&empty[s], (uint32_t)(((k / kWsStages) - 1) & 1));
+                    if (!__all_sync(0xffffffffu, freed)) {
+                        if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+                        stop = true;
+                        break;
+                    }
                 }
-            }
-            const int phys = phys_next;
-            if (k + 1 < n_my) phys_next = __ldg(bt_row + p0 + pw + kWsPairs * (k + 1));
-            const bool ok = phys >= 0 && phys < p.num_pages;
-            uint8_t* st = stages + s * kWsStageBytes;
-            if constexpr (kAppend) {   // the sequence's last page: store the new token first
-                if (ok && p0 + pw + kWsPairs * k == npages - 1) append_new_token(wp, b, h, phys, ctx, lane);
-            }
-            if (lane == 0) {
-                *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
+                const int phys = phys_next;
+                if (i + 1 < n_seg) phys_next = __ldg(bt_row + lp + kWsPairs);
+                const bool ok = phys >= 0 && phys < p.num_pages;
+                uint8_t* st = stages + s * kWsStageBytes;
+                if constexpr (kAppend) {   // the sequence's last page: store the new token first
+                    if (ok && lp == npages - 1) append_new_token(wp, b, h, phys, ctx, lane);
+                }
+                if (lane == 0) {
+                    *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
+                    if (ok) {
+                        const int z = phys * p.num_kv_heads + h;
+                        const size_t ph = (size_t)z;
+                        mbar_arrive_expect_tx(&full[s], (uint32_t)(kStageBytes + (kValue ? 64 : 0)));
+                        tma_page(st + kWsOffK, &wp.k_map, z, &full[s]);
+                        tma_page(st + kWsOffV, &wp.v_map, z, &full[s]);
+                        bulk_g2s(st + kWsOffKs, p.k_scale + ph * kPage, 32, &full[s]);
+                        bulk_g2s(st + kWsOffVs, p.v_scale + ph * kPage, 32, &full[s]);
+                        bulk_g2s(st + kWsOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
+                        if constexpr (kValue) bulk_g2s(st + kWsOffVw, p.v_witness + ph * (kPage * 2), 64, &full[s]);
+                    } else {
+                        atomicOr(p.status, WC_DEV_BAD_PAGE);
+                        asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+                    }
+                }
+                issued = k + 1;
                 if (ok) {
-                    const int z = phys * p.num_kv_heads + h;
-                    const size_t ph = (size_t)z;
-                    mbar_arrive_expect_tx(&full[s], (uint32_t)(kStageBytes + (kValue ? 64 : 0)));
-                    tma_page(st + kWsOffK, &wp.k_map, z, &full[s]);
-                    tma_page(st + kWsOffV, &wp.v_map, z, &full[s]);
-                    bulk_g2s(st + kWsOffKs, p.k_scale + ph * kPage, 32, &full[s]);
-                    bulk_g2s(st + kWsOffVs, p.v_scale + ph * kPage, 32, &full[s]);
-                    bulk_g2s(st + kWsOffW, p.k_witness + ph * (kPage * kBands), 256, &full[s]);
-                    if constexpr (kValue) bulk_g2s(st + kWsOffVw, p.v_witness + ph * (kPage * 2), 64, &full[s]);
-                } else {
-                    atomicOr(p.status, WC_DEV_BAD_PAGE);
-                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
+                    // dither bytes j[token][channel]: one Philox call covers 16
+                    // channels of one token (channel i = byte i%4 of word i/4)
+                    const uint32_t slot0 = (uint32_t)phys * kPage;
+                    uint4 dk[4], dv[4];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x channel groups 2c, 2c+1
+                        dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
+                        dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        *reinterpret_cast<uint4*>(st + kWsOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j)
+                        *reinterpret_cast<uint4*>(st + kWsOffVd + swz(tv[j], g)) = dv[j];
                 }
+                __syncwarp();
+                if (lane == 0)   // second arrival: dither tiles and header are written
+                    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
             }
-            issued = k + 1;
-            if (ok) {
-                // dither bytes j[token][channel]: one Philox call covers 16
-                // channels of one token (channel i = byte i%4 of word i/4)
-                const uint32_t slot0 = (uint32_t)phys * kPage;
-                uint4 dk[4], dv[4];
-#pragma unroll
-                for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x channel groups 2c, 2c+1
-                    dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
-#pragma unroll
-                for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
-                    dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
-#pragma unroll
-                for (int i = 0; i < 4; ++i)
-                    *reinterpret_cast<uint4*>(st + kWsOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
-#pragma unroll
-                for (int j = 0; j < 4; ++j)
-                    *reinterpret_cast<uint4*>(st + kWsOffVd + swz(tv[j], g)) = dv[j];
-            }
-            __syncwarp();
-            if (lane == 0)   // second arrival: dither tiles and header are written
-                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
         }
         // copies still in flight must land before the CTA's smem is released
-        for (int k = max(0, issued - kWsStages); k < issued; ++k)
-            (void)mbar_wait_bounded(&full[k % kWsStages], (uint32_t)((k / kWsStages) & 1));
+        for (int j = max(0, issued - kWsStages); j < issued; ++j)
+            (void)mbar_wait_bounded(&full[j % kWsStages], (uint32_t)((j / kWsStages) & 1));
         return;
     }
 
     // ---------------------------- consumer warps ------------------------------------
-    const bool row_valid = g < G;
-    uint32_t qw[16];
-    load_q_frag(p, b, h, G, g, c, qw);
-    float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[i]));
-        qsum += f.x + f.y;
-        part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));
-    }
-    qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
-    qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
-    // Tier B (§4.2): u_t = alpha s_t with alpha = sqrt(2 log(2S/delta) ||q||^2 / (12 d)),
-    // for this thread's softmax heads 2c and 2c+1
-    float alpha0 = 0.f, alpha1 = 0.f;
-    if constexpr (kTierB) {
-        float qn2 = part[0] + part[1] + part[2] + part[3];   // ||q_g||^2 over channels 32c .. 32c+31
-        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
-        qn2 += __shfl_xor_sync(0xffffffffu, qn2, 2);
-        const float lg = p.tb_log_2_over_delta + logf((float)max(ctx, 1));   // log(2S / delta)
-        const float al = sqrtf(2.0f * lg * qn2 * (1.0f / (12.0f * kHeadDim)));
-        alpha0 = __shfl_sync(0xffffffffu, al, 8 * c);
-        alpha1 = __shfl_sync(0xffffffffu, al, 8 * c + 4);
-    }
-    float band_a, band_b;
-    if (p.rope_layout == WC_ROPE_HALF) {
-#pragma unroll
-        for (int i = 0; i < 4; ++i) part[i] += __shfl_xor_sync(0xffffffffu, part[i], 2);
-        const int src = (lane & ~3) | (c >> 1);
-        float v[4];
-#pragma unroll
-        for (int i = 0; i < 4; ++i) v[i] = __shfl_sync(0xffffffffu, part[i], src);
-        band_a = (c & 1) ? v[2] : v[0];
-        band_b = (c & 1) ? v[3] : v[1];
-    } else {
-        band_a = part[0] + part[1];
-        band_b = part[2] + part[3];
-    }
-    uint32_t a_hi = 0, a_lo = 0;
-    if (row_valid) {
-        const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
-        const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
-        a_hi = pack_h2(__half2float(h0), __half2float(h1));
-        a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
-    }
-    const float zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
-    const float zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
-
-    float m_run[2] = {-INFINITY, -INFINITY};
-    float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
-    float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
-    float vt_part[2] = {0.f, 0.f};   // value side: sum p~ rho^v (kValue)
-    float vmax = 0.f;                // value side: max ||v|| over this thread's tokens
-    float acc[8][4];
-#pragma unroll
-    for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-    int lam_exp = INT_MIN;
+    // The CTA merge's buffer [warp][head][kPartialStride]: the stage area in the
+    // split plan (one segment, the producers are done with it), a buffer of its
+    // own in the flattened plan (the producers stage the next segment meanwhile).
+    float* mbuf = reinterpret_cast<float*>(kFlat ? smem + kWsMergeOff : smem);
     const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
-
-    for (int k = 0; k < n_my; ++k) {
-        const int s = k % kWsStages;
-        const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kWsStages) & 1));
-        if (!__all_sync(0xffffffffu, landed)) {
-            if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
-            break;
+    int k = 0;   // stage ring position, continued across segments
+    bool failed = false;
+    for (bool more = have; more; more = ws_step<kFlat>(p, my_seg, lane)) {
+        const WsSeg& cs = kFlat ? *my_seg : sg;
+        const int b = cs.b, h = cs.h, ctx = cs.ctx;
+        const bool row_valid = g < G;
+        if constexpr (kFlat) load_q_frag(p, b, h, G, g, c, qw);
+        float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qw[i]));
+            qsum += f.x + f.y;
+            part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));
         }
-        const uint8_t* st = stages + s * kWsStageBytes;
-        const int lp = p0 + pw + kWsPairs * k;
-        if (*reinterpret_cast<const int*>(st + kWsOffHdr) >= 0) {
-            const int nvalid = min(kPage, ctx - lp * kPage);
-
-            // ---------------- QK: S[token][head] = code.q - h'.q -------------------
-            float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-            for (int gp = 0; gp < 2; ++gp) {
-                const int q16 = 2 * c + gp;   // 16-byte chunk: channels 32c + 16gp .. +15
-                const uint4 ka = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g, q16));
-                const uint4 kb = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g + 8, q16));
-                const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g, q16));
-                const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g + 8, q16));
-#pragma unroll
-                for (int kk = 0; kk < 4; ++kk) {
-                    const int ks = 4 * gp + kk;
-                    const uint32_t xa = word_of(ka, kk) ^ 0x80808080u, xb = word_of(kb, kk) ^ 0x80808080u;
-                    const uint32_t A[4] = {s8x2_to_h2(xa, kSel01), s8x2_to_h2(xb, kSel01), s8x2_to_h2(xa, kSel23),
-                                           s8x2_to_h2(xb, kSel23)};
-                    mma16816(dc, A, qw[2 * ks], qw[2 * ks + 1]);
-                    const uint32_t ya = word_of(ja, kk), yb = word_of(jb, kk);
-                    const uint32_t H[4] = {h8(ya, kSel01), h8(yb, kSel01), h8(ya, kSel23), h8(yb, kSel23)};
-                    mma16816(dd, H, qw[2 * ks], qw[2 * ks + 1]);
-                }
-            }
-
-            // ---------------- logits, bound, softmax ------------------------------
-            float cb[4] = {0.f, 0.f, 0.f, 0.f};
-            {
-                const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (g * kBands + 2 * c) * 2);
-                const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kWsOffW + ((g + 8) * kBands + 2 * c) * 2);
-                mma1688(cb, wa, wb, a_hi);
-                mma1688(cb, wa, wb, a_lo);
-            }
-            const __half* ksc = reinterpret_cast<const __half*>(st + kWsOffKs);
-            const __half* vsc = reinterpret_cast<const __half*>(st + kWsOffVs);
-            float sk[2] = {__half2float(ksc[g]), __half2float(ksc[g + 8])};
-            float sv[2] = {__half2float(vsc[g]), __half2float(vsc[g + 8])};
-            float y[4], P[4];
-            const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = i >> 1, e = i & 1;
-                const bool okr = r ? ok1 : ok0;
-                const float raw = dc[i] - dd[i] + (e ? zoff1 : zoff0);
-                y[i] = okr ? raw * (sk[r] * kRsdLog2e) : -INFINITY;
-                if (!okr) cb[i] = 0.f;                 // tail slots may hold any bits
-            }
-            if (!ok0) sv[0] = 0.f;
-            if (!ok1) sv[1] = 0.f;
-            if constexpr (kTierB) {
-                if (!ok0) sk[0] = 0.f;
-                if (!ok1) sk[1] = 0.f;
-            }
-            float rho[2] = {0.f, 0.f};   // value witness of tokens g, g+8 (0 past the context)
-            if constexpr (kValue) {
-                const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * g));
-                const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * (g + 8)));
-                if (ok0) { rho[0] = w0.x; vmax = fmaxf(vmax, w0.y); }
-                if (ok1) { rho[1] = w1.x; vmax = fmaxf(vmax, w1.y); }
-            }
-            float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
-#pragma unroll
-            for (int o = 4; o < 32; o <<= 1) {
-                mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-                mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-            }
-            const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
-            if (__any_sync(0xffffffffu, mv0 || mv1)) {
-                const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
-                const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
-                if (mv0) m_run[0] = mx0;
-                if (mv1) m_run[1] = mx1;
-                l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
-                l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
-                if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
-                if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    acc[mt][0] *= a0; acc[mt][2] *= a0;
-                    acc[mt][1] *= a1; acc[mt][3] *= a1;
-                }
-            }
-            float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = i >> 1, e = i & 1;
-                const float pe = fast_exp2(y[i] - m_run[e]);
-                l_part[e] += pe;
-                const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
-                d_part[e] = fmaf(pe, em1, d_part[e]);
-                if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
-                if constexpr (kTierB)
-                    db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
-                if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
-                P[i] = pe * sv[r];
-                spv_part[e] += P[i];
-            }
-            if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
-            {
-                const float smax = fmaxf(sv[0], sv[1]);
-                const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
-                if (wmax > 0.f) {
-                    const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
-                    const int want = 6 - e;
-                    if (lam_exp == INT_MIN) {
-                        lam_exp = want;
-                    } else if (want < lam_exp) {
-                        const float f = pow2(want - lam_exp);
-#pragma unroll
-                        for (int mt = 0; mt < 8; ++mt)
-#pragma unroll
-                            for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
-                        lam_exp = want;
-                    }
-                }
-            }
-            uint32_t bp0, bp1, bl0, bl1;
-            {
-                const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
-                const float x0 = P[0] * lam, x1 = P[1] * lam, x2 = P[2] * lam, x3 = P[3] * lam;
-                const uint32_t h01 = pack_h2(x0, x1), h23 = pack_h2(x2, x3);
-                const float2 r01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
-                const float2 r23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
-                const uint32_t l01 = pack_h2(x0 - r01.x, x1 - r01.y), l23 = pack_h2(x2 - r23.x, x3 - r23.y);
-                bp0 = movmatrix_t(h01);
-                bp1 = movmatrix_t(h23);
-                bl0 = movmatrix_t(l01);
-                bl1 = movmatrix_t(l23);
-            }
-
-            // ---------------- PV: acc[dim][head] ------------------------------------
-            {
-                uint4 vq[4];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) vq[j] = *reinterpret_cast<const uint4*>(st + kWsOffV + swz(tv[j], g));
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    const int wi = mt >> 1, pos = 2 * (mt & 1);
-                    uint32_t A[4];
-#pragma unroll
-                    for (int pr = 0; pr < 2; ++pr) {
-                        const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
-                                                word_of(vq[2 * pr + 1], wi) ^ 0x80808080u, sel_interleave(pos));
-                        A[2 * pr] = s8x2_to_h2(X, kSel01);
-                        A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
-                    }
-                    mma16816(acc[mt], A, bp0, bp1);
-                    mma16816(acc[mt], A, bl0, bl1);
-                }
-            }
-            {
-                const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
-                const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
-                uint4 dv[4];
-#pragma unroll
-                for (int j = 0; j < 4; ++j) dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + swz(tv[j], g));
-#pragma unroll
-                for (int mt = 0; mt < 8; ++mt) {
-                    const int wi = mt >> 1, pos = 2 * (mt & 1);
-                    uint32_t H[4];
-#pragma unroll
-                    for (int pr = 0; pr < 2; ++pr) {
-                        const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
-                                                sel_interleave(pos));
-                        H[2 * pr] = h8(Y, kSel01);
-                        H[2 * pr + 1] = h8(Y, kSel23);
-                    }
-                    mma16816(acc[mt], H, bn0, bn1);
-                    mma16816(acc[mt], H, bm0, bm1);
-                }
-            }
-        } else if constexpr (kRepair) {
-            emit_skipped_page(p, b, h, G, lp, lane);
+        qsum += __shfl_xor_sync(0xffffffffu, qsum, 1);
+        qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
+        // Tier B (§4.2): u_t = alpha s_t with alpha = sqrt(2 log(2S/delta) ||q||^2 / (12 d)),
+        // for this thread's softmax heads 2c and 2c+1
+        float alpha0 = 0.f, alpha1 = 0.f;
+        if constexpr (kTierB) {
+            float qn2 = part[0] + part[1] + part[2] + part[3];   // ||q_g||^2 over channels 32c .. 32c+31
+            qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
+            qn2 += __shfl_xor_sync(0xffffffffu, qn2, 2);
+            const float lg = p.tb_log_2_over_delta + logf((float)max(ctx, 1));   // log(2S / delta)
+            const float al = sqrtf(2.0f * lg * qn2 * (1.0f / (12.0f * kHeadDim)));
+            alpha0 = __shfl_sync(0xffffffffu, al, 8 * c);
+            alpha1 = __shfl_sync(0xffffffffu, al, 8 * c + 4);
         }
-        __syncwarp();
-        if (lane == 0)   // release the stage to the producer
-            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&empty[s])) : "memory");
-    }
-
-    // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
+        float band_a, band_b;
+        if (p.rope_layout == WC_ROPE_HALF) {
 #pragma unroll
-    for (int o = 4; o < 32; o <<= 1)
+            for (int i = 0; i < 4; ++i) part[i] += __shfl_xor_sync(0xffffffffu, part[i], 2);
+            const int src = (lane & ~3) | (c >> 1);
+            float v[4];
 #pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
-            d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
-            if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
-            if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
-            spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
-        }
-    if constexpr (kValue)
-        for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
-    const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
-
-    // ---- CTA merge over the consumer warps: one partial per CTA ------------------------
-    consumer_sync();   // all consumers are done with their stages (reused below)
-    float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
-    {
-        float* wb = mbuf + pw * kMaxGroup * kPartialStride;
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            float* row = wb + (2 * c + e) * kPartialStride + 16 * g;
-            const float add = kKappa * spv_part[e];
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                float4 v;
-                v.x = fmaf(acc[2 * q4][e], inv_lam, add);
-                v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
-                v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
-                v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
-                *reinterpret_cast<float4*>(row + 4 * q4) = v;
-            }
-            if (g == 0) {
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
-                if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
-                if constexpr (kValue) {
-                    wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
-                    wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
-                }
-            }
-        }
-    }
-    consumer_sync();
-    const size_t unit = (size_t)b * p.num_kv_heads + h;
-    float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
-    for (int idx = threadIdx.x; idx < G * 33; idx += 32 * kWsPairs) {
-        const int hh = idx / 33, ch = idx % 33;
-        float mw[kWsPairs];
-        float M = -INFINITY;
-#pragma unroll
-        for (int w = 0; w < kWsPairs; ++w) {
-            mw[w] = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
-            M = fmaxf(M, mw[w]);
-        }
-        float4 s4 = make_float4(0.f, 0.f, 0.f, 0.f);
-        const int col = (ch < 32) ? 4 * ch : kHeadDim + 1;
-#pragma unroll
-        for (int w = 0; w < kWsPairs; ++w) {
-            if (mw[w] == -INFINITY) continue;   // a warp without pages: its values are not read
-            const float wt = fast_exp2(mw[w] - M);
-            const float* src = mbuf + (w * kMaxGroup + hh) * kPartialStride + col;
-            if (ch < 32) {
-                const float4 v = *reinterpret_cast<const float4*>(src);
-                s4.x = fmaf(wt, v.x, s4.x); s4.y = fmaf(wt, v.y, s4.y);
-                s4.z = fmaf(wt, v.z, s4.z); s4.w = fmaf(wt, v.w, s4.w);
-            } else {
-                s4.x = fmaf(wt, src[0], s4.x);
-                s4.y = fmaf(wt, src[1], s4.y);
-                if constexpr (kTierB) s4.z = fmaf(wt, src[2], s4.z);
-                if constexpr (kValue) s4.w = fmaf(wt, src[3], s4.w);
-            }
-        }
-        float* dst = part_out + hh * kPartialStride;
-        if (ch < 32) {
-            *reinterpret_cast<float4*>(dst + 4 * ch) = s4;
+            for (int i = 0; i < 4; ++i) v[i] = __shfl_sync(0xffffffffu, part[i], src);
+            band_a = (c & 1) ? v[2] : v[0];
+            band_b = (c & 1) ? v[3] : v[1];
         } else {
-            dst[kHeadDim] = M;
-            dst[kHeadDim + 1] = s4.x;
-            dst[kHeadDim + 2] = s4.y;
-            if constexpr (kTierB) dst[kHeadDim + 3] = s4.z;
-            if constexpr (kValue) {
-                float vm = 0.f;
-                for (int w = 0; w < kWsPairs; ++w)
-                    vm = fmaxf(vm, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim + 5]);
-                dst[kHeadDim + 4] = s4.w;
-                dst[kHeadDim + 5] = vm;
+            band_a = part[0] + part[1];
+            band_b = part[2] + part[3];
+        }
+        uint32_t a_hi = 0, a_lo = 0;
+        if (row_valid) {
+            const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
+            const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
+            a_hi = pack_h2(__half2float(h0), __half2float(h1));
+            a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
+        }
+        const float zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
+        const float zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
+
+        float m_run[2] = {-INFINITY, -INFINITY};
+        float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
+        float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
+        float vt_part[2] = {0.f, 0.f};   // value side: sum p~ rho^v (kValue)
+        float vmax = 0.f;                // value side: max ||v|| over this thread's tokens
+        float acc[8][4];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+        int lam_exp = INT_MIN;
+
+        int first;
+        const int n_seg = ws_seg_pages(cs, pw, first);
+        for (int i = 0; i < n_seg && !failed; ++i, ++k) {
+            const int s = k % kWsStages;
+            const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kWsStages) & 1));
+            if (!__all_sync(0xffffffffu, landed)) {
+                if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
+                failed = true;   // later pages are not waited for; the merges still run
+                break;
+            }
+            const uint8_t* st = stages + s * kWsStageBytes;
+            const int lp = first + kWsPairs * i;
+            if (*reinterpret_cast<const int*>(st + kWsOffHdr) >= 0) {
+                const int nvalid = min(kPage, ctx - lp * kPage);
+
+                // ---------------- QK: S[token][head] = code.q - h'.q -------------------
+                float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+                for (int gp = 0; gp < 2; ++gp) {
+                    const int q16 = 2 * c + gp;   // 16-byte chunk: channels 32c + 16gp .. +15
+                    const uint4 ka = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g, q16));
+                    const uint4 kb = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g + 8, q16));
+                    const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g, q16));
+                    const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g + 8, q16));
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const int ks = 4 * gp + kk;
+                        const uint32_t xa = word_of(ka, kk) ^ 0x80808080u, xb = word_of(kb, kk) ^ 0x80808080u;
+                        const uint32_t A[4] = {s8x2_to_h2(xa, kSel01), s8x2_to_h2(xb, kSel01), s8x2_to_h2(xa, kSel23),
+                                               s8x2_to_h2(xb, kSel23)};
+                        mma16816(dc, A, qw[2 * ks], qw[2 * ks + 1]);
+                        const uint32_t ya = word_of(ja, kk), yb = word_of(jb, kk);
+                        const uint32_t H[4] = {h8(ya, kSel01), h8(yb, kSel01), h8(ya, kSel23), h8(yb, kSel23)};
+                        mma16816(dd, H, qw[2 * ks], qw[2 * ks + 1]);
+                    }
+                }
+
+                // ---------------- logits, bound, softmax ------------------------------
+                float cb[4] = {0.f, 0.f, 0.f, 0.f};
+                {
+                    const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (g * kBands + 2 * c) * 2);
+                    const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kWsOffW + ((g + 8) * kBands + 2 * c) * 2);
+                    mma1688(cb, wa, wb, a_hi);
+                    mma1688(cb, wa, wb, a_lo);
+                }
+                const __half* ksc = reinterpret_cast<const __half*>(st + kWsOffKs);
+                const __half* vsc = reinterpret_cast<const __half*>(st + kWsOffVs);
+                float sk[2] = {__half2float(ksc[g]), __half2float(ksc[g + 8])};
+                float sv[2] = {__half2float(vsc[g]), __half2float(vsc[g + 8])};
+                float y[4], P[4];
+                const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = i >> 1, e = i & 1;
+                    const bool okr = r ? ok1 : ok0;
+                    const float raw = dc[i] - dd[i] + (e ? zoff1 : zoff0);
+                    y[i] = okr ? raw * (sk[r] * kRsdLog2e) : -INFINITY;
+                    if (!okr) cb[i] = 0.f;                 // tail slots may hold any bits
+                }
+                if (!ok0) sv[0] = 0.f;
+                if (!ok1) sv[1] = 0.f;
+                if constexpr (kTierB) {
+                    if (!ok0) sk[0] = 0.f;
+                    if (!ok1) sk[1] = 0.f;
+                }
+                float rho[2] = {0.f, 0.f};   // value witness of tokens g, g+8 (0 past the context)
+                if constexpr (kValue) {
+                    const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * g));
+                    const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * (g + 8)));
+                    if (ok0) { rho[0] = w0.x; vmax = fmaxf(vmax, w0.y); }
+                    if (ok1) { rho[1] = w1.x; vmax = fmaxf(vmax, w1.y); }
+                }
+                float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+#pragma unroll
+                for (int o = 4; o < 32; o <<= 1) {
+                    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+                    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+                }
+                const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
+                if (__any_sync(0xffffffffu, mv0 || mv1)) {
+                    const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
+                    const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
+                    if (mv0) m_run[0] = mx0;
+                    if (mv1) m_run[1] = mx1;
+                    l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                    l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                    if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
+                    if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
+#pragma unroll
+                    for (int mt = 0; mt < 8; ++mt) {
+                        acc[mt][0] *= a0; acc[mt][2] *= a0;
+                        acc[mt][1] *= a1; acc[mt][3] *= a1;
+                    }
+                }
+                float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int r = i >> 1, e = i & 1;
+                    const float pe = fast_exp2(y[i] - m_run[e]);
+                    l_part[e] += pe;
+                    const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
+                    d_part[e] = fmaf(pe, em1, d_part[e]);
+                    if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
+                    if constexpr (kTierB)
+                        db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
+                    if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
+                    P[i] = pe * sv[r];
+                    spv_part[e] += P[i];
+                }
+                if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
+                {
+                    const float smax = fmaxf(sv[0], sv[1]);
+                    const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
+                    if (wmax > 0.f) {
+                        const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
+                        const int want = 6 - e;
+                        if (lam_exp == INT_MIN) {
+                            lam_exp = want;
+                        } else if (want < lam_exp) {
+                            const float f = pow2(want - lam_exp);
+#pragma unroll
+                            for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+                                for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
+                            lam_exp = want;
+                        }
+                    }
+                }
+                uint32_t bp0, bp1, bl0, bl1;
+                {
+                    const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
+                    const float x0 = P[0] * lam, x1 = P[1] * lam, x2 = P[2] * lam, x3 = P[3] * lam;
+                    const uint32_t h01 = pack_h2(x0, x1), h23 = pack_h2(x2, x3);
+                    const float2 r01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
+                    const float2 r23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
+                    const uint32_t l01 = pack_h2(x0 - r01.x, x1 - r01.y), l23 = pack_h2(x2 - r23.x, x3 - r23.y);
+                    bp0 = movmatrix_t(h01);
+                    bp1 = movmatrix_t(h23);
+                    bl0 = movmatrix_t(l01);
+                    bl1 = movmatrix_t(l23);
+                }
+
+                // ---------------- PV: acc[dim][head] ------------------------------------
+                {
+                    uint4 vq[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) vq[j] = *reinterpret_cast<const uint4*>(st + kWsOffV + swz(tv[j], g));
+#pragma unroll
+                    for (int mt = 0; mt < 8; ++mt) {
+                        const int wi = mt >> 1, pos = 2 * (mt & 1);
+                        uint32_t A[4];
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
+                                                    word_of(vq[2 * pr + 1], wi) ^ 0x80808080u, sel_interleave(pos));
+                            A[2 * pr] = s8x2_to_h2(X, kSel01);
+                            A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
+                        }
+                        mma16816(acc[mt], A, bp0, bp1);
+                        mma16816(acc[mt], A, bl0, bl1);
+                    }
+                }
+                {
+                    const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
+                    const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
+                    uint4 dv[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + swz(tv[j], g));
+#pragma unroll
+                    for (int mt = 0; mt < 8; ++mt) {
+                        const int wi = mt >> 1, pos = 2 * (mt & 1);
+                        uint32_t H[4];
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
+                                                    sel_interleave(pos));
+                            H[2 * pr] = h8(Y, kSel01);
+                            H[2 * pr + 1] = h8(Y, kSel23);
+                        }
+                        mma16816(acc[mt], H, bn0, bn1);
+                        mma16816(acc[mt], H, bm0, bm1);
+                    }
+                }
+            } else if constexpr (kRepair) {
+                emit_skipped_page(p, b, h, G, lp, lane);
+            }
+            __syncwarp();
+            if (lane == 0)   // release the stage to the producer
+                asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&empty[s])) : "memory");
+        }
+
+        // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
+                d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+                if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
+                if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
+                spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
+            }
+        if constexpr (kValue)
+            for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+        const float inv_lam = pow2(lam_exp == INT_MIN ? 0 : -lam_exp);
+
+        // ---- CTA merge over the consumer warps: one partial per segment --------------------
+        consumer_sync();   // all consumers are done with their stages and with mbuf's last use
+        {
+            float* wb = mbuf + pw * kMaxGroup * kPartialStride;
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                float* row = wb + (2 * c + e) * kPartialStride + 16 * g;
+                const float add = kKappa * spv_part[e];
+#pragma unroll
+                for (int q4 = 0; q4 < 4; ++q4) {
+                    float4 v;
+                    v.x = fmaf(acc[2 * q4][e], inv_lam, add);
+                    v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
+                    v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
+                    v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
+                    *reinterpret_cast<float4*>(row + 4 * q4) = v;
+                }
+                if (g == 0) {
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+                    if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                    if constexpr (kValue) {
+                        wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                        wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                    }
+                }
+            }
+        }
+        consumer_sync();
+        const size_t unit = (size_t)b * p.num_kv_heads + h;
+        // flattened plan: share j's segment of sequence b goes to partial h (shares + batch) + j + b
+        const int shares = p.splits / p.num_kv_heads;
+        const size_t pid = kFlat ? (size_t)h * (shares + p.batch) + blockIdx.x / p.num_kv_heads + b
+                                 : unit * p.splits + blockIdx.x;
+        float* part_out = p.partials + pid * (kMaxGroup * kPartialStride);
+        for (int idx = threadIdx.x; idx < G * 33; idx += 32 * kWsPairs) {
+            const int hh = idx / 33, ch = idx % 33;
+            float mw[kWsPairs];
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < kWsPairs; ++w) {
+                mw[w] = mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim];
+                M = fmaxf(M, mw[w]);
+            }
+            float4 s4 = make_float4(0.f, 0.f, 0.f, 0.f);
+            const int col = (ch < 32) ? 4 * ch : kHeadDim + 1;
+#pragma unroll
+            for (int w = 0; w < kWsPairs; ++w) {
+                if (mw[w] == -INFINITY) continue;   // a warp without pages: its values are not read
+                const float wt = fast_exp2(mw[w] - M);
+                const float* src = mbuf + (w * kMaxGroup + hh) * kPartialStride + col;
+                if (ch < 32) {
+                    const float4 v = *reinterpret_cast<const float4*>(src);
+                    s4.x = fmaf(wt, v.x, s4.x); s4.y = fmaf(wt, v.y, s4.y);
+                    s4.z = fmaf(wt, v.z, s4.z); s4.w = fmaf(wt, v.w, s4.w);
+                } else {
+                    s4.x = fmaf(wt, src[0], s4.x);
+                    s4.y = fmaf(wt, src[1], s4.y);
+                    if constexpr (kTierB) s4.z = fmaf(wt, src[2], s4.z);
+                    if constexpr (kValue) s4.w = fmaf(wt, src[3], s4.w);
+                }
+            }
+            float* dst = part_out + hh * kPartialStride;
+            if (ch < 32) {
+                *reinterpret_cast<float4*>(dst + 4 * ch) = s4;
+            } else {
+                dst[kHeadDim] = M;
+                dst[kHeadDim + 1] = s4.x;
+                dst[kHeadDim + 2] = s4.y;
+                if constexpr (kTierB) dst[kHeadDim + 3] = s4.z;
+                if constexpr (kValue) {
+                    float vm = 0.f;
+                    for (int w = 0; w < kWsPairs; ++w)
+                        vm = fmaxf(vm, mbuf[(w * kMaxGroup + hh) * kPartialStride + kHeadDim + 5]);
+                    dst[kHeadDim + 4] = s4.w;
+                    dst[kHeadDim + 5] = vm;
+                }
             }
         }
     }
@@ -1155,6 +1332,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int h = hq / p.group, hh = hq % p.group;
     const size_t unit = (size_t)b * p.num_kv_heads + h;
+    const int count = p.splits;   // split plan (the flattened plan has merge_flat_kernel)
     const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride) + hh * kPartialStride;
     const size_t split_stride = kMaxGroup * kPartialStride;
     __shared__ float red[kMergeWarps][38];
@@ -1164,14 +1342,14 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     constexpr int kMaxRows = 16;   // rows per warp and round
     constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0, repair = (kX & kXRepair) != 0;
     float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f, Vt = 0.f, Vm = 0.f;
-    for (int s0 = warp; s0 < p.splits; s0 += kMergeWarps * kMaxRows) {
+    for (int s0 = warp; s0 < count; s0 += kMergeWarps * kMaxRows) {
         float ms[kMaxRows], v[kMaxRows], ls[kMaxRows], ds[kMaxRows], dbs[kMaxRows], vts[kMaxRows];
 #pragma unroll
         for (int i = 0; i < kMaxRows; ++i) {
             const int s = s0 + i * kMergeWarps;
             ms[i] = -INFINITY;
             v[i] = ls[i] = ds[i] = dbs[i] = vts[i] = 0.f;
-            if (s < p.splits) {
+            if (s < count) {
                 const float* ps = base + s * split_stride;
                 ms[i] = __ldcg(ps + kHeadDim);
                 v[i] = __ldcg(ps + 32 * chunk + lane);
@@ -1304,10 +1482,20 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
     }
     pl.pages_per_split = (int)best_pps;
     pl.splits = (int)std::max<long>(1, (max_pages + best_pps - 1) / best_pps);
+    pl.flat = 0;
+    long partials = units * pl.splits;
+    // A batch of several sequences (lengths unknown to the host, often ragged)
+    // takes the flattened plan: one CTA per SM, equal shares of the pages.
+    if (use_ws(scheme, bits) && batch > 1 && (long long)batch * max_pages < (1LL << 31)) {
+        pl.flat = 1;
+        pl.splits = num_kv_heads * std::max(1, num_sms / num_kv_heads);   // a share per num_kv_heads CTAs
+        pl.pages_per_split = 0;
+        partials = pl.splits + units;
+    }
     auto align = [](size_t x) { return (x + 255) & ~(size_t)255; };
     pl.counters_off = 256;
     pl.partials_off = 256;
-    pl.total = align(pl.partials_off + sizeof(float) * (size_t)units * pl.splits * kMaxGroup * kPartialStride);
+    pl.total = align(pl.partials_off + sizeof(float) * (size_t)partials * kMaxGroup * kPartialStride);
     return pl;
 }
 
@@ -1317,6 +1505,119 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
 // (unused), so no two share an SM and the merge runs spread over the GPU
 // instead of packed onto the first few SMs to free up.
 constexpr int kMergeSpreadSmem = 118784;
+
+// Merge under the flattened plan, where a unit has only a few partials (its
+// sequence's cuts): one warp per (sequence, query head, 32 output dims) folds
+// all of them in order with the same running-maximum update as merge_kernel,
+// so a CTA of 8 warps serves 8 outputs and needs no block barrier.
+template <int kX>
+__global__ void __launch_bounds__(32 * kMergeWarps) merge_flat_kernel(const __grid_constant__ DecodeParams p) {
+    grid_dep_launch();   // the next kernel waits for this grid before reading its outputs
+    grid_dep_wait();
+    const int lane = threadIdx.x & 31;
+    const long long item = (long long)blockIdx.x * kMergeWarps + (threadIdx.x >> 5);
+    if (item >= (long long)p.batch * p.num_q_heads * (kHeadDim / 32)) return;   // warp-uniform
+    const int chunk = (int)(item % (kHeadDim / 32));
+    const int hq = (int)((item / (kHeadDim / 32)) % p.num_q_heads);
+    const int b = (int)(item / ((kHeadDim / 32) * p.num_q_heads));
+    const int h = hq / p.group, hh = hq % p.group;
+    constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0, repair = (kX & kXRepair) != 0;
+
+    // This unit's partials.  The batch's pages lie end to end (sequence b from
+    // P_b = sum_{b' < b} n_b', page counts of the clamped context lengths, as in
+    // the decode); share j of the splits / Hkv shares took positions
+    // [j R, (j + 1) R), R = ceil(total / shares), in each head, so the unit's
+    // segments are those of shares P_b / R .. (P_b + n_b - 1) / R, stored at
+    // partials h (shares + batch) + j + b, consecutive.
+    int before = 0, total = 0;
+    for (int i = lane; i < p.batch; i += 32) {
+        const int np = (max(0, min(__ldg(p.ctx_lens + i), p.max_pages * kPage)) + kPage - 1) / kPage;
+        total += np;
+        if (i < b) before += np;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        before += __shfl_xor_sync(0xffffffffu, before, o);
+        total += __shfl_xor_sync(0xffffffffu, total, o);
+    }
+    const int nb = (max(0, min(__ldg(p.ctx_lens + b), p.max_pages * kPage)) + kPage - 1) / kPage;
+    const int shares = max(1, p.splits / p.num_kv_heads);
+    const long long R = max(1LL, ((long long)total + shares - 1) / shares);
+    const long long j0 = before / R;
+    const int count = nb > 0 ? (int)(((long long)before + nb - 1) / R - j0 + 1) : 0;
+    const float* base = p.partials +
+                        ((size_t)h * (shares + p.batch) + (size_t)(j0 + b)) * (kMaxGroup * kPartialStride) +
+                        hh * kPartialStride;
+
+    constexpr int kRows = 8;   // rows loaded per round before any is combined
+    float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f, Vt = 0.f, Vm = 0.f;
+    for (int s0 = 0; s0 < count; s0 += kRows) {
+        float ms[kRows], v[kRows], ls[kRows], ds[kRows], dbs[kRows], vts[kRows];
+#pragma unroll
+        for (int i = 0; i < kRows; ++i) {
+            ms[i] = -INFINITY;
+            v[i] = ls[i] = ds[i] = dbs[i] = vts[i] = 0.f;
+            if (s0 + i < count) {
+                const float* ps = base + (size_t)(s0 + i) * (kMaxGroup * kPartialStride);
+                ms[i] = __ldcg(ps + kHeadDim);
+                v[i] = __ldcg(ps + 32 * chunk + lane);
+                ls[i] = __ldcg(ps + kHeadDim + 1);
+                ds[i] = __ldcg(ps + kHeadDim + 2);
+                if (tier_b) dbs[i] = __ldcg(ps + kHeadDim + 3);
+                if (vside) {
+                    vts[i] = __ldcg(ps + kHeadDim + 4);
+                    Vm = fmaxf(Vm, __ldcg(ps + kHeadDim + 5));
+                }
+            }
+        }
+        float Mr = M;
+#pragma unroll
+        for (int i = 0; i < kRows; ++i) Mr = fmaxf(Mr, ms[i]);
+        if (Mr == -INFINITY) continue;
+        if (Mr > M) {
+            const float f = (M == -INFINITY) ? 0.f : fast_exp2(M - Mr);
+            acc *= f; L *= f; Dn *= f; Db *= f; Vt *= f;
+            M = Mr;
+        }
+#pragma unroll
+        for (int i = 0; i < kRows; ++i) {
+            if (ms[i] == -INFINITY) continue;
+            const float w = fast_exp2(ms[i] - M);
+            acc = fmaf(w, v[i], acc);
+            L = fmaf(w, ls[i], L);
+            Dn = fmaf(w, ds[i], Dn);
+            Db = fmaf(w, dbs[i], Db);
+            Vt = fmaf(w, vts[i], Vt);
+        }
+    }
+    const size_t cell = (size_t)b * p.num_q_heads + hq;
+    p.out[cell * kHeadDim + 32 * chunk + lane] = L > 0.f ? acc / L : 0.f;
+    if (chunk == 0 && lane == 0) {
+        float raw = 0.f;
+        if (L > 0.f) {
+            const float D = Dn / L;
+            raw = 0.5f * D * (D + 2.0f);
+        }
+        p.meter_raw[cell] = raw;
+        p.meter[cell] = fminf(1.0f, raw);
+        if (repair) p.softmax_norm[cell] = make_float2(M, L);
+        if (tier_b) {
+            float rb = 0.f;
+            if (L > 0.f) {
+                const float D = Db / L;
+                rb = 0.5f * D * (D + 2.0f);
+            }
+            p.meter_b_raw[cell] = rb;
+            p.meter_b[cell] = fminf(1.0f, rb);
+        }
+        if (vside) {
+            const float vterm = L > 0.f ? Vt / L : 0.f;
+            p.value_term[cell] = vterm;
+            p.v_max[cell] = Vm;
+            p.out_bound[cell] = 2.0f * fminf(1.0f, raw) * Vm + vterm;
+        }
+    }
+}
 
 template <int kX>
 static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
@@ -1333,6 +1634,11 @@ static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
                                    (int)cudaSharedmemCarveoutMaxShared);
         (void)cudaGetLastError();   // a refused hint leaves no sticky error behind
     });
+    if (p.pages_per_split == 0) {   // flattened plan
+        const long warps = (long)p.batch * p.num_q_heads * (kHeadDim / 32);
+        return launch_pdl(merge_flat_kernel<kX>, dim3((unsigned)((warps + kMergeWarps - 1) / kMergeWarps)),
+                          dim3(32 * kMergeWarps), 0, stream, p);
+    }
     const dim3 grid(kHeadDim / 32, p.num_q_heads, p.batch);
     const long ctas = (long)grid.x * grid.y * grid.z;
     const size_t smem = (num_sms > 0 && ctas <= num_sms) ? kMergeSpreadSmem : 0;
@@ -1403,7 +1709,7 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     static bool configured = false;
     if (!configured) {
         cudaError_t e = cudaFuncSetAttribute(decode_ws_kernel<kX>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             kWsSmemBytes);
+                                             kWsSmemFlat);
         if (e != cudaSuccess) return e;
         e = cudaFuncSetAttribute(decode_ws_kernel<kX>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  (int)cudaSharedmemCarveoutMaxShared);
@@ -1433,10 +1739,19 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     if (!encode_page_map(&wp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
         !encode_page_map(&wp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
-    dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_ws_kernel<kX>, grid, dim3(kWsThreads), kWsSmemBytes, stream, wp);
+    const bool flat = p.pages_per_split == 0;
+    const dim3 grid = flat ? dim3(p.splits, 1, 1) : dim3(p.splits, p.num_kv_heads, p.batch);
+    cudaError_t e = launch_pdl(decode_ws_kernel<kX>, grid, dim3(kWsThreads), flat ? kWsSmemFlat : kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
-    return launch_merge<kX & ~kXAppend>(p, stream);
+    return launch_merge<kX & ~(kXAppend | kXFlat)>(p, stream);
+}
+
+template <int kF>
+static cudaError_t launch_ws_x(const DecodeParams& p, int x, cudaStream_t stream) {
+    return x == kXTierB  ? launch_ws<kXTierB | kF>(p, stream)
+         : x == kXValue  ? launch_ws<kXValue | kF>(p, stream)
+         : x == kXRepair ? launch_ws<kXRepair | kF>(p, stream)
+         : x == kXAppend ? launch_ws<kXAppend | kF>(p, stream) : launch_ws<kF>(p, stream);
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStream_t stream) {
@@ -1450,11 +1765,8 @@ cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStrea
         return x == kXValue  ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
              : x == kXRepair ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXRepair>(p, stream)
                              : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
-    if (use_ws(scheme, bits))
-        return x == kXTierB  ? launch_ws<kXTierB>(p, stream)
-             : x == kXValue  ? launch_ws<kXValue>(p, stream)
-             : x == kXRepair ? launch_ws<kXRepair>(p, stream)
-             : x == kXAppend ? launch_ws<kXAppend>(p, stream) : launch_ws<0>(p, stream);
+    if (use_ws(scheme, bits))   // pages_per_split == 0: the flattened plan
+        return p.pages_per_split == 0 ? launch_ws_x<kXFlat>(p, x, stream) : launch_ws_x<0>(p, x, stream);
     return x == kXTierB  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
          : x == kXValue  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
          : x == kXRepair ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXRepair>(p, stream)

@@ -61,8 +61,15 @@ struct DecodeParams {
     int32_t num_bypass = 0;
     uint32_t* status;     // workspace word
     uint32_t* counters;   // [batch * Hkv], zero between calls
-    float* partials;      // [batch * Hkv * splits][kMaxGroup][kPartialStride]
+    float* partials;      // [batch * Hkv * splits] (flattened: [splits + batch * Hkv]) x [kMaxGroup][kPartialStride]
     int32_t batch, max_pages, num_q_heads, num_kv_heads, group, num_pages, layer, rope_layout;
+    // pages_per_split == 0 marks the flattened plan (warp-specialized kernel,
+    // batch > 1): the grid is `splits` CTAs, a multiple of Hkv; CTA c serves KV
+    // head c mod Hkv with the (c / Hkv)-th equal share of the batch's pages laid
+    // end to end, cut at sequence boundaries into segments.  Share j's segment of
+    // sequence b writes partial h (shares + batch) + j + b (unique: along the
+    // pages each next segment increments j, b or both), so splits + batch Hkv
+    // partials suffice.
     int32_t splits, pages_per_split;
     PhiloxKeys keys;
 };
@@ -76,8 +83,9 @@ constexpr int kPartialStride = kHeadDim + 12;
 // Workspace layout (bytes): [0, 256) status word, then counters, then
 // partials, each 256-byte aligned.
 struct DecodePlan {
-    int splits;
+    int splits;            // flat: the grid's CTAs
     int pages_per_split;
+    int flat;
     size_t counters_off, partials_off, total;
 };
 

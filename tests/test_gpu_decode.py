@@ -83,6 +83,67 @@ def test_decode_many_splits_long_context():
     _compare(g, o)
 
 
+@pytest.mark.parametrize("ctx_lens,hq,hkv", [
+    ([0, 1, 16, 17, 40, 0, 33, 5] * 25, 8, 2),      # 200 short sequences: CTAs walk many segments
+    ([3000, 1, 0, 16, 2049, 17, 0, 700], 28, 4),     # one long sequence among short and empty ones
+    ([0, 5], 8, 2),
+])
+def test_decode_flattened_plan_batches(ctx_lens, hq, hkv):
+    """A batch of several sequences runs the flattened split plan (each CTA an
+    equal share of all units' pages, cut at unit boundaries): every sequence
+    against the oracle, empty sequences give out = 0 and meter 0."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("f", 1, hq, hkv, ctx_lens, shuffle_pages=True, seed=9)
+    bt, sm, k, v, q = make_inputs(wl, 0)
+    od, gd = descs(hq, hkv, wl.num_pages, 0, 8, 0, 3)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, 0, k.numpy(), v.numpy(), sm, ocache)
+    gcache = wc.LayerCache.empty(gd)
+    wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), gcache)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
+    out, meter, raw = wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, meter, raw = out.cpu().numpy(), meter.cpu().numpy(), raw.cpu().numpy()
+    offs = np.concatenate([[0], np.cumsum(ctx_lens)[:-1]])
+    for b, S in enumerate(ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(meter[b] == 0) and np.all(raw[b] == 0)
+            continue
+        o = offs[b]
+        r = OP.decode_sequence(od, 0, q.numpy()[b], bt[b], S, ocache, k.numpy()[o:o + S], v.numpy()[o:o + S])
+        assert_close(out[b], r["out"], f"out[{b}]")
+        assert_close(meter[b], r["meter"], f"meter[{b}]")
+        assert_close(raw[b], r["meter_raw"], f"meter_raw[{b}]")
+        assert np.all(raw[b] >= r["tv"] * (1 - 1e-3))
+
+
+def test_decode_flattened_plan_bad_ctx_sets_status():
+    """Out-of-range context lengths in a batch are clamped and reported."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("fb", 1, 8, 2, [64, 30], seed=2)
+    bt, sm, k, v, q = make_inputs(wl)
+    od, gd = descs(8, 2, wl.num_pages)
+    cache = wc.LayerCache.empty(gd)
+    wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
+    ws = wc.Workspace(gd, 2, wl.max_pages)
+    btd = torch.from_numpy(bt).cuda()
+    ref = wc.metered_decode_attention(gd, 0, q.cuda(), btd, torch.tensor([64, 30], dtype=torch.int32,
+                                                                            device="cuda"), cache, ws)
+    ref = [t.clone() for t in ref]
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    for bad in ([-5, 30], [64, 10_000]):
+        res = wc.metered_decode_attention(gd, 0, q.cuda(), btd, torch.tensor(bad, dtype=torch.int32, device="cuda"),
+                                          cache, ws)
+        torch.cuda.synchronize()
+        assert wc.read_status(ws) & wc.DEV_BAD_CTX
+        keep = 1 if bad[0] < 0 else 0       # the sequence whose length is valid is unaffected
+        for name, x, y in zip(("out", "meter", "meter_raw"), res, ref):   # (its pages split differently)
+            assert_close(x[keep].cpu().numpy(), y[keep].cpu().numpy().astype(np.float64), name)
+
+
 def test_decode_zero_context_and_repeat_calls():
     """ctx 0 gives out = 0 and meter 0; the workspace is reusable call after call."""
     import paper_2607_28699_gb300 as wc

@@ -102,7 +102,7 @@ def test_fullsize_batch16_paged_prefill():
     wl = W.config(3)
     layer, seed = 27, 202
     gd, bt, sm, k, v, q, cache, out, meter, raw = _gpu_layer(wl, layer, seed)
-    for b, h in [(0, 0), (9, 3), (15, 1)]:
+    for b, h in [(0, 0), (4, 2), (9, 3), (12, 0), (15, 1)]:   # the flattened split plan's segments
         _check_cell(wl, layer, seed, b, h, bt, k, v, q, cache, out, meter, raw)
 
 

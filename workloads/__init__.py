@@ -181,8 +181,9 @@ def layer_kv(wl, layer, device="cpu", seq_range=None):
         g = _gen(wl, layer, 1000 + b, device)
         k = torch.randn(S, H, d, generator=g, device=device) * sig_k
         v = torch.randn(S, H, d, generator=g, device=device) * sig_v
-        k[0] *= 8.0
-        v[0] *= 8.0
+        if S > 0:   # the sink token (an empty sequence has none)
+            k[0] *= 8.0
+            v[0] *= 8.0
         pos = torch.arange(S, device=device)
         ks.append(rope(k, pos).to(torch.float16))
         vs.append(v.to(torch.float16))
