@@ -861,9 +861,6 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     }
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
-    __shared__ int s_wtot[kWsThreads / 32];
-    __shared__ long long s_start;
-    __shared__ WsSeg s_seg[kWsThreads / 32];
     // Split plan: this pair's first page-table entry and the consumer's query
     // fragment are loaded alongside the context length (both in bounds
     // whatever the length; used only if the pair has pages).
@@ -876,19 +873,26 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         if (!producer) load_q_frag(p, blockIdx.z, blockIdx.y, G, g, c, qw);
     }
     WsSeg sg;
-    const bool have = ws_first_segment<kFlat>(p, sg, s_wtot, &s_start);
-    WsSeg* const my_seg = &s_seg[warp];
+    bool have;
+    WsSeg* my_seg = nullptr;   // flattened plan: this warp's walker, in shared memory
     if constexpr (kFlat) {
+        __shared__ int s_wtot[kWsThreads / 32];
+        __shared__ long long s_start;
+        __shared__ WsSeg s_seg[kWsThreads / 32];
+        have = ws_first_segment<true>(p, sg, s_wtot, &s_start);
+        my_seg = &s_seg[warp];
         if (lane == 0) *my_seg = sg;
         __syncwarp();
+    } else {
+        have = ws_first_segment<false>(p, sg, nullptr, nullptr);
     }
 
     if (producer) {
         const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
         int k = 0, issued = 0;   // stage ring position, continued across segments
         bool stop = false;
-        for (bool more = have; more && !stop; more = ws_step<kFlat>(p, my_seg, lane)) {
-            const WsSeg& cs = kFlat ? *my_seg : sg;
+        // one segment's pages (the split plan has one segment: no loop around it)
+        auto produce = [&](const WsSeg& cs) {
             const int b = cs.b, h = cs.h, ctx = cs.ctx, npages = cs.np;
             const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
             const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
@@ -953,6 +957,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 if (lane == 0)   // second arrival: dither tiles and header are written
                     asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(&full[s])) : "memory");
             }
+        };
+        if constexpr (kFlat) {
+            for (bool more = have; more && !stop; more = ws_step<true>(p, my_seg, lane)) produce(*my_seg);
+        } else {
+            produce(sg);
         }
         // copies still in flight must land before the CTA's smem is released
         for (int j = max(0, issued - kWsStages); j < issued; ++j)
@@ -968,8 +977,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
     int k = 0;   // stage ring position, continued across segments
     bool failed = false;
-    for (bool more = have; more; more = ws_step<kFlat>(p, my_seg, lane)) {
-        const WsSeg& cs = kFlat ? *my_seg : sg;
+    // one segment: query setup, pages, CTA merge (the split plan has one segment)
+    auto consume = [&](const WsSeg& cs) {
         const int b = cs.b, h = cs.h, ctx = cs.ctx;
         const bool row_valid = g < G;
         if constexpr (kFlat) load_q_frag(p, b, h, G, g, c, qw);
@@ -1314,6 +1323,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 }
             }
         }
+    };
+    if constexpr (kFlat) {
+        for (bool more = have; more; more = ws_step<true>(p, my_seg, lane)) consume(*my_seg);
+    } else {
+        if (have) consume(sg);
     }
 }
 
