@@ -657,142 +657,6 @@ __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWsPairs) : "memory");
 }
 
-// A CTA's work as segments: pages [a, e) of unit (b, h); page stream (warp
-// pair) w takes pages a + ((w - ph) & 7) + 8 i.  Split plan: one segment, the
-// CTA's split (possibly empty).  Flattened plan: CTA c serves KV head
-// h = c mod Hkv and takes share j = c / Hkv of the batch's pages laid end to
-// end (sequence after sequence), cut at sequence boundaries; the Hkv CTAs of a
-// share read the same pages together (the heads of a page are adjacent in the
-// cache).  ph keeps the streams' round robin running across the cuts, so
-// every stream gets ceil or floor of (hi - lo) / 8 pages.
-struct WsSeg {
-    int b, h, a, e, ph, ctx, np;
-    long long pos;      // flattened position of page a
-    long long lo, hi;   // the CTA's share
-};
-
-__device__ __forceinline__ int clamped_ctx(const DecodeParams& p, int b) {
-    return max(0, min(__ldg(p.ctx_lens + b), p.max_pages * kPage));
-}
-
-// First segment; called by every thread of the CTA (the flattened plan scans
-// the batch's page counts with two block barriers).  False: no pages.
-template <bool kFlat>
-__device__ __forceinline__ bool ws_first_segment(const DecodeParams& p, WsSeg& sg, int* s_wtot, long long* s_start) {
-    if constexpr (!kFlat) {
-        sg.b = blockIdx.z;
-        sg.h = blockIdx.y;
-        int ctx = __ldg(p.ctx_lens + sg.b);
-        if (ctx < 0 || ctx > p.max_pages * kPage) {
-            if (threadIdx.x == 0 && blockIdx.x == 0 && sg.h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
-            ctx = max(0, min(ctx, p.max_pages * kPage));
-        }
-        sg.ctx = ctx;
-        sg.np = (ctx + kPage - 1) / kPage;
-        sg.a = blockIdx.x * p.pages_per_split;
-        sg.e = min(sg.a + p.pages_per_split, sg.np);
-        sg.ph = 0;
-        sg.pos = sg.lo = sg.hi = 0;
-        return true;
-    } else {
-        const int nt = blockDim.x, t = threadIdx.x, per = (p.batch + nt - 1) / nt;
-        int loc = 0;
-        bool bad = false;
-        for (int i = 0; i < per; ++i) {
-            const int bb = t * per + i;
-            if (bb < p.batch) {
-                const int cx = __ldg(p.ctx_lens + bb);
-                bad |= cx < 0 || cx > p.max_pages * kPage;
-                loc += (max(0, min(cx, p.max_pages * kPage)) + kPage - 1) / kPage;
-            }
-        }
-        if (bad && blockIdx.x == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
-        int inc = loc;   // inclusive scan over the warp
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int v = __shfl_up_sync(0xffffffffu, inc, o);
-            if ((t & 31) >= o) inc += v;
-        }
-        if ((t & 31) == 31) s_wtot[t >> 5] = inc;
-        __syncthreads();
-        int before = 0, total = 0;
-        for (int w = 0; w < nt / 32; ++w) {
-            const int v = s_wtot[w];
-            total += v;
-            if (w < (t >> 5)) before += v;
-        }
-        const int excl = before + inc - loc;   // pages of the sequences before this thread's
-        const int hk = p.num_kv_heads, shares = max(1, p.splits / hk);
-        const long long R = max(1LL, ((long long)total + shares - 1) / shares);
-        const long long lo = (long long)(blockIdx.x / hk) * R, hi = min((long long)total, lo + R);
-        if (lo < hi && excl <= lo && lo < (long long)excl + loc) {
-            long long acc = excl;   // exactly one thread: the one whose sequences hold lo
-            for (int i = 0; i < per; ++i) {
-                const int bb = t * per + i;
-                if (bb >= p.batch) break;
-                const int np = (clamped_ctx(p, bb) + kPage - 1) / kPage;
-                if (lo < acc + np) {
-                    *s_start = ((long long)bb << 32) | (long long)(lo - acc);
-                    break;
-                }
-                acc += np;
-            }
-        }
-        __syncthreads();
-        if (lo >= hi) return false;
-        const long long st = *s_start;
-        sg.b = (int)(st >> 32);
-        sg.a = (int)(st & 0xffffffffLL);
-        sg.h = blockIdx.x % hk;
-        sg.ctx = clamped_ctx(p, sg.b);
-        sg.np = (sg.ctx + kPage - 1) / kPage;
-        sg.e = (int)min((long long)sg.np, sg.a + (hi - lo));
-        sg.ph = 0;
-        sg.pos = sg.lo = lo;
-        sg.hi = hi;
-        return true;
-    }
-}
-
-// Next segment of the flattened plan (the next sequence with pages); false
-// at the end of the CTA's share, and always in the split plan.
-template <bool kFlat>
-__device__ __forceinline__ bool ws_next_segment(const DecodeParams& p, WsSeg& sg) {
-    if constexpr (!kFlat) return false;
-    sg.pos += sg.e - sg.a;
-    if (sg.pos >= sg.hi) return false;
-    do {   // sequences without pages hold no part of the share
-        if (sg.b + 1 >= p.batch) return false;
-        ++sg.b;
-        sg.ctx = clamped_ctx(p, sg.b);
-        sg.np = (sg.ctx + kPage - 1) / kPage;
-    } while (sg.np == 0);
-    sg.a = 0;
-    sg.e = (int)min((long long)sg.np, sg.hi - sg.pos);
-    sg.ph = (int)((sg.pos - sg.lo) & (kWsPairs - 1));
-    return true;
-}
-
-static_assert((kWsPairs & (kWsPairs - 1)) == 0, "the page streams' round robin uses a mask");
-
-// Flattened plan: each warp's walker lives in a shared slot, so that only the
-// current segment's indices take registers in the page loop; lane 0 advances it.
-template <bool kFlat>
-__device__ __forceinline__ bool ws_step(const DecodeParams& p, WsSeg* slot, int lane) {
-    if constexpr (!kFlat) {
-        return false;
-    } else {
-        __syncwarp();
-        int more = 0;
-        if (lane == 0) more = ws_next_segment<true>(p, *slot);
-        __syncwarp();
-        return __shfl_sync(0xffffffffu, more, 0) != 0;
-    }
-}
-__device__ __forceinline__ int ws_seg_pages(const WsSeg& sg, int w, int& first) {
-    first = sg.a + ((w - sg.ph) & (kWsPairs - 1));
-    return first < sg.e ? (sg.e - first + kWsPairs - 1) / kWsPairs : 0;
-}
 
 // q fragment of the B operand (head g, channels 32c + 2i, +1 in word i).
 __device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h, int G, int g, int c,
@@ -897,7 +761,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
             const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
             int first;
-            const int n_seg = ws_seg_pages(cs, pw, first);
+            const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);
             int phys_next = kFlat ? (n_seg > 0 ? __ldg(bt_row + first) : -1) : phys_first;
             for (int i = 0; i < n_seg; ++i, ++k) {
                 const int lp = first + kWsPairs * i;
@@ -959,7 +823,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             }
         };
         if constexpr (kFlat) {
-            for (bool more = have; more && !stop; more = ws_step<true>(p, my_seg, lane)) produce(*my_seg);
+            for (bool more = have; more && !stop; more = ws_step<kWsPairs, true>(p, my_seg, lane)) produce(*my_seg);
         } else {
             produce(sg);
         }
@@ -1038,7 +902,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         int lam_exp = INT_MIN;
 
         int first;
-        const int n_seg = ws_seg_pages(cs, pw, first);
+        const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);
         for (int i = 0; i < n_seg && !failed; ++i, ++k) {
             const int s = k % kWsStages;
             const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kWsStages) & 1));
@@ -1325,7 +1189,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         }
     };
     if constexpr (kFlat) {
-        for (bool more = have; more; more = ws_step<true>(p, my_seg, lane)) consume(*my_seg);
+        for (bool more = have; more; more = ws_step<kWsPairs, true>(p, my_seg, lane)) consume(*my_seg);
     } else {
         if (have) consume(sg);
     }
@@ -1500,7 +1364,8 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
     long partials = units * pl.splits;
     // A batch of several sequences (lengths unknown to the host, often ragged)
     // takes the flattened plan: one CTA per SM, equal shares of the pages.
-    if (use_ws(scheme, bits) && batch > 1 && (long long)batch * max_pages < (1LL << 31)) {
+    if ((use_ws(scheme, bits) || scheme == WC_SCHEME_DITHER_INT8_G32) && batch > 1 &&
+        (long long)batch * max_pages < (1LL << 31)) {
         pl.flat = 1;
         pl.splits = num_kv_heads * std::max(1, num_sms / num_kv_heads);   // a share per num_kv_heads CTAs
         pl.pages_per_split = 0;

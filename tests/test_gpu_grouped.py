@@ -112,6 +112,38 @@ def test_grouped_decode_matches_oracle(m, layout):
     assert np.all(ref["tv"] <= raw.cpu().numpy() * (1 + 1e-3))        # the GPU's meter bounds the true TV
 
 
+@pytest.mark.parametrize("ctx_lens", [[0, 1, 16, 17, 40, 0, 33, 5] * 25, [3000, 1, 0, 16, 2049, 17, 0, 700]])
+def test_grouped_decode_flattened_plan_batches(ctx_lens):
+    """A batch runs the grouped decode under the flattened split plan (6 page
+    streams per CTA, shares cut at sequence boundaries): every sequence against
+    the oracle, with and without Tier B; empty sequences give out = 0, meter 0."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("gf", 1, 28, 4, ctx_lens, shuffle_pages=True, seed=61)
+    layer, m = 1, 4
+    bt, k, v, q, od, gd, ocache, _ = _write_both(wl, layer, m, Q.ROPE_HALF, 17)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
+    qd, btd = q.cuda(), torch.from_numpy(bt).cuda()
+    delta = 1e-4
+    out, meter, raw = wc.metered_decode_attention(gd, layer, qd, btd, ctx, gcache, ws)
+    res_b = wc.metered_decode_attention_tier_b(gd, layer, qd, btd, ctx, gcache, ws, delta)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, raw, raw_b = out.cpu().numpy(), raw.cpu().numpy(), res_b[4].cpu().numpy()
+    offs = np.concatenate([[0], np.cumsum(ctx_lens)[:-1]])
+    for b, S in enumerate(ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(raw[b] == 0) and np.all(raw_b[b] == 0)
+            continue
+        r = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, k[offs[b]:offs[b] + S],
+                               v[offs[b]:offs[b] + S], delta_loc=delta)
+        assert_close(out[b], r["out"], f"out[{b}]", atol=1e-4)
+        assert_close(raw[b], r["meter_raw"], f"meter_raw[{b}]")
+        assert_close(raw_b[b], r["meter_b_raw"], f"meter_b_raw[{b}]")
+        assert np.all(r["tv"] <= raw[b] * (1 + 1e-3))
+
+
 def test_grouped_bypass_lowers_the_meter_on_massive_pairs():
     """Table "amax" on the GPU path: with massive pairs, the grouped cache
     that bypasses them (and leaves them out of the amax) meters far lower."""
