@@ -178,7 +178,10 @@ size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_p
  *   c_t             = (1/sqrt(128)) sum_b ||q_b|| w_{t,b}
  *   meter_raw[b][hq] = 1/2 (A^2 - 1), A = sum_t p~_t e^{c_t}  (+inf on fp32 overflow)
  *   meter[b][hq]    = min(1, meter_raw)
- * The context is split across CTAs; partial softmax, output and A
+ * The context is split across CTAs (one sequence: every KV head's pages in
+ * equal splits; several sequences, whose lengths only the device sees: each
+ * CTA serves one KV head and an equal share of the batch's pages laid end to
+ * end, cut at sequence boundaries); partial softmax, output and A
  * accumulators are merged under log-sum-exp weights (A is a p~-weighted mean,
  * §6.2.2) by a second kernel, launched as a programmatic dependent of the
  * first (two launches per call).  A sequence with
@@ -272,8 +275,9 @@ wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer
  *   dev_status  optional device uint32 that collects WC_DEV_* bits (OR); when
  *               NULL the bits go to a word inside the built-in scratch.
  * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
- * more scratch than 4 MiB (about 930 (sequence, KV head, split) partial
- * results; the split count follows wc_workspace_size's plan).
+ * more scratch than 4 MiB (about 930 partial results: one per (KV head,
+ * split) for one sequence; the SM count plus batch x Hkv for several
+ * sequences; the count follows wc_workspace_size's plan).
  * The first call on each device looks up the scratch address and clears its
  * status word (a synchronous cudaMemset); make that first call before any
  * stream capture.  All calls share the one scratch array and it keeps the
