@@ -7,8 +7,10 @@
 // split measured slower).  A producer stages a page (code tiles by TMA with the
 // 128-byte swizzle; scales, witness and bypass values by bulk copy) and
 // regenerates its dither into swizzled byte tiles; its consumer runs the math
-// below with no Philox on its path.  The split-K partials and the merge are the
-// per-token kernel's.  What differs from the per-token math:
+// below with no Philox on its path.  The split plans (one sequence: equal
+// splits; a batch: the flattened plan's per-head shares, walked as segments),
+// the split-K partials and the merges are the per-token kernel's.  What differs
+// from the per-token math:
 //
 //  - A row is stored in the order the mma fragments consume it (storage
 //    position p of K holds channel 16 ((p >> 2) & 7) + 4 (p >> 5) + (p & 3),
