@@ -87,6 +87,7 @@ def test_decode_many_splits_long_context():
     ([0, 1, 16, 17, 40, 0, 33, 5] * 25, 8, 2),      # 200 short sequences: CTAs walk many segments
     ([3000, 1, 0, 16, 2049, 17, 0, 700], 28, 4),     # one long sequence among short and empty ones
     ([0, 5], 8, 2),
+    ([(37 * i) % 41 for i in range(600)], 8, 2),    # more sequences than the CTA's threads: several each
 ])
 def test_decode_flattened_plan_batches(ctx_lens, hq, hkv):
     """A batch of several sequences runs the flattened split plan (each CTA an

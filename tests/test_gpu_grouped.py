@@ -112,7 +112,8 @@ def test_grouped_decode_matches_oracle(m, layout):
     assert np.all(ref["tv"] <= raw.cpu().numpy() * (1 + 1e-3))        # the GPU's meter bounds the true TV
 
 
-@pytest.mark.parametrize("ctx_lens", [[0, 1, 16, 17, 40, 0, 33, 5] * 25, [3000, 1, 0, 16, 2049, 17, 0, 700]])
+@pytest.mark.parametrize("ctx_lens", [[0, 1, 16, 17, 40, 0, 33, 5] * 25, [3000, 1, 0, 16, 2049, 17, 0, 700],
+                                      [(37 * i) % 41 for i in range(500)]])
 def test_grouped_decode_flattened_plan_batches(ctx_lens):
     """A batch runs the grouped decode under the flattened split plan (6 page
     streams per CTA, shares cut at sequence boundaries): every sequence against
