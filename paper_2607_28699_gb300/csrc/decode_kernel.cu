@@ -1360,13 +1360,12 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
     }
     pl.pages_per_split = (int)best_pps;
     pl.splits = (int)std::max<long>(1, (max_pages + best_pps - 1) / best_pps);
-    pl.flat = 0;
     long partials = units * pl.splits;
     // A batch of several sequences (lengths unknown to the host, often ragged)
-    // takes the flattened plan: one CTA per SM, equal shares of the pages.
+    // takes the flattened plan: Hkv x floor(SMs / Hkv) CTAs, one per SM, each
+    // an equal share of one KV head's pages.
     if ((use_ws(scheme, bits) || scheme == WC_SCHEME_DITHER_INT8_G32) && batch > 1 &&
         (long long)batch * max_pages < (1LL << 31)) {
-        pl.flat = 1;
         pl.splits = num_kv_heads * std::max(1, num_sms / num_kv_heads);   // a share per num_kv_heads CTAs
         pl.pages_per_split = 0;
         partials = pl.splits + units;

@@ -83,9 +83,8 @@ constexpr int kPartialStride = kHeadDim + 12;
 // Workspace layout (bytes): [0, 256) status word, then counters, then
 // partials, each 256-byte aligned.
 struct DecodePlan {
-    int splits;            // flat: the grid's CTAs
-    int pages_per_split;
-    int flat;
+    int splits;            // flattened plan: the grid's CTAs
+    int pages_per_split;   // 0: the flattened plan
     size_t counters_off, partials_off, total;
 };
 
