@@ -1,0 +1,56 @@
+"""bench.py's host side, without a GPU: the reference arm's JSON line (the
+oracle on the host's cores, as the benchmark contract specifies it) and the
+single-buffer packing the end-to-end step copies with."""
+
+import importlib.util
+import json
+import os
+import subprocess
+import sys
+
+import torch
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _bench_module():
+    spec = importlib.util.spec_from_file_location("bench_under_test", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_pack_views_share_one_aligned_buffer():
+    b = _bench_module()
+    q = torch.randn(3, 2, 5, 128).half()
+    ctx = torch.tensor([7, 9, 0], dtype=torch.int32)
+    meter = torch.rand(3, 2, 5)
+    keep = torch.randint(0, 2, (30,), dtype=torch.uint8)
+    buf, (q2, ctx2, meter2, keep2) = b._pack((q, ctx, meter, keep))
+    for orig, view in ((q, q2), (ctx, ctx2), (meter, meter2), (keep, keep2)):
+        assert torch.equal(orig, view) and view.shape == orig.shape and view.dtype == orig.dtype
+        assert (view.data_ptr() - buf.data_ptr()) % 256 == 0
+        assert buf.data_ptr() <= view.data_ptr() < buf.data_ptr() + buf.numel()
+    ctx2[1] = 41                                  # a write through a view lands in the buffer
+    off = ctx2.data_ptr() - buf.data_ptr()
+    assert buf[off:off + 12].view(torch.int32).tolist() == [7, 41, 0]
+    assert buf.numel() % 256 == 0
+
+
+def test_reference_arm_prints_the_contract_line():
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "1",
+                        "--steps", "1", "--warmup", "3", "--cpu-budget", "0.5"],
+                       capture_output=True, text=True, timeout=600, env=env, cwd=ROOT)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = [x for x in r.stdout.splitlines() if x.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+                "scaling", "vs_baseline", "dtype", "data", "config", "impl", "cpu_baseline", "e2e"):
+        assert key in d, key
+    assert d["impl"] == "reference" and d["value"] > 0 and d["higher_is_better"] is True
+    assert d["cpu_baseline"]["kind"] == "oracle" and d["cpu_baseline"]["cores"] >= 1
+    assert d["cpu_baseline"]["value"] == d["value"]
+    assert d["e2e"] == {"value": d["value"], "unit": d["unit"], "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
+    assert d["config"]["workload"].startswith("1L-8q2kv-S4096")
