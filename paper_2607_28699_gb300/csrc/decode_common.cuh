@@ -41,6 +41,8 @@ struct DitherConst<10> {  // xi = (j + 1/2)/1024 - 1/2 = h' - kappa, h' = 1 + j/
 
 // h' pair (fp16) for two 8-bit dithers: bytes of x at the selector.
 __device__ __forceinline__ uint32_t h8(uint32_t x, uint32_t sel) { return prmt(x, 0x44444444u, sel); }
+// -h' pair (fp16) for two 8-bit dithers: the same bytes under a negative high byte.
+__device__ __forceinline__ uint32_t nh8(uint32_t x, uint32_t sel) { return prmt(x, 0xC4C4C4C4u, sel); }
 // h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
 __device__ __forceinline__ uint32_t h10(uint32_t x) { return (x & 0x03FF03FFu) | 0x3C003C00u; }
 
@@ -56,6 +58,21 @@ __device__ __forceinline__ uint32_t movmatrix_t(uint32_t x) {
     uint32_t y;
     asm volatile("movmatrix.sync.aligned.m8n8.trans.b16 %0, %1;" : "=r"(y) : "r"(x));
     return y;
+}
+
+// Token held by row r of a 16-row QK / softmax tile in the warp-specialized
+// decode: rows 2i, 2i+1 hold tokens 4i, 4i+1 and rows 8+2i, 9+2i tokens
+// 4i+2, 4i+3, so the P fragment transposed by movmatrix gives lane (g, c) the
+// tokens 4c .. 4c+3 that ldmatrix.trans delivers for V.
+__device__ __forceinline__ int tok_row(int r) { return 4 * ((r & 7) >> 1) + 2 * (r >> 3) + (r & 1); }
+
+// ldmatrix.trans of two 16x16 byte blocks: lanes 0-15 address the 16 rows of
+// the first, lanes 16-31 those of the second; lane (g, c) receives, per block,
+// column g (first word) and column g + 8 (second word) at rows 4c .. 4c+3.
+__device__ __forceinline__ void ldsm_t_b8_x2(uint32_t (&d)[4], const void* row) {
+    asm volatile("ldmatrix.sync.aligned.m16n16.x2.trans.shared.b8 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(d[0]), "=r"(d[1]), "=r"(d[2]), "=r"(d[3])
+                 : "r"(smem_addr(row)));
 }
 
 // Byte offset of 16-byte chunk q of token row t in a tile written with the

@@ -752,7 +752,6 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     }
 
     if (producer) {
-        const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
         int k = 0, issued = 0;   // stage ring position, continued across segments
         bool stop = false;
         // one segment's pages (the split plan has one segment: no loop around it)
@@ -801,21 +800,24 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 issued = k + 1;
                 if (ok) {
                     // dither bytes j[token][channel]: one Philox call covers 16
-                    // channels of one token (channel i = byte i%4 of word i/4)
+                    // channels of one token (channel i = byte i%4 of word i/4).
+                    // Each lane draws K and V for the same (token, channel group)
+                    // (tokens g, g+8 x groups 2c, 2c+1), so the two calls share
+                    // their first round's product.
                     const uint32_t slot0 = (uint32_t)phys * kPage;
                     uint4 dk[4], dv[4];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x channel groups 2c, 2c+1
-                        dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
+                    for (int i = 0; i < 4; ++i) {
+                        const uint32_t slot = slot0 + g + 8 * (i >> 1), grp = (uint32_t)(2 * c + (i & 1));
+                        dk[i] = philox(slot, c1, grp, 0u, p.keys);
+                        dv[i] = philox(slot, c1, grp, 1u, p.keys);
+                    }
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x channel group g
-                        dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        *reinterpret_cast<uint4*>(st + kWsOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        *reinterpret_cast<uint4*>(st + kWsOffVd + swz(tv[j], g)) = dv[j];
+                    for (int i = 0; i < 4; ++i) {
+                        const int off = swz(g + 8 * (i >> 1), 2 * c + (i & 1));
+                        *reinterpret_cast<uint4*>(st + kWsOffKd + off) = dk[i];
+                        *reinterpret_cast<uint4*>(st + kWsOffVd + off) = dv[i];
+                    }
                 }
                 __syncwarp();
                 if (lane == 0)   // second arrival: dither tiles and header are written
@@ -838,7 +840,10 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     // split plan (one segment, the producers are done with it), a buffer of its
     // own in the flattened plan (the producers stage the next segment meanwhile).
     float* mbuf = reinterpret_cast<float*>(kFlat ? smem + kWsMergeOff : smem);
-    const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
+    // Token rows: row g of the QK and softmax tiles holds token t0, row g + 8
+    // token t1 (tok_row), so that the P fragment transposed by movmatrix pairs
+    // tokens (4c, 4c+1) and (4c+2, 4c+3), as ldmatrix.trans delivers V.
+    const int t0 = tok_row(g), t1 = tok_row(g + 8);
     int k = 0;   // stage ring position, continued across segments
     bool failed = false;
     // one segment: query setup, pages, CTA merge (the split plan has one segment)
@@ -881,9 +886,9 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             band_a = part[0] + part[1];
             band_b = part[2] + part[3];
         }
-        uint32_t a_hi = 0, a_lo = 0;
+        uint32_t a_hi = 0, a_lo = 0;   // ||q_b|| log2(e) / sqrt(d), hi + lo: the bound in log2 units
         if (row_valid) {
-            const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
+            const float x0 = sqrtf(band_a) * kRsdLog2e, x1 = sqrtf(band_b) * kRsdLog2e;
             const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
             a_hi = pack_h2(__half2float(h0), __half2float(h1));
             a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
@@ -900,6 +905,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
         int lam_exp = INT_MIN;
+        float sv_lim = 0.f;   // 2^(6 - lam_exp); 0 until the first positive scale
 
         int first;
         const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);
@@ -917,14 +923,15 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const int nvalid = min(kPage, ctx - lp * kPage);
 
                 // ---------------- QK: S[token][head] = code.q - h'.q -------------------
+                // Row g of the QK tile holds token t0, row g + 8 token t1 (see tok_row).
                 float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
                 for (int gp = 0; gp < 2; ++gp) {
                     const int q16 = 2 * c + gp;   // 16-byte chunk: channels 32c + 16gp .. +15
-                    const uint4 ka = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g, q16));
-                    const uint4 kb = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(g + 8, q16));
-                    const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g, q16));
-                    const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(g + 8, q16));
+                    const uint4 ka = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(t0, q16));
+                    const uint4 kb = *reinterpret_cast<const uint4*>(st + kWsOffK + swz(t1, q16));
+                    const uint4 ja = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(t0, q16));
+                    const uint4 jb = *reinterpret_cast<const uint4*>(st + kWsOffKd + swz(t1, q16));
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk) {
                         const int ks = 4 * gp + kk;
@@ -939,149 +946,145 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 }
 
                 // ---------------- logits, bound, softmax ------------------------------
-                float cb[4] = {0.f, 0.f, 0.f, 0.f};
+                float cb[4] = {0.f, 0.f, 0.f, 0.f};   // log2-domain bound (a carries log2 e)
                 {
-                    const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (g * kBands + 2 * c) * 2);
-                    const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kWsOffW + ((g + 8) * kBands + 2 * c) * 2);
+                    const uint32_t wa = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (t0 * kBands + 2 * c) * 2);
+                    const uint32_t wb = *reinterpret_cast<const uint32_t*>(st + kWsOffW + (t1 * kBands + 2 * c) * 2);
                     mma1688(cb, wa, wb, a_hi);
                     mma1688(cb, wa, wb, a_lo);
                 }
                 const __half* ksc = reinterpret_cast<const __half*>(st + kWsOffKs);
                 const __half* vsc = reinterpret_cast<const __half*>(st + kWsOffVs);
-                float sk[2] = {__half2float(ksc[g]), __half2float(ksc[g + 8])};
-                float sv[2] = {__half2float(vsc[g]), __half2float(vsc[g + 8])};
-                float y[4], P[4];
-                const bool ok0 = g < nvalid, ok1 = g + 8 < nvalid;
+                float sk[2] = {__half2float(ksc[t0]), __half2float(ksc[t1])};
+                float sv[2] = {__half2float(vsc[t0]), __half2float(vsc[t1])};
+                float y[4];
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = i >> 1, e = i & 1;
-                    const bool okr = r ? ok1 : ok0;
-                    const float raw = dc[i] - dd[i] + (e ? zoff1 : zoff0);
-                    y[i] = okr ? raw * (sk[r] * kRsdLog2e) : -INFINITY;
-                    if (!okr) cb[i] = 0.f;                 // tail slots may hold any bits
+                    y[i] = (dc[i] - dd[i] + (e ? zoff1 : zoff0)) * (sk[r] * kRsdLog2e);
                 }
-                if (!ok0) sv[0] = 0.f;
-                if (!ok1) sv[1] = 0.f;
-                if constexpr (kTierB) {
-                    if (!ok0) sk[0] = 0.f;
-                    if (!ok1) sk[1] = 0.f;
-                }
-                float rho[2] = {0.f, 0.f};   // value witness of tokens g, g+8 (0 past the context)
+                float rho[2] = {0.f, 0.f};   // value witness of tokens t0, t1 (0 past the context)
                 if constexpr (kValue) {
-                    const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * g));
-                    const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * (g + 8)));
-                    if (ok0) { rho[0] = w0.x; vmax = fmaxf(vmax, w0.y); }
-                    if (ok1) { rho[1] = w1.x; vmax = fmaxf(vmax, w1.y); }
-                }
-                float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
-#pragma unroll
-                for (int o = 4; o < 32; o <<= 1) {
-                    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-                    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
-                }
-                const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
-                if (__any_sync(0xffffffffu, mv0 || mv1)) {
-                    const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
-                    const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
-                    if (mv0) m_run[0] = mx0;
-                    if (mv1) m_run[1] = mx1;
-                    l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
-                    l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
-                    if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
-                    if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
-#pragma unroll
-                    for (int mt = 0; mt < 8; ++mt) {
-                        acc[mt][0] *= a0; acc[mt][2] *= a0;
-                        acc[mt][1] *= a1; acc[mt][3] *= a1;
+                    const float2 w0 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * t0));
+                    const float2 w1 = __half22float2(*reinterpret_cast<const __half2*>(st + kWsOffVw + 4 * t1));
+                    rho[0] = w0.x;
+                    rho[1] = w1.x;
+                    if (nvalid == kPage) vmax = fmaxf(vmax, fmaxf(w0.y, w1.y));
+                    else {
+                        if (t0 < nvalid) vmax = fmaxf(vmax, w0.y);
+                        if (t1 < nvalid) vmax = fmaxf(vmax, w1.y);
                     }
                 }
+                if (nvalid < kPage) {   // the context's last page (warp-uniform): slots past it hold any bits
+                    const bool ok0 = t0 < nvalid, ok1 = t1 < nvalid;
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        if (!((i >> 1) ? ok1 : ok0)) {
+                            y[i] = -INFINITY;
+                            cb[i] = 0.f;
+                        }
+                    if (!ok0) sv[0] = sk[0] = rho[0] = 0.f;
+                    if (!ok1) sv[1] = sk[1] = rho[1] = 0.f;
+                }
+                // running maximum, moved lazily: only when a logit exceeds it by more
+                // than 8 (the column maximum over the token rows is reduced only then)
+                {
+                    float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+                    if (__any_sync(0xffffffffu, mx0 > m_run[0] + 8.0f || mx1 > m_run[1] + 8.0f)) {
+#pragma unroll
+                        for (int o = 4; o < 32; o <<= 1) {
+                            mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+                            mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+                        }
+                        const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
+                        const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
+                        const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
+                        if (mv0) m_run[0] = mx0;
+                        if (mv1) m_run[1] = mx1;
+                        l_part[0] *= a0; d_part[0] *= a0; spv_part[0] *= a0;
+                        l_part[1] *= a1; d_part[1] *= a1; spv_part[1] *= a1;
+                        if constexpr (kTierB) { db_part[0] *= a0; db_part[1] *= a1; }
+                        if constexpr (kValue) { vt_part[0] *= a0; vt_part[1] *= a1; }
+#pragma unroll
+                        for (int mt = 0; mt < 8; ++mt) {
+                            acc[mt][0] *= a0; acc[mt][2] *= a0;
+                            acc[mt][1] *= a1; acc[mt][3] *= a1;
+                        }
+                    }
+                }
+                // P * s_v * 2^lam_exp stays below 2^14 (fp16): s_v * 2^lam_exp < 2^6.
+                // lam_exp only decreases; sv_lim = 2^(6 - lam_exp) is the scale at which it must.
+                if (__any_sync(0xffffffffu, fmaxf(sv[0], sv[1]) >= sv_lim)) {
+                    const float smax = fmaxf(sv[0], sv[1]);
+                    const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
+                    const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
+                    const int want = 6 - e;
+                    if (lam_exp != INT_MIN) {   // want < lam_exp here
+                        const float f = pow2(want - lam_exp);
+#pragma unroll
+                        for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+                            for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
+                        spv_part[0] *= f;
+                        spv_part[1] *= f;
+                    }
+                    lam_exp = want;
+                    sv_lim = pow2(6 - lam_exp);
+                }
+                const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
+                const float svl[2] = {sv[0] * lam, sv[1] * lam};   // exact: lam is a power of two
                 float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
+                float x[4];                  // P * s_v * lam, the PV operand
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = i >> 1, e = i & 1;
                     const float pe = fast_exp2(y[i] - m_run[e]);
                     l_part[e] += pe;
-                    const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
+                    const float em1 = fast_exp2(cb[i]) - 1.f;
                     d_part[e] = fmaf(pe, em1, d_part[e]);
                     if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
                     if constexpr (kTierB)
                         db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                     if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
-                    P[i] = pe * sv[r];
-                    spv_part[e] += P[i];
+                    x[i] = pe * svl[r];
+                    spv_part[e] += x[i];     // sum P s_v, in the lam frame
                 }
                 if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
-                {
-                    const float smax = fmaxf(sv[0], sv[1]);
-                    const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
-                    if (wmax > 0.f) {
-                        const int e = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^e
-                        const int want = 6 - e;
-                        if (lam_exp == INT_MIN) {
-                            lam_exp = want;
-                        } else if (want < lam_exp) {
-                            const float f = pow2(want - lam_exp);
-#pragma unroll
-                            for (int mt = 0; mt < 8; ++mt)
-#pragma unroll
-                                for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
-                            lam_exp = want;
-                        }
-                    }
-                }
                 uint32_t bp0, bp1, bl0, bl1;
                 {
-                    const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
-                    const float x0 = P[0] * lam, x1 = P[1] * lam, x2 = P[2] * lam, x3 = P[3] * lam;
-                    const uint32_t h01 = pack_h2(x0, x1), h23 = pack_h2(x2, x3);
+                    const uint32_t h01 = pack_h2(x[0], x[1]), h23 = pack_h2(x[2], x[3]);
                     const float2 r01 = __half22float2(*reinterpret_cast<const __half2*>(&h01));
                     const float2 r23 = __half22float2(*reinterpret_cast<const __half2*>(&h23));
-                    const uint32_t l01 = pack_h2(x0 - r01.x, x1 - r01.y), l23 = pack_h2(x2 - r23.x, x3 - r23.y);
+                    const uint32_t l01 = pack_h2(x[0] - r01.x, x[1] - r01.y), l23 = pack_h2(x[2] - r23.x, x[3] - r23.y);
+                    // B operand: P[tokens 4c, 4c+1][head g] and P[tokens 4c+2, 4c+3][head g]
                     bp0 = movmatrix_t(h01);
                     bp1 = movmatrix_t(h23);
                     bl0 = movmatrix_t(l01);
                     bl1 = movmatrix_t(l23);
                 }
 
-                // ---------------- PV: acc[dim][head] ------------------------------------
-                {
-                    uint4 vq[4];
+                // ---------------- PV: acc[dim][head] += (code - h') P -----------------
+                // ldmatrix.trans of a 16x16 byte block (tokens x dims 16mt..16mt+15)
+                // gives lane (g, c) dims 16mt + g (first word) and 16mt + g + 8 (second)
+                // at tokens 4c .. 4c+3: the A operand with k slots 2c, 2c+1, 2c+8,
+                // 2c+9 holding tokens 4c .. 4c+3, the order B was built in.
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) vq[j] = *reinterpret_cast<const uint4*>(st + kWsOffV + swz(tv[j], g));
+                for (int mp = 0; mp < 4; ++mp) {   // m-tiles 2mp, 2mp+1
+                    uint32_t v[4], j[4];
+                    ldsm_t_b8_x2(v, st + kWsOffV + swz(lane & 15, 2 * mp + (lane >> 4)));
+                    ldsm_t_b8_x2(j, st + kWsOffVd + swz(lane & 15, 2 * mp + (lane >> 4)));
 #pragma unroll
-                    for (int mt = 0; mt < 8; ++mt) {
-                        const int wi = mt >> 1, pos = 2 * (mt & 1);
-                        uint32_t A[4];
-#pragma unroll
-                        for (int pr = 0; pr < 2; ++pr) {
-                            const uint32_t X = prmt(word_of(vq[2 * pr], wi) ^ 0x80808080u,
-                                                    word_of(vq[2 * pr + 1], wi) ^ 0x80808080u, sel_interleave(pos));
-                            A[2 * pr] = s8x2_to_h2(X, kSel01);
-                            A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
-                        }
+                    for (int u = 0; u < 2; ++u) {
+                        const int mt = 2 * mp + u;
+                        const uint32_t x0 = v[2 * u] ^ 0x80808080u, x1 = v[2 * u + 1] ^ 0x80808080u;
+                        const uint32_t A[4] = {s8x2_to_h2(x0, kSel01), s8x2_to_h2(x1, kSel01), s8x2_to_h2(x0, kSel23),
+                                               s8x2_to_h2(x1, kSel23)};
                         mma16816(acc[mt], A, bp0, bp1);
                         mma16816(acc[mt], A, bl0, bl1);
-                    }
-                }
-                {
-                    const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
-                    const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
-                    uint4 dv[4];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) dv[j] = *reinterpret_cast<const uint4*>(st + kWsOffVd + swz(tv[j], g));
-#pragma unroll
-                    for (int mt = 0; mt < 8; ++mt) {
-                        const int wi = mt >> 1, pos = 2 * (mt & 1);
-                        uint32_t H[4];
-#pragma unroll
-                        for (int pr = 0; pr < 2; ++pr) {
-                            const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
-                                                    sel_interleave(pos));
-                            H[2 * pr] = h8(Y, kSel01);
-                            H[2 * pr + 1] = h8(Y, kSel23);
-                        }
-                        mma16816(acc[mt], H, bn0, bn1);
-                        mma16816(acc[mt], H, bm0, bm1);
+                        const uint32_t H[4] = {nh8(j[2 * u], kSel01), nh8(j[2 * u + 1], kSel01),
+                                               nh8(j[2 * u], kSel23), nh8(j[2 * u + 1], kSel23)};
+                        mma16816(acc[mt], H, bp0, bp1);
+                        mma16816(acc[mt], H, bl0, bl1);
                     }
                 }
             } else if constexpr (kRepair) {
@@ -1113,16 +1116,12 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             float* wb = mbuf + pw * kMaxGroup * kPartialStride;
 #pragma unroll
             for (int e = 0; e < 2; ++e) {
-                float* row = wb + (2 * c + e) * kPartialStride + 16 * g;
-                const float add = kKappa * spv_part[e];
+                float* row = wb + (2 * c + e) * kPartialStride;
+                const float add = kKappa * spv_part[e] * inv_lam;   // spv is in the lam frame
 #pragma unroll
-                for (int q4 = 0; q4 < 4; ++q4) {
-                    float4 v;
-                    v.x = fmaf(acc[2 * q4][e], inv_lam, add);
-                    v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
-                    v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
-                    v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
-                    *reinterpret_cast<float4*>(row + 4 * q4) = v;
+                for (int mt = 0; mt < 8; ++mt) {   // m-tile rows g, g + 8: dims 16 mt + g, 16 mt + g + 8
+                    row[16 * mt + g] = fmaf(acc[mt][e], inv_lam, add);
+                    row[16 * mt + g + 8] = fmaf(acc[mt][e + 2], inv_lam, add);
                 }
                 if (g == 0) {
                     wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
