@@ -46,6 +46,22 @@ __device__ __forceinline__ uint32_t nh8(uint32_t x, uint32_t sel) { return prmt(
 // h' pair (fp16) for two 10-bit dithers in the low bits of each 16-bit lane.
 __device__ __forceinline__ uint32_t h10(uint32_t x) { return (x & 0x03FF03FFu) | 0x3C003C00u; }
 
+// Upward margin on the merged e-form accumulator D = E_p~[e^c - 1] (and the
+// Tier-B one) before the meter (A^2 - 1)/2 = D (D + 2)/2 is formed, so the
+// fp32 meter lands on or above the exact value of §3 Thm. "Sound replacement"
+// instead of within rounding either side of it.  It covers:
+//  - ex2.approx near 1 (relative error below 2^-22 of 2^c, i.e. an absolute
+//    error below 2^-22 in each e^c - 1 and so in their p~-weighted mean): kDAbs;
+//  - the fp32 sums of p~ and p~ (e^c - 1) (per lane about a thousand terms
+//    at 32k tokens, then the warp, CTA and split merges: n u < 2^-13), the
+//    hi + lo fp16 bound operand (2^-22) and the rounding of the logits that
+//    move p~ (their effect on D, measured against the fp64 oracle, stays near
+//    10^-5 relative): kDRel, at about 4x the larger of these.
+// At 1 + 2^-12 it stays well inside the 1e-3 relative parity tolerance.
+constexpr float kDRel = 1.0f + 0x1p-12f;
+constexpr float kDAbs = 0x1p-21f;
+__device__ __forceinline__ float d_upper(float d) { return fmaf(d, kDRel, kDAbs); }
+
 // 2^n for -126 <= n <= 127.
 __device__ __forceinline__ float pow2(int n) { return __int_as_float((127 + n) << 23); }
 

@@ -1293,7 +1293,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
         if (chunk == 0 && lane == 0) {
             float raw = 0.f;
             if (l > 0.f) {
-                const float D = dn / l;                 // A - 1
+                const float D = d_upper(dn / l);        // A - 1, rounded up
                 raw = 0.5f * D * (D + 2.0f);            // (A^2 - 1) / 2, +inf on overflow
             }
             p.meter_raw[cell] = raw;
@@ -1302,14 +1302,14 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             if (tier_b) {
                 float rb = 0.f;
                 if (l > 0.f) {
-                    const float D = db / l;
+                    const float D = d_upper(db / l);
                     rb = 0.5f * D * (D + 2.0f);
                 }
                 p.meter_b_raw[cell] = rb;
                 p.meter_b[cell] = fminf(1.0f, rb);
             }
             if (vside) {   // ||y - y^|| <= 2 TV max ||v|| + sum p~ rho^v, TV <= meter
-                const float vterm = l > 0.f ? vt / l : 0.f;
+                const float vterm = l > 0.f ? vt / l * kDRel : 0.f;   // rounded up like D
                 p.value_term[cell] = vterm;
                 p.v_max[cell] = vm;
                 p.out_bound[cell] = 2.0f * fminf(1.0f, raw) * vm + vterm;
@@ -1472,7 +1472,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_flat_kernel(const __gr
     if (chunk == 0 && lane == 0) {
         float raw = 0.f;
         if (L > 0.f) {
-            const float D = Dn / L;
+            const float D = d_upper(Dn / L);
             raw = 0.5f * D * (D + 2.0f);
         }
         p.meter_raw[cell] = raw;
@@ -1481,14 +1481,14 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_flat_kernel(const __gr
         if (tier_b) {
             float rb = 0.f;
             if (L > 0.f) {
-                const float D = Db / L;
+                const float D = d_upper(Db / L);
                 rb = 0.5f * D * (D + 2.0f);
             }
             p.meter_b_raw[cell] = rb;
             p.meter_b[cell] = fminf(1.0f, rb);
         }
         if (vside) {
-            const float vterm = L > 0.f ? Vt / L : 0.f;
+            const float vterm = L > 0.f ? Vt / L * kDRel : 0.f;
             p.value_term[cell] = vterm;
             p.v_max[cell] = Vm;
             p.out_bound[cell] = 2.0f * fminf(1.0f, raw) * Vm + vterm;

@@ -37,6 +37,24 @@ def assert_close(gpu, ref, what, rtol=RTOL, atol=ATOL):
                              f"gpu={g[tuple(idx.T)]} ref={r[tuple(idx.T)]}")
 
 
+def assert_sound(gpu, ref, tv, what):
+    """One-sided soundness of a GPU meter (§3 Thm. "Sound replacement"): on or
+    above the oracle's fp64 meter and the true TV, per cell, with no slack."""
+    g = np.asarray(gpu, np.float64)
+    below = g < np.asarray(ref, np.float64)
+    assert not np.any(below), f"{what}: {int(below.sum())} cells below the oracle's fp64 meter"
+    if tv is not None:
+        under = g < np.asarray(tv, np.float64)
+        assert not np.any(under), f"{what}: {int(under.sum())} cells below the true TV"
+
+
+def witness_step_up(w):
+    """Every stored fp16 witness one fp16 step up (0 to the least subnormal):
+    the largest value the GPU write may store for it."""
+    w = np.asarray(w, dtype=np.float16)
+    return (w.view(np.uint16) + 1).view(np.float16)
+
+
 def descs(n_q, n_kv, num_pages, scheme=0, bits=8, layout=0, seed=0, num_bypass_pairs=0):
     import paper_2607_28699_gb300 as wc
     o = OP.Desc(num_q_heads=n_q, num_kv_heads=n_kv, num_pages=num_pages, scheme=scheme,

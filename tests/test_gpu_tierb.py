@@ -8,7 +8,7 @@ import torch
 
 import workloads as W
 from oracle import pipeline as OP
-from tests._parity import assert_close, descs, make_inputs
+from tests._parity import assert_close, assert_sound, descs, make_inputs
 
 pytestmark = pytest.mark.gpu
 
@@ -35,6 +35,7 @@ def _run(wl, bits=8, layout=0, layer=0, seed=1, delta=1e-6):
         r = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, delta_loc=delta)
         mb.append(r["meter_b"]); mbr.append(r["meter_b_raw"])
     assert_close(res_b[4].cpu().numpy(), np.stack(mbr), "meter_b_raw")
+    assert_sound(res_b[4].cpu().numpy(), np.stack(mbr), None, "meter_b_raw")
     assert_close(res_b[3].cpu().numpy(), np.stack(mb), "meter_b")
 
 
