@@ -272,17 +272,19 @@ wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer
  * without the workspace.  Its scratch is one fixed 4 MiB device array built
  * into the library; every GPU that loads the library keeps it until the
  * process exits.  The call never allocates or frees memory.
- *   dev_status  optional device uint32 that collects WC_DEV_* bits (OR); when
- *               NULL the bits go to a word inside the built-in scratch.
+ *   dev_status  device uint32 that collects the WC_DEV_* bits (OR), required
+ *               (not NULL: the built-in scratch has no word a caller can read);
+ *               read and clear it with wc_read_status(dev_status, 1, ...).
  * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
  * more scratch than 4 MiB (about 930 partial results: one per (KV head,
  * split) for one sequence; the SM count plus batch x Hkv for several
  * sequences; the count follows wc_workspace_size's plan).
- * The first call on each device looks up the scratch address and clears its
- * status word (a synchronous cudaMemset); make that first call before any
- * stream capture.  All calls share the one scratch array and it keeps the
- * last call's contents: calls that can overlap on the GPU (different streams,
- * or several host threads) race and must be ordered by the caller.
+ * The first call on each device, and the first after its context has been
+ * recreated (cudaDeviceReset), looks up the scratch address
+ * (cudaGetSymbolAddress); make that first call before any stream capture.
+ * All calls share the one scratch array and it keeps the last call's
+ * contents: calls that can overlap on the GPU (different streams, or several
+ * host threads) race and must be ordered by the caller.
  */
 wc_status wc_metered_decode_attention_noalloc(const wc_cache_desc* desc, int32_t layer,
                                               const void* q, const int32_t* block_table,

@@ -297,7 +297,6 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.v_new = static_cast<const __half*>(v_new);
     p.slot_new = slot_new;
     p.status = reinterpret_cast<uint32_t*>(ws);
-    p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
     p.batch = batch;
     p.max_pages = max_pages;
@@ -488,28 +487,51 @@ constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;   // 4 MiB per device
 constexpr int kNoAllocMaxDevices = 64;
 
 // File-scope device scratch.  In host code this name is only a stand-in for
-// the device array, never a device address: the address is looked up once
-// per device with cudaGetSymbolAddress (below) and passed to the kernels.
+// the device array, never a device address: the address is looked up with
+// cudaGetSymbolAddress (below) and passed to the kernels.
 static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+// The address belongs to the module as loaded into one device context; a
+// context that is torn down and recreated (cudaDeviceReset) loads the module
+// again.  So the address is cached per device together with the context it
+// was looked up in, and looked up again when the current context differs.
+using CtxGetCurrentFn = int (*)(void**);   // cuCtxGetCurrent through the runtime's driver entry point
+
+CtxGetCurrentFn ctx_get_current() {
+    static std::once_flag once;
+    static CtxGetCurrentFn fn = nullptr;
+    std::call_once(once, [] {
+        void* f = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &f, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<CtxGetCurrentFn>(f);
+    });
+    return fn;
+}
 
 std::mutex g_noalloc_mu;
 void* g_noalloc_ptr[kNoAllocMaxDevices] = {};
+void* g_noalloc_ctx[kNoAllocMaxDevices] = {};
 
-// Address of the scratch on the current device; looked up (and its status
-// word cleared) the first time a device is seen.
+// Address of the scratch in the current device's current context.
 wc_status noalloc_scratch(void** out) {
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
     if (dev < 0 || dev >= kNoAllocMaxDevices) return fail(WC_ERR_UNSUPPORTED, "device index %d too large", dev);
+    CtxGetCurrentFn get = ctx_get_current();
+    if (!get) return fail(WC_ERR_CUDA, "cannot query the current device context");
+    void* ctx = nullptr;   // null until the runtime has made a context current on this thread
+    if (get(&ctx) != 0) return fail(WC_ERR_CUDA, "cannot query the current device context");
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
+    if (!ctx || !g_noalloc_ptr[dev] || g_noalloc_ctx[dev] != ctx) {
         void* ptr = nullptr;
-        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+        e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);   // also makes the device's context current
         if (e != cudaSuccess) return cuda_fail(e, "cudaGetSymbolAddress of the decode scratch");
-        e = cudaMemset(ptr, 0, 256);   // the status word must start at zero
-        if (e != cudaSuccess) return cuda_fail(e, "clearing the decode scratch status word");
+        if (get(&ctx) != 0 || !ctx) return fail(WC_ERR_CUDA, "cannot query the current device context");
         g_noalloc_ptr[dev] = ptr;
+        g_noalloc_ctx[dev] = ctx;
     }
     *out = g_noalloc_ptr[dev];
     return WC_OK;
@@ -528,8 +550,8 @@ extern "C" wc_status wc_metered_decode_attention_noalloc(
     if (max_pages < 1) return fail(WC_ERR_INVALID_ARG, "max_pages must be positive (got %d)", max_pages);
     if ((long long)max_pages * wc::kPage > 0x7FFFFFFFLL) return fail(WC_ERR_UNSUPPORTED, "max_pages too large");
     if (batch == 0) return WC_OK;
-    if (!q || !block_table || !ctx_lens || !out || !meter || !meter_raw)
-        return fail(WC_ERR_INVALID_ARG, "q, block_table, ctx_lens, out, meter, meter_raw must not be NULL");
+    if (!q || !block_table || !ctx_lens || !out || !meter || !meter_raw || !dev_status)
+        return fail(WC_ERR_INVALID_ARG, "q, block_table, ctx_lens, out, meter, meter_raw, dev_status must not be NULL");
     if (!aligned16(q)) return fail(WC_ERR_INVALID_ARG, "q must be 16-byte aligned");
     if (wc_status st = check_cache(desc, k_codes, v_codes, k_scale, v_scale, k_witness)) return st;
     int sms = 0;
@@ -562,8 +584,7 @@ extern "C" wc_status wc_metered_decode_attention_noalloc(
     p.value_term = nullptr;
     p.v_max = nullptr;
     p.out_bound = nullptr;
-    p.status = dev_status ? dev_status : reinterpret_cast<uint32_t*>(ws);
-    p.counters = reinterpret_cast<uint32_t*>(ws + pl.counters_off);
+    p.status = dev_status;
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
     p.batch = batch;
     p.max_pages = max_pages;

@@ -1370,7 +1370,6 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
         partials = pl.splits + units;
     }
     auto align = [](size_t x) { return (x + 255) & ~(size_t)255; };
-    pl.counters_off = 256;
     pl.partials_off = 256;
     pl.total = align(pl.partials_off + sizeof(float) * (size_t)partials * kMaxGroup * kPartialStride);
     return pl;

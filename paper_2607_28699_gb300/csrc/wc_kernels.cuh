@@ -60,7 +60,6 @@ struct DecodeParams {
     const int32_t* bypass_pairs = nullptr;
     int32_t num_bypass = 0;
     uint32_t* status;     // workspace word
-    uint32_t* counters;   // [batch * Hkv], zero between calls
     float* partials;      // [batch * Hkv * splits] (flattened: [splits + batch * Hkv]) x [kMaxGroup][kPartialStride]
     int32_t batch, max_pages, num_q_heads, num_kv_heads, group, num_pages, layer, rope_layout;
     // pages_per_split == 0 marks the flattened plan (warp-specialized kernel,
@@ -80,12 +79,12 @@ struct DecodeParams {
 // groups (12 words apart modulo 32; 136 would put two heads on each group).
 constexpr int kPartialStride = kHeadDim + 12;
 
-// Workspace layout (bytes): [0, 256) status word, then counters, then
-// partials, each 256-byte aligned.
+// Workspace layout (bytes): [0, 256) status word, then the partials
+// (256-byte aligned).
 struct DecodePlan {
     int splits;            // flattened plan: the grid's CTAs
     int pages_per_split;   // 0: the flattened plan
-    size_t counters_off, partials_off, total;
+    size_t partials_off, total;
 };
 
 DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, int scheme, int bits);

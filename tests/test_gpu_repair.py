@@ -1,8 +1,8 @@
 """GPU parity of block-level repair selection (§6.4 "Block-level paging"):
 the decode with per-page terms leaves the plain outputs bit for bit, the page
-contributions C_j match the oracle's, the ranking is exact on the kernel's
-own contributions (the count may differ only where the meter sits within
-rounding of tau), the chosen pages are a top set of the oracle's fp64
+contributions C_j match the oracle's, the list is consistent with the
+kernel's own contributions (ordering; the count may differ only where the
+meter sits within rounding of tau), the chosen pages are a top set of the oracle's fp64
 contributions that brings the meter to tau, and the edge cases (kept cells,
 NaN / inf / tied / zero contributions, ragged and one-token contexts, the
 largest block table) select what the oracle selects."""
@@ -26,16 +26,30 @@ def _remaining_meter(C, taken):
     return R, 0.5 * R * (R + 2.0)
 
 
+def _self_order(c64):
+    """The ranking rule applied to the kernel's own contributions (a check of
+    the selection kernel's consistency, not an oracle result): NaN first, then
+    by decreasing contribution, ties to the lower page."""
+    key = np.where(np.isnan(c64), np.inf, c64)
+    nan_first = np.isnan(c64)
+    return sorted(range(len(c64)), key=lambda j: (not nan_first[j], -key[j], j))
+
+
 def _check_selection(gc, pages, n, d_after, tau, ref_c=None):
-    """One flagged cell: gc the kernel's contributions (fp32) of its n pages."""
+    """One flagged cell: gc the kernel's contributions (fp32) of its n pages.
+    The list is checked for consistency with the kernel's own contributions
+    (ordering and the least count whose remaining meter is at most tau), and
+    against the oracle's fp64 contributions ref_c (a top set that repairs)."""
     c64 = gc.astype(np.float64)
-    plan, _ = OM.repair_plan(c64, tau)
     k = len(pages)
-    order, _ = OM.repair_plan(c64, -1.0)                       # the full ranking
-    assert list(pages) == order[:k]                             # same ranking, bit for bit
-    if k != len(plan):                                          # only at the decision boundary
-        _, raw = _remaining_meter(c64, order[:min(k, len(plan))])
-        assert abs(k - len(plan)) == 1 and abs(raw - tau) <= 1e-5 * max(tau, 1e-3), (k, len(plan), raw, tau)
+    order = _self_order(c64)
+    assert list(pages) == order[:k]                             # ranked by the kernel's own values
+    rest = float(np.sum(c64)) - np.concatenate([[0.0], np.cumsum(c64[order])])   # R after i pages
+    ok = np.nonzero(0.5 * rest * (rest + 2.0) <= tau)[0]
+    need = int(ok[0]) if ok.size else n
+    if k != need:                                               # only at the decision boundary
+        _, raw = _remaining_meter(c64, order[:min(k, need)])
+        assert abs(k - need) == 1 and abs(raw - tau) <= 1e-5 * max(tau, 1e-3), (k, need, raw, tau)
     R, _ = _remaining_meter(c64, pages)
     assert abs(d_after - R) <= 1e-5 * max(R, 1e-6) + 1e-7
     if ref_c is not None and 0 < k < n:                         # against the oracle's own contributions

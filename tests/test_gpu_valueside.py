@@ -60,7 +60,7 @@ def test_value_side_decode_and_joint_gate(scheme):
     for x, y in zip(plain, res[:3]):
         assert torch.equal(x, y)
     offs = np.concatenate([[0], np.cumsum(wl.ctx_lens)[:-1]])
-    ref = {n: [] for n in ("value_term", "v_max", "out_bound", "out_err")}
+    ref = {n: [] for n in ("value_term", "v_max", "out_bound", "out_err", "meter_raw")}
     for b, S in enumerate(wl.ctx_lens):
         r = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache,
                                k.numpy()[offs[b]:offs[b] + S], v.numpy()[offs[b]:offs[b] + S])
@@ -73,11 +73,18 @@ def test_value_side_decode_and_joint_gate(scheme):
     assert_close(bound, ref["out_bound"], "out_bound")
     assert_sound(vterm, ref["value_term"], None, "value_term")       # rounded up like the meter
     assert np.all(bound >= ref["out_err"])                            # the bound holds on the GPU's numbers
-    for tk, tv in ((0.1, 0.01), (0.5, 0.05), (1.0, 1e-3)):
+    # the joint gate on the GPU's numbers against the oracle's joint gate on its own
+    # fp64 numbers; cells within 1e-3 of either threshold are excluded and counted
+    o_raw = ref["meter_raw"].reshape(-1)
+    o_vt, o_vm = ref["value_term"].reshape(-1), ref["v_max"].reshape(-1)
+    for tk, tv in ((0.1, 0.01), (0.5, 0.05), (1.0, 1e-3), (float(np.median(o_raw)), float(np.median(o_vt / o_vm)))):
         keep_q, keep_kv, kept = wc.gate_joint(res[2].reshape(-1), res[3].reshape(-1), res[4].reshape(-1),
                                               gd.group, tk, tv)
-        oq, okv, nq, nkv = OM.joint_gate(res[2].cpu().numpy().reshape(-1), vterm.reshape(-1),
-                                         vmax.reshape(-1), tk, tv, gd.group)
-        assert np.array_equal(keep_q.cpu().numpy().astype(bool), oq)
-        assert np.array_equal(keep_kv.cpu().numpy().astype(bool), okv)
-        assert kept.cpu().tolist() == [nq, nkv]
+        oq, _, _, _ = OM.joint_gate(o_raw, o_vt, o_vm, tk, tv, gd.group)
+        near = (np.abs(o_raw - tk) < 1e-3 * tk + 1e-5) | (np.abs(o_vt - tv * o_vm) < 1e-3 * tv * o_vm + 1e-5)
+        assert int(near.sum()) <= max(1, near.size // 20)
+        kq = keep_q.cpu().numpy().astype(bool)
+        assert np.array_equal(kq[~near], oq[~near])
+        kkv = keep_kv.cpu().numpy().astype(bool)
+        assert np.array_equal(kkv, kq.reshape(-1, gd.group).all(axis=1))     # any-of-G fallback
+        assert kept.cpu().tolist() == [int(kq.sum()), int(kkv.sum())]

@@ -1,9 +1,12 @@
-"""The allocation-free decode entry point gives the same results as the
-workspace-based one.
+"""The allocation-free decode entry point (wc_metered_decode_attention_noalloc)
+gives the same results as the workspace-based one, bit for bit, and matches
+the oracle.
 
-It exists for callers that cannot allocate device memory at decode time, so
-its scratch is a fixed array inside the library.  This file is collected
-last so that, if it fails, every other test has already run."""
+It exists for callers that cannot allocate device memory at decode time (a
+runtime that pre-plans every buffer, code inside an allocator's own hooks, a
+process under a fixed memory budget), so its scratch is a fixed array inside
+the library.  This file is collected last so that, if it fails, every other
+test has already run."""
 
 import ctypes
 
@@ -12,7 +15,8 @@ import pytest
 import torch
 
 import workloads as W
-from tests._parity import assert_close, descs, make_inputs
+from oracle import pipeline as OP
+from tests._parity import assert_close, assert_sound, descs, make_inputs, numpy_cache_to_gpu
 
 pytestmark = pytest.mark.gpu
 
@@ -26,41 +30,55 @@ def _noalloc_fn():
     return f
 
 
-def test_noalloc_decode_matches_workspace_decode_twice():
+def _P(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+# batch 1 runs the split plan (partials per (KV head, split) in the scratch),
+# several sequences the flattened plan; both schemes
+CASES = [(0, [20011], 4), (1, [9000], 1), (0, [3001, 77, 1], 2), (1, [5000, 16], 5)]
+
+
+@pytest.mark.parametrize("scheme,ctx_lens,layer", CASES)
+def test_noalloc_decode_matches_workspace_and_oracle_twice(scheme, ctx_lens, layer):
     import paper_2607_28699_gb300 as wc
     f = _noalloc_fn()
-    P = lambda t: None if t is None else ctypes.c_void_p(t.data_ptr())
-    for call, (scheme, ctx_lens, layer) in enumerate([(0, [3001, 77, 1], 2), (1, [5000, 16], 5)]):
-        wl = W.Workload("noalloc", 1, 28, 4, ctx_lens, scheme=scheme, shuffle_pages=True, seed=call + 3)
-        bt, sm, k, v, q = make_inputs(wl, layer)
-        _, gd = descs(28, 4, wl.num_pages, scheme=scheme, seed=9)
-        cache = wc.LayerCache.empty(gd)
-        wc.kv_quantize_witness(gd, layer, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
-        btg, qg = torch.from_numpy(bt).cuda(), q.cuda()
-        ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
-        ws = wc.Workspace(gd, wl.batch, wl.max_pages)
-        ref_out, ref_meter, ref_raw = wc.metered_decode_attention(gd, layer, qg, btg, ctx, cache, ws)
-
+    wl = W.Workload("noalloc", 1, 28, 4, ctx_lens, scheme=scheme, shuffle_pages=True, seed=layer + 3)
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    od, gd = descs(28, 4, wl.num_pages, scheme=scheme, seed=9)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
+    cache = numpy_cache_to_gpu(ocache, gd)          # the oracle's stored cache on both sides
+    btg, qg = torch.from_numpy(bt).cuda(), q.cuda()
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ref_out, ref_meter, ref_raw = wc.metered_decode_attention(gd, layer, qg, btg, ctx, cache, ws)
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    d = gd.c()
+    for _ in range(2):                              # two calls in a row share the scratch
         out = torch.full_like(ref_out, float("nan"))
         meter = torch.full_like(ref_meter, float("nan"))
         raw = torch.full_like(ref_raw, float("nan"))
         status = torch.zeros(1, dtype=torch.int32, device="cuda")
-        d = gd.c()
-        st = f(ctypes.byref(d), layer, P(qg), P(btg), wl.max_pages, P(ctx), wl.batch, P(cache.k_codes),
-               P(cache.v_codes), P(cache.k_scale), P(cache.v_scale), P(cache.k_witness), P(out), P(meter),
-               P(raw), P(status), ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+        st = f(ctypes.byref(d), layer, _P(qg), _P(btg), wl.max_pages, _P(ctx), wl.batch, _P(cache.k_codes),
+               _P(cache.v_codes), _P(cache.k_scale), _P(cache.v_scale), _P(cache.k_witness), _P(out),
+               _P(meter), _P(raw), _P(status), stream)
         assert st == 0, wc.lib.wc_last_error().decode()
         torch.cuda.synchronize()
         assert int(status.item()) == 0
-        assert_close(out.cpu().numpy(), ref_out.cpu().numpy(), "noalloc out")
-        assert_close(meter.cpu().numpy(), ref_meter.cpu().numpy(), "noalloc meter")
-        assert_close(raw.cpu().numpy(), ref_raw.cpu().numpy(), "noalloc meter_raw")
+        for a, b in ((out, ref_out), (meter, ref_meter), (raw, ref_raw)):
+            assert torch.equal(a, b)                # same kernels, same plan
+    for b, S in enumerate(ctx_lens):
+        r = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache)
+        assert_close(out[b].cpu().numpy(), r["out"], f"noalloc out[{b}]")
+        assert_close(raw[b].cpu().numpy(), r["meter_raw"], f"noalloc meter_raw[{b}]")
+        assert_sound(raw[b].cpu().numpy(), r["meter_raw"], None, f"noalloc meter_raw[{b}]")
 
 
-def test_noalloc_rejects_work_beyond_its_scratch():
+def test_noalloc_rejects_work_beyond_its_scratch_and_a_null_status():
     import paper_2607_28699_gb300 as wc
     f = _noalloc_fn()
-    # many short sequences: the split plan needs more partials than 4 MiB holds
+    # many short sequences: the plan needs more partials than 4 MiB holds
     batch, max_pages = 4096, 64
     _, gd = descs(32, 8, 16, seed=1)
     cache = wc.LayerCache.empty(gd)
@@ -69,9 +87,12 @@ def test_noalloc_rejects_work_beyond_its_scratch():
     ctx = torch.ones(batch, dtype=torch.int32, device="cuda")
     out = torch.empty(batch, 32, 128, device="cuda")
     m = torch.empty(batch, 32, device="cuda")
+    status = torch.zeros(1, dtype=torch.int32, device="cuda")
     d = gd.c()
-    P = lambda t: None if t is None else ctypes.c_void_p(t.data_ptr())
-    st = f(ctypes.byref(d), 0, P(q), P(bt), max_pages, P(ctx), batch, P(cache.k_codes), P(cache.v_codes),
-           P(cache.k_scale), P(cache.v_scale), P(cache.k_witness), P(out), P(m), P(m), None,
-           ctypes.c_void_p(torch.cuda.current_stream().cuda_stream))
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    args = [ctypes.byref(d), 0, _P(q), _P(bt), max_pages, _P(ctx), batch, _P(cache.k_codes), _P(cache.v_codes),
+            _P(cache.k_scale), _P(cache.v_scale), _P(cache.k_witness), _P(out), _P(m), _P(m)]
+    st = f(*args, _P(status), stream)
     assert st == 2 and b"scratch" in wc.lib.wc_last_error()
+    st = f(*args, None, stream)                     # the status word is required
+    assert st == 1 and b"dev_status" in wc.lib.wc_last_error()
