@@ -169,9 +169,11 @@ def _pack(tensors, align=256):
 
 
 class Setup:
-    """Caches, queries and the per-step buffers of one workload on one GPU."""
+    """Caches, queries and the per-step buffers of one workload on one GPU.
+    extras: also the value-witness and grouped-scale caches of the §8(f) rows
+    (the headline workload only)."""
 
-    def __init__(self, wl, dither_bits=8):
+    def __init__(self, wl, dither_bits=8, extras=True):
         import paper_2607_28699_gb300 as wc
         self.wc, self.wl = wc, wl
         self.desc = wc.CacheDesc(num_q_heads=wl.n_q_heads, num_kv_heads=wl.n_kv_heads,
@@ -192,15 +194,16 @@ class Setup:
             cache = wc.LayerCache.empty(self.desc)
             wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, cache)   # prefill write
             self.caches.append(cache)
-            # the same cache viewed with a value witness too (value-side measurement only)
-            vc = dataclasses.replace(cache, v_witness=torch.zeros(cache.k_witness.shape[:-1] + (2,),
-                                                                  dtype=torch.float16, device="cuda"))
-            wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, vc)
-            self.vcaches.append(vc)
-            gc = wc.LayerCache.empty(self.gdesc, num_bypass_pairs=self.BYPASS_PAIRS)
-            wc.select_bypass_pairs(k, self.BYPASS_PAIRS, self.desc.rope_layout, pairs=gc.bypass_pairs)
-            wc.kv_quantize_witness(self.gdesc, layer, k, v, self.sm, gc)
-            self.gcaches.append(gc)
+            if extras:
+                # the same cache viewed with a value witness too (value-side measurement only)
+                vc = dataclasses.replace(cache, v_witness=torch.zeros(cache.k_witness.shape[:-1] + (2,),
+                                                                      dtype=torch.float16, device="cuda"))
+                wc.kv_quantize_witness(self.desc, layer, k, v, self.sm, vc)
+                self.vcaches.append(vc)
+                gc = wc.LayerCache.empty(self.gdesc, num_bypass_pairs=self.BYPASS_PAIRS)
+                wc.select_bypass_pairs(k, self.BYPASS_PAIRS, self.desc.rope_layout, pairs=gc.bypass_pairs)
+                wc.kv_quantize_witness(self.gdesc, layer, k, v, self.sm, gc)
+                self.gcaches.append(gc)
             li = torch.from_numpy(last).cuda()
             self.k_new.append(k[li].contiguous())
             self.v_new.append(v[li].contiguous())
@@ -218,18 +221,19 @@ class Setup:
         e.record()
         e.synchronize()
         self.write_call_s = s.elapsed_time(e) / 1e3 / reps
-        s.record()                                   # the same with the value witness stored too
-        for _ in range(reps):
-            wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.vcaches[-1])
-        e.record()
-        e.synchronize()
-        self.write_v_call_s = s.elapsed_time(e) / 1e3 / reps
-        s.record()                                   # the grouped cache's write
-        for _ in range(reps):
-            wc.kv_quantize_witness(self.gdesc, wl.n_layers - 1, k, v, self.sm, self.gcaches[-1])
-        e.record()
-        e.synchronize()
-        self.write_g_call_s = s.elapsed_time(e) / 1e3 / reps
+        if extras:
+            s.record()                                   # the same with the value witness stored too
+            for _ in range(reps):
+                wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.vcaches[-1])
+            e.record()
+            e.synchronize()
+            self.write_v_call_s = s.elapsed_time(e) / 1e3 / reps
+            s.record()                                   # the grouped cache's write
+            for _ in range(reps):
+                wc.kv_quantize_witness(self.gdesc, wl.n_layers - 1, k, v, self.sm, self.gcaches[-1])
+            e.record()
+            e.synchronize()
+            self.write_g_call_s = s.elapsed_time(e) / 1e3 / reps
         del k, v
         # the step's new tokens as one stacked tensor per side (one copy in the end-to-end step)
         self.k_new_all, self.v_new_all = torch.stack(self.k_new), torch.stack(self.v_new)
@@ -377,6 +381,85 @@ def capture(fn):
     return g
 
 
+def timed_graph_ms(g, steps, warmup):
+    """Average ms per replay of a captured graph (events at the graph ends)."""
+    for _ in range(warmup):
+        g.replay()
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for _ in range(steps):
+        g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    return t0.elapsed_time(t1) / steps
+
+
+def meter_off_call_ms(st, args):
+    """The headline's decode calls through the library built with the
+    certificate compiled out of the warp-specialized decode (-DWC_METER_OFF:
+    no witness copy, bound MMAs or meter accumulator), for the certificate's
+    marginal cost (§8(d) meter on / off).  Outputs go to scratch buffers."""
+    import ctypes
+    path = os.path.join(ROOT, "paper_2607_28699_gb300", "_lib", "libwitcert_meteroff.so")
+    lib = ctypes.CDLL(path)
+    vp, i32 = ctypes.c_void_p, ctypes.c_int32
+    f = lib.wc_metered_decode_attention
+    f.argtypes = [vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp, ctypes.c_size_t, vp]
+    f.restype = ctypes.c_int
+    wl, d = st.wl, st.desc.c()
+    out, meter, raw = torch.empty_like(st.out[0]), torch.empty_like(st.meter[0]), torch.empty_like(st.raw[0])
+    P = lambda t: ctypes.c_void_p(t.data_ptr())
+
+    def calls():
+        s = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+        for layer in range(wl.n_layers):
+            c = st.caches[layer]
+            r = f(ctypes.byref(d), layer, P(st.q[layer]), P(st.bt), wl.max_pages, P(st.ctx), wl.batch,
+                  P(c.k_codes), P(c.v_codes), P(c.k_scale), P(c.v_scale), P(c.k_witness), P(out), P(meter), P(raw),
+                  st.ws.ptr(), st.ws.nbytes, s)
+            if r != 0:
+                raise RuntimeError(f"meter-off decode failed: {lib.wc_last_error().decode()}")
+
+    return timed_graph_ms(capture(calls), args.steps, args.warmup) / wl.n_layers
+
+
+def measure_config(cfg, args, world):
+    """One of the other workloads, measured like the headline: the step (every
+    layer's write + metered decode, then the gate) as a graph, the decode calls
+    alone (roofline), the end-to-end step with host copies, and the prefill
+    write of one layer."""
+    wl = W.config(cfg, seed=args.seed)
+    st = Setup(wl, dither_bits=8, extras=False)
+    peak = (_peaks() or {}).get("hbm_gbs", 6800.0)
+    step_ms = timed_graph_ms(capture(st.step), args.steps, args.warmup)
+    dec_ms = timed_graph_ms(capture(st.decode_all), args.steps, args.warmup) / wl.n_layers
+    status = st.wc.read_status(st.ws)
+    e2e = run_e2e(st, args, world)
+    algo = st.decode_bytes_per_launch()
+    write_th = sum(wl.ctx_lens) * wl.n_kv_heads
+    kept = st.n_kept.cpu().tolist()
+    ncell = wl.n_layers * wl.batch * wl.n_q_heads
+    gate = {"tau": st.tau, "kept_q_frac": kept[0] / ncell}
+    if len(wl.taus) > 1:   # the sweep of taus on the step's meters (risk-ranked gating, §4.3)
+        raw = st.raw.reshape(-1)
+        gate["kept_q_frac_by_tau"] = {str(t): float((raw <= t).float().mean()) for t in wl.taus}
+    res = {"workload": wl.name, "layers": wl.n_layers, "batch": wl.batch, "ctx_tokens": sum(wl.ctx_lens),
+           "scheme": "dither-int8" if wl.scheme == 0 else "fp8-e4m3",
+           "step": "write of each new token fused into its decode" if st.fused_append else "write kernel, then decode",
+           "ms_per_step": step_ms, "kv_tokens_per_s": wl.kv_tokens / (step_ms / 1e3),
+           "decode_call_ms": dec_ms, "decode_gbs": algo / (dec_ms / 1e3) / 1e9,
+           "frac": algo / (dec_ms / 1e3) / 1e9 / peak, "algorithmic_bytes_per_call": algo,
+           "traffic": _traffic(wl.name),
+           "e2e": e2e,
+           "witness_write_gbs": write_th * WRITE_BYTES_PER_TOKEN_HEAD[wl.scheme] / st.write_call_s / 1e9,
+           "gate": gate, "device_status": status,
+           "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step vs 129 MB L2; no flush"}
+    del st
+    torch.cuda.empty_cache()
+    return res
+
+
 def run_ours(args, rank, world, local):
     wl = rank_workload(args.config, args.seed, rank)
     if args.layers:
@@ -416,6 +499,14 @@ def run_ours(args, rank, world, local):
     d1.record()
     torch.cuda.synchronize()
     dec_avg_ms = d0.elapsed_time(d1) / (args.steps * wl.n_layers)
+
+    # ---- the certificate's marginal cost: the same calls with it compiled out ----
+    meter_off = None
+    if wl.scheme == 0 and args.dither_bits == 8:
+        off_ms = meter_off_call_ms(st, args)
+        meter_off = {"decode_call_ms_meter_on": dec_avg_ms, "decode_call_ms_meter_off": off_ms,
+                     "certificate_cost": dec_avg_ms / off_ms - 1.0,
+                     "build": "libwitcert_meteroff.so (-DWC_METER_OFF): no witness copy, bound MMAs or meter sums"}
 
     # ---- the same calls with the value side too (its marginal cost) ----
     vgraph = capture(st.decode_all_value)
@@ -532,6 +623,7 @@ def run_ours(args, rank, world, local):
                    "l2": f"inputs {st.caches[0].nbytes() * wl.n_layers / 1e9:.2f} GB per step > 129 MB L2; no flush"},
         "hbm_gbs_step": step_gbs,
         "decode_call_ms": dec_avg_ms,
+        "meter_off": meter_off,
         "tier_b": tier_b,
         "value_side": value_side,
         "repair": repair,
@@ -553,6 +645,11 @@ def run_ours(args, rank, world, local):
         "clocks": clk.summary(),
         "e2e": e2e,
     }
+    if world == 1 and not args.no_configs:
+        # the other workloads, each at its full size on this GPU (not in the headline value)
+        st = graph = dgraph = vgraph = bgraph = None   # free the headline's caches and graphs first
+        torch.cuda.empty_cache()
+        res["configs"] = {f"config{c}": measure_config(c, args, world) for c in range(1, 6) if c != args.config}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         res["cpu_baseline"] = cpu_baseline(wl, args)
     return res
@@ -697,6 +794,7 @@ def main():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-configs", action="store_true", help="skip the other workloads' measurements")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
