@@ -474,6 +474,29 @@ wc_status wc_gate_joint(const float* meter_raw, const float* value_term, const f
 wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word,
                          uint32_t* bits, void* stream);
 
+/*
+ * Failure-detection test support (no counterpart in the paper; the library's
+ * own test of its bounded waits).  Runs wc_metered_decode_attention for one
+ * sequence (batch 1, dithered INT8 cache with the 8-bit dither) except that
+ * the copies of logical page `stall_page` are never issued: the consumer that
+ * waits for that page, and then its producer, give up after a short bounded
+ * wait (64 tries of mbarrier.try_wait), set WC_DEV_TIMEOUT in the workspace's
+ * status word and finish; copies already issued are waited for before the
+ * kernel exits.  Nothing faults or hangs, and the context stays usable: read
+ * the bits with wc_read_status.  The outputs of the call are not meaningful.
+ *   stall_page  in [0, max_pages), else WC_ERR_INVALID_ARG
+ * Other arguments as wc_metered_decode_attention (ctx_lens holds one length).
+ */
+wc_status wc_testing_decode_stalled_page(const wc_cache_desc* desc, int32_t layer,
+                                         const void* q, const int32_t* block_table,
+                                         int32_t max_pages, const int32_t* ctx_lens,
+                                         const void* k_codes, const void* v_codes,
+                                         const void* k_scale, const void* v_scale,
+                                         const void* k_witness,
+                                         float* out, float* meter, float* meter_raw,
+                                         void* workspace, size_t workspace_bytes,
+                                         int32_t stall_page, void* stream);
+
 /* Thread-local description of the last non-OK status on this thread. */
 const char* wc_last_error(void);
 

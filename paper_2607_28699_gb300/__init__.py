@@ -36,7 +36,7 @@ EXPORTS = ("wc_kv_quantize_witness", "wc_workspace_size", "wc_metered_decode_att
            "wc_kv_quantize_witness_v", "wc_metered_decode_attention_v", "wc_gate_joint",
            "wc_metered_decode_attention_repair", "wc_repair_select",
            "wc_kv_quantize_witness_g32", "wc_metered_decode_attention_g32", "wc_select_bypass_pairs",
-           "wc_metered_decode_attention_append",
+           "wc_metered_decode_attention_append", "wc_testing_decode_stalled_page",
            "wc_gate", "wc_read_status", "wc_last_error", "wc_version")
 
 
@@ -63,6 +63,9 @@ def _load():
                                                        ctypes.c_double, vp, vp, vp, vp, vp, vp, ctypes.c_size_t,
                                                        vp]
     lib.wc_metered_decode_attention_tier_b.restype = ctypes.c_int
+    lib.wc_testing_decode_stalled_page.argtypes = [vp, i32, vp, vp, i32, vp, vp, vp, vp, vp, vp, vp, vp, vp,
+                                                   vp, ctypes.c_size_t, i32, vp]
+    lib.wc_testing_decode_stalled_page.restype = ctypes.c_int
     lib.wc_gate.argtypes = [vp, i32, i32, ctypes.c_float, vp, vp, vp, vp]
     lib.wc_gate.restype = ctypes.c_int
     lib.wc_gate_joint.argtypes = [vp, vp, vp, i32, i32, ctypes.c_float, ctypes.c_float, vp, vp, vp, vp]

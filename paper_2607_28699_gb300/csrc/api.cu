@@ -213,7 +213,7 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
                                        void* stream, bool grouped = false, const void* k_bypass = nullptr,
                                        const int32_t* bypass_pairs = nullptr, int32_t num_bypass = 0,
                                        const void* k_new = nullptr, const void* v_new = nullptr,
-                                       const int32_t* slot_new = nullptr) {
+                                       const int32_t* slot_new = nullptr, int32_t stall_page = -1) {
     if (wc_status st = check_desc(desc, grouped)) return st;
     if (k_new || v_new || slot_new) {
         if (!k_new || !v_new || !slot_new)
@@ -296,6 +296,7 @@ static wc_status decode_with_workspace(const wc_cache_desc* desc, int32_t layer,
     p.k_new = static_cast<const __half*>(k_new);
     p.v_new = static_cast<const __half*>(v_new);
     p.slot_new = slot_new;
+    p.stall_page = stall_page;
     p.status = reinterpret_cast<uint32_t*>(ws);
     p.partials = reinterpret_cast<float*>(ws + pl.partials_off);
     p.batch = batch;
@@ -322,6 +323,23 @@ wc_status wc_metered_decode_attention(const wc_cache_desc* desc, int32_t layer, 
     return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, batch, k_codes, v_codes, k_scale,
                                  v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
                                  nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream);
+}
+
+wc_status wc_testing_decode_stalled_page(const wc_cache_desc* desc, int32_t layer, const void* q,
+                                        const int32_t* block_table, int32_t max_pages, const int32_t* ctx_lens,
+                                        const void* k_codes, const void* v_codes, const void* k_scale,
+                                        const void* v_scale, const void* k_witness, float* out, float* meter,
+                                        float* meter_raw, void* workspace, size_t workspace_bytes,
+                                        int32_t stall_page, void* stream) {
+    if (wc_status st = check_desc(desc)) return st;
+    if (desc->scheme != WC_SCHEME_DITHER_INT8 || desc->dither_bits != 8)
+        return fail(WC_ERR_UNSUPPORTED, "the stalled-page test runs the dithered INT8 cache with the 8-bit dither");
+    if (stall_page < 0 || stall_page >= max_pages)
+        return fail(WC_ERR_INVALID_ARG, "stall_page must be in [0, max_pages) (got %d)", stall_page);
+    return decode_with_workspace(desc, layer, q, block_table, max_pages, ctx_lens, 1, k_codes, v_codes, k_scale,
+                                 v_scale, k_witness, out, meter, meter_raw, nullptr, nullptr, 0.0, nullptr, nullptr,
+                                 nullptr, nullptr, nullptr, nullptr, workspace, workspace_bytes, stream, false, nullptr,
+                                 nullptr, 0, nullptr, nullptr, nullptr, stall_page);
 }
 
 wc_status wc_metered_decode_attention_tier_b(const wc_cache_desc* desc, int32_t layer, const void* q,

@@ -18,6 +18,10 @@ constexpr int kXValue = 2;   // value-side witness terms and output bound (§3, 
 constexpr int kXRepair = 4;  // per-page meter terms for block-level repair selection (§6.4)
 constexpr int kXAppend = 8;  // the decode writes the step's new token before reading it
 constexpr int kXFlat = 16;   // warp-specialized kernel under the flattened split plan
+// failure-detection test (warp-specialized kernel, split plan): one page's
+// copies are never issued and every wait gives up after kStallTries tries
+constexpr int kXStall = 32;
+constexpr int kStallTries = 64;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRsd = 0.08838834764831845f;                      // 1/sqrt(128)
 constexpr float kRsdLog2e = 0.08838834764831845f * 1.4426950408889634f;

@@ -685,6 +685,8 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
     constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
     constexpr bool kAppend = (kX & kXAppend) != 0;
     constexpr bool kFlat = (kX & kXFlat) != 0;   // flattened split plan (pages_per_split == 0)
+    constexpr bool kStall = (kX & kXStall) != 0;
+    constexpr int kTries = kStall ? kStallTries : kMaxWaitTries;
     const DecodeParams& p = wp.p;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
@@ -775,7 +777,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const int lp = first + kWsPairs * i;
                 const int s = k % kWsStages;
                 if (k >= kWsStages) {
-                    const bool freed = mbar_wait_bounded(&empty[s], (uint32_t)(((k / kWsStages) - 1) & 1));
+                    const bool freed = mbar_wait_bounded<kTries>(&empty[s], (uint32_t)(((k / kWsStages) - 1) & 1));
                     if (!__all_sync(0xffffffffu, freed)) {
                         if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
                         stop = true;
@@ -788,6 +790,12 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 uint8_t* st = stages + s * kWsStageBytes;
                 if constexpr (kAppend) {   // the sequence's last page: store the new token first
                     if (ok && lp == npages - 1) append_new_token(wp, b, h, phys, ctx, lane);
+                }
+                if constexpr (kStall) {   // failure-detection test: this page is never staged
+                    if (lp == p.stall_page) {
+                        issued = k + 1;
+                        continue;
+                    }
                 }
                 if (lane == 0) {
                     *reinterpret_cast<int*>(st + kWsOffHdr) = ok ? phys : -1;
@@ -842,7 +850,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         }
         // copies still in flight must land before the CTA's smem is released
         for (int j = max(0, issued - kWsStages); j < issued; ++j)
-            (void)mbar_wait_bounded(&full[j % kWsStages], (uint32_t)((j / kWsStages) & 1));
+            (void)mbar_wait_bounded<kTries>(&full[j % kWsStages], (uint32_t)((j / kWsStages) & 1));
         return;
     }
 
@@ -922,7 +930,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
         const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);
         for (int i = 0; i < n_seg && !failed; ++i, ++k) {
             const int s = k % kWsStages;
-            const bool landed = mbar_wait_bounded(&full[s], (uint32_t)((k / kWsStages) & 1));
+            const bool landed = mbar_wait_bounded<kTries>(&full[s], (uint32_t)((k / kWsStages) & 1));
             if (!__all_sync(0xffffffffu, landed)) {
                 if (lane == 0) atomicOr(p.status, WC_DEV_TIMEOUT);
                 failed = true;   // later pages are not waited for; the merges still run
@@ -1632,7 +1640,7 @@ static cudaError_t launch_ws(const DecodeParams& p, cudaStream_t stream) {
     const dim3 grid = flat ? dim3(p.splits, 1, 1) : dim3(p.splits, p.num_kv_heads, p.batch);
     cudaError_t e = launch_pdl(decode_ws_kernel<kX>, grid, dim3(kWsThreads), flat ? kWsSmemFlat : kWsSmemBytes, stream, wp);
     if (e != cudaSuccess) return e;
-    return launch_merge<kX & ~(kXAppend | kXFlat)>(p, stream);
+    return launch_merge<kX & ~(kXAppend | kXFlat | kXStall)>(p, stream);
 }
 
 template <int kF>
@@ -1654,6 +1662,9 @@ cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStrea
         return x == kXValue  ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
              : x == kXRepair ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXRepair>(p, stream)
                              : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
+    if (p.stall_page >= 0)   // failure-detection test (checked by the caller: 8-bit dither, no extras)
+        return use_ws(scheme, bits) && p.pages_per_split > 0 && x == 0 ? launch_ws<kXStall>(p, stream)
+                                                                        : cudaErrorNotSupported;
     if (use_ws(scheme, bits))   // pages_per_split == 0: the flattened plan
         return p.pages_per_split == 0 ? launch_ws_x<kXFlat>(p, x, stream) : launch_ws_x<0>(p, x, stream);
     return x == kXTierB  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)

@@ -159,8 +159,9 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 // kMaxWaitTries bounds the wait to a few seconds before giving up.
 constexpr int kMaxWaitTries = 4000;
 
+template <int kTries = kMaxWaitTries>
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity) {
-    for (int i = 0; i < kMaxWaitTries; ++i)
+    for (int i = 0; i < kTries; ++i)
         if (mbar_try_wait(bar, parity)) return true;
     return false;
 }

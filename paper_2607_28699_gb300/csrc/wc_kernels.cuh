@@ -59,6 +59,9 @@ struct DecodeParams {
     const __half* k_bypass = nullptr;
     const int32_t* bypass_pairs = nullptr;
     int32_t num_bypass = 0;
+    // failure-detection test only (wc_testing_decode_stalled_page): the logical
+    // page whose copies are never issued, so that the bounded waits run out; -1: none
+    int32_t stall_page = -1;
     uint32_t* status;     // workspace word
     float* partials;      // [batch * Hkv * splits] (flattened: [splits + batch * Hkv]) x [kMaxGroup][kPartialStride]
     int32_t batch, max_pages, num_q_heads, num_kv_heads, group, num_pages, layer, rope_layout;
