@@ -296,9 +296,9 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
             band_a = part[0] + part[1];
             band_b = part[2] + part[3];
         }
-        uint32_t a_hi = 0, a_lo = 0;   // B operand of the bound: a[head g][bands 2c, 2c+1]
+        uint32_t a_hi = 0, a_lo = 0;   // B operand of the bound: a[head g][bands 2c, 2c+1], log2 units
         if (row_valid) {
-            const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
+            const float x0 = sqrtf(band_a) * kRsdLog2e, x1 = sqrtf(band_b) * kRsdLog2e;
             const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
             a_hi = pack_h2(__half2float(h0), __half2float(h1));
             a_lo = pack_h2(x0 - __half2float(h0), x1 - __half2float(h1));
@@ -312,6 +312,7 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
         int lam_exp = INT_MIN;   // P s_g 2^lam_exp stays below 2^14 (fp16)
+        float sv_lim = 1.17549435e-38f;   // 2^(6 - lam_exp): the scale at which lam_exp must drop
         const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
 
         int first;
@@ -347,10 +348,12 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                             sv[r][2 * q2] = fv.x; sv[r][2 * q2 + 1] = fv.y;
                         }
                 }
+                if (nvalid < kPage) {   // the context's last page (warp-uniform): tail slots hold any bits
 #pragma unroll
-                for (int gi = 0; gi < 4; ++gi) {   // tail slots may hold any bits
-                    if (!ok0) { sk[0][gi] = 0.f; sv[0][gi] = 0.f; }
-                    if (!ok1) { sk[1][gi] = 0.f; sv[1][gi] = 0.f; }
+                    for (int gi = 0; gi < 4; ++gi) {
+                        if (!ok0) { sk[0][gi] = 0.f; sv[0][gi] = 0.f; }
+                        if (!ok1) { sk[1][gi] = 0.f; sv[1][gi] = 0.f; }
+                    }
                 }
 
                 // ---------------- QK, folded per group ------------------------------------
@@ -408,9 +411,7 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = i >> 1, e = i & 1;
-                    const bool okr = r ? ok1 : ok0;
-                    y[i] = okr ? raw[i] * kRsdLog2e : -INFINITY;
-                    if (!okr) cb[i] = 0.f;
+                    y[i] = raw[i] * kRsdLog2e;
                     if constexpr (kTierB) {   // u = sqrt(2 log(2S/delta) varsigma^2), grouped proxy
                         float ss = 0.f;
 #pragma unroll
@@ -418,14 +419,24 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                         u[i] = sqrtf(tbk * ss);
                     }
                 }
-                float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+                if (nvalid < kPage) {
 #pragma unroll
-                for (int o = 4; o < 32; o <<= 1) {
-                    mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
-                    mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+                    for (int i = 0; i < 4; ++i)
+                        if (!((i >> 1) ? ok1 : ok0)) {
+                            y[i] = -INFINITY;
+                            cb[i] = 0.f;
+                        }
                 }
-                const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
-                if (__any_sync(0xffffffffu, mv0 || mv1)) {
+                float mx0 = fmaxf(y[0], y[2]), mx1 = fmaxf(y[1], y[3]);
+                // the reference moves lazily (a logit above it by more than 8); the
+                // column maximum over the token rows is reduced only then
+                if (__any_sync(0xffffffffu, mx0 > m_run[0] + 8.0f || mx1 > m_run[1] + 8.0f)) {
+#pragma unroll
+                    for (int o = 4; o < 32; o <<= 1) {
+                        mx0 = fmaxf(mx0, __shfl_xor_sync(0xffffffffu, mx0, o));
+                        mx1 = fmaxf(mx1, __shfl_xor_sync(0xffffffffu, mx1, o));
+                    }
+                    const bool mv0 = mx0 > m_run[0] + 8.0f, mv1 = mx1 > m_run[1] + 8.0f;
                     const float a0 = mv0 ? (m_run[0] == -INFINITY ? 0.f : fast_exp2(m_run[0] - mx0)) : 1.f;
                     const float a1 = mv1 ? (m_run[1] == -INFINITY ? 0.f : fast_exp2(m_run[1] - mx1)) : 1.f;
                     if (mv0) m_run[0] = mx0;
@@ -446,29 +457,29 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                     const int e = i & 1;
                     pe[i] = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
                     l_part[e] += pe[i];
-                    d_part[e] = fmaf(pe[i], fast_exp2(cb[i] * kLog2e) - 1.f, d_part[e]);
+                    d_part[e] = fmaf(pe[i], fast_exp2(cb[i]) - 1.f, d_part[e]);
                     if constexpr (kTierB) db_part[e] = fmaf(pe[i], fast_exp2(u[i] * kLog2e) - 1.f, db_part[e]);
 #pragma unroll
                     for (int gi = 0; gi < 4; ++gi) spv[gi][e] = fmaf(pe[i], sv[i >> 1][gi], spv[gi][e]);
                 }
-                {   // P s_g 2^lam_exp < 2^14: s_g 2^lam_exp < 2^6 for every group of the page
+                {   // P s_g 2^lam_exp < 2^14: s_g 2^lam_exp < 2^6 for every group of the page;
+                    // lam_exp only decreases, checked per lane against sv_lim, reduced only then
                     float smax = 0.f;
 #pragma unroll
                     for (int gi = 0; gi < 4; ++gi) smax = fmaxf(smax, fmaxf(sv[0][gi], sv[1][gi]));
-                    const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
-                    if (wmax > 0.f) {
+                    if (__any_sync(0xffffffffu, smax >= sv_lim)) {
+                        const float wmax = __int_as_float(__reduce_max_sync(0xffffffffu, __float_as_int(smax)));
                         const int ex = ((__float_as_int(wmax) >> 23) & 0xFF) - 126;   // wmax < 2^ex
                         const int want = 6 - ex;
-                        if (lam_exp == INT_MIN) {
-                            lam_exp = want;
-                        } else if (want < lam_exp) {
+                        if (lam_exp != INT_MIN) {   // want < lam_exp here
                             const float f = pow2(want - lam_exp);
 #pragma unroll
                             for (int mt = 0; mt < 8; ++mt)
 #pragma unroll
                                 for (int e2 = 0; e2 < 4; ++e2) acc[mt][e2] *= f;
-                            lam_exp = want;
                         }
+                        lam_exp = want;
+                        sv_lim = pow2(6 - lam_exp);
                     }
                 }
                 const float lam = pow2(lam_exp == INT_MIN ? 0 : lam_exp);
@@ -497,8 +508,6 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                         bl0 = movmatrix_t(l01);
                         bl1 = movmatrix_t(l23);
                     }
-                    const uint32_t bn0 = bp0 ^ 0x80008000u, bn1 = bp1 ^ 0x80008000u;
-                    const uint32_t bm0 = bl0 ^ 0x80008000u, bm1 = bl1 ^ 0x80008000u;
 #pragma unroll
                     for (int mm = 0; mm < 2; ++mm) {
                         const int mt = 2 * gi + mm, wi = mt >> 1, pos = 2 * (mt & 1);
@@ -511,13 +520,13 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                             A[2 * pr + 1] = s8x2_to_h2(X, kSel23);
                             const uint32_t Y = prmt(word_of(dv[2 * pr], wi), word_of(dv[2 * pr + 1], wi),
                                                     sel_interleave(pos));
-                            H[2 * pr] = h8(Y, kSel01);
-                            H[2 * pr + 1] = h8(Y, kSel23);
+                            H[2 * pr] = nh8(Y, kSel01);       // -h'
+                            H[2 * pr + 1] = nh8(Y, kSel23);
                         }
                         mma16816(acc[mt], A, bp0, bp1);
                         mma16816(acc[mt], A, bl0, bl1);
-                        mma16816(acc[mt], H, bn0, bn1);
-                        mma16816(acc[mt], H, bm0, bm1);
+                        mma16816(acc[mt], H, bp0, bp1);
+                        mma16816(acc[mt], H, bl0, bl1);
                     }
                 }
             }
