@@ -113,7 +113,6 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
     }
 
     if (producer) {
-        const int tv[4] = {2 * c, 2 * c + 1, 2 * c + 8, 2 * c + 9};
         int k = 0, issued = 0;   // stage ring position, continued across segments
         bool stop = false;
         // one segment's pages (the split plan has one segment: no loop around it)
@@ -158,20 +157,27 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                 }
                 issued = k + 1;
                 if (ok) {   // dither bytes j[token][storage position], swizzled like the code tiles
+                    // K and V of tokens g, g+8 x position chunks 2c, 2c+1 (call 2i: K, 2i+1:
+                    // V), advanced round by round
                     const uint32_t slot0 = (uint32_t)phys * kPage;
-                    uint4 dk[4], dv[4];
+                    uint32_t x0[8], x1[8], x2[8], x3[8];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i)   // K: tokens g, g+8 x position chunks 2c, 2c+1
-                        dk[i] = philox(slot0 + g + 8 * (i >> 1), c1, (uint32_t)(2 * c + (i & 1)), 0u, p.keys);
+                    for (int j = 0; j < 8; ++j) {
+                        const int i = j >> 1;
+                        x0[j] = slot0 + g + 8 * (i >> 1);
+                        x1[j] = c1;
+                        x2[j] = (uint32_t)(2 * c + (i & 1));
+                        x3[j] = (uint32_t)(j & 1);
+                    }
+                    philox_n<8>(x0, x1, x2, x3, p.keys);
 #pragma unroll
-                    for (int j = 0; j < 4; ++j)   // V: tokens 2c, 2c+1, 2c+8, 2c+9 x position chunk g
-                        dv[j] = philox(slot0 + tv[j], c1, (uint32_t)g, 1u, p.keys);
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        *reinterpret_cast<uint4*>(st + kGwOffKd + swz(g + 8 * (i >> 1), 2 * c + (i & 1))) = dk[i];
-#pragma unroll
-                    for (int j = 0; j < 4; ++j)
-                        *reinterpret_cast<uint4*>(st + kGwOffVd + swz(tv[j], g)) = dv[j];
+                    for (int i = 0; i < 4; ++i) {
+                        const int off = swz(g + 8 * (i >> 1), 2 * c + (i & 1));
+                        *reinterpret_cast<uint4*>(st + kGwOffKd + off) =
+                            make_uint4(x0[2 * i], x1[2 * i], x2[2 * i], x3[2 * i]);
+                        *reinterpret_cast<uint4*>(st + kGwOffVd + off) =
+                            make_uint4(x0[2 * i + 1], x1[2 * i + 1], x2[2 * i + 1], x3[2 * i + 1]);
+                    }
                 }
                 __syncwarp();
                 if (lane == 0)   // second arrival: dither tiles and header are written

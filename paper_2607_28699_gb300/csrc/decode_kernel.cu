@@ -825,11 +825,22 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                     // their first round's product.
                     const uint32_t slot0 = (uint32_t)phys * kPage;
                     uint4 dk[4], dv[4];
+                    {   // call 2i: K, 2i+1: V of token g + 8 (i >> 1), group 2c + (i & 1)
+                        uint32_t x0[8], x1[8], x2[8], x3[8];
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) {
-                        const uint32_t slot = slot0 + g + 8 * (i >> 1), grp = (uint32_t)(2 * c + (i & 1));
-                        dk[i] = philox(slot, c1, grp, 0u, p.keys);
-                        dv[i] = philox(slot, c1, grp, 1u, p.keys);
+                        for (int j = 0; j < 8; ++j) {
+                            const int i = j >> 1;
+                            x0[j] = slot0 + g + 8 * (i >> 1);
+                            x1[j] = c1;
+                            x2[j] = (uint32_t)(2 * c + (i & 1));
+                            x3[j] = (uint32_t)(j & 1);
+                        }
+                        philox_n<8>(x0, x1, x2, x3, p.keys);
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            dk[i] = make_uint4(x0[2 * i], x1[2 * i], x2[2 * i], x3[2 * i]);
+                            dv[i] = make_uint4(x0[2 * i + 1], x1[2 * i + 1], x2[2 * i + 1], x3[2 * i + 1]);
+                        }
                     }
 #pragma unroll
                     for (int i = 0; i < 4; ++i) {

@@ -56,6 +56,28 @@ __device__ __forceinline__ uint4 philox(uint32_t c0, uint32_t c1, uint32_t c2, u
     return make_uint4(c0, c1, c2, c3);
 }
 
+// N independent Philox4x32-10 calls advanced round by round: counters in
+// (x0, x1, x2, x3)[j], results in place.  The calls' multiplies issue back to
+// back, so their latencies overlap (one call's rounds are a dependent chain).
+template <int N>
+__device__ __forceinline__ void philox_n(uint32_t (&x0)[N], uint32_t (&x1)[N], uint32_t (&x2)[N], uint32_t (&x3)[N],
+                                         const PhiloxKeys& key) {
+#pragma unroll
+    for (int r = 0; r < kPhiloxRounds; ++r) {
+#pragma unroll
+        for (int j = 0; j < N; ++j) {
+            const uint64_t p0 = (uint64_t)kPhiloxM0 * x0[j];
+            const uint64_t p1 = (uint64_t)kPhiloxM1 * x2[j];
+            const uint32_t n0 = (uint32_t)(p1 >> 32) ^ x1[j] ^ key.k0[r];
+            const uint32_t n2 = (uint32_t)(p0 >> 32) ^ x3[j] ^ key.k1[r];
+            x1[j] = (uint32_t)p1;
+            x3[j] = (uint32_t)p0;
+            x0[j] = n0;
+            x2[j] = n2;
+        }
+    }
+}
+
 // ---- byte / half packing -------------------------------------------------
 
 __device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
