@@ -210,30 +210,15 @@ class Setup:
             if layer + 1 < wl.n_layers:
                 del k, v
         # write-path throughput: the last layer's whole prefill, rewritten
-        # (same inputs, same slots) by warm, back-to-back calls
-        reps = 10
-        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.caches[-1])
-        torch.cuda.synchronize()
-        s.record()
-        for _ in range(reps):
-            wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.caches[-1])
-        e.record()
-        e.synchronize()
-        self.write_call_s = s.elapsed_time(e) / 1e3 / reps
+        # (same inputs, same slots) by warm, back-to-back calls replayed as a
+        # graph (device time, without the host's launch overhead)
+        def write_s(desc, cache, reps=10):
+            one = lambda: [wc.kv_quantize_witness(desc, wl.n_layers - 1, k, v, self.sm, cache) for _ in range(reps)]
+            return timed_graph_ms(capture(one), 5, 3) / 1e3 / reps
+        self.write_call_s = write_s(self.desc, self.caches[-1])
         if extras:
-            s.record()                                   # the same with the value witness stored too
-            for _ in range(reps):
-                wc.kv_quantize_witness(self.desc, wl.n_layers - 1, k, v, self.sm, self.vcaches[-1])
-            e.record()
-            e.synchronize()
-            self.write_v_call_s = s.elapsed_time(e) / 1e3 / reps
-            s.record()                                   # the grouped cache's write
-            for _ in range(reps):
-                wc.kv_quantize_witness(self.gdesc, wl.n_layers - 1, k, v, self.sm, self.gcaches[-1])
-            e.record()
-            e.synchronize()
-            self.write_g_call_s = s.elapsed_time(e) / 1e3 / reps
+            self.write_v_call_s = write_s(self.desc, self.vcaches[-1])   # the value witness stored too
+            self.write_g_call_s = write_s(self.gdesc, self.gcaches[-1])  # the grouped cache's write
         del k, v
         # the step's new tokens as one stacked tensor per side (one copy in the end-to-end step)
         self.k_new_all, self.v_new_all = torch.stack(self.k_new), torch.stack(self.v_new)

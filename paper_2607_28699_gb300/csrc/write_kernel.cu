@@ -117,11 +117,28 @@ __global__ void __launch_bounds__(128) write_kernel(const __grid_constant__ Writ
             raw[t][1] = __ldg(src + 1);
         }
     }
+    // 8-bit dither: the tasks' Philox calls (one per lane each) advanced together
+    uint4 w[kTasks];
+    constexpr bool kPre = kScheme != WC_SCHEME_FP8_E4M3 && kBits == 8;
+    if constexpr (kPre) {
+        uint32_t x0[kTasks], x1[kTasks], x2[kTasks], x3[kTasks];
+#pragma unroll
+        for (int t = 0; t < kTasks; ++t) {
+            x0[t] = (uint32_t)max(slot[t], 0);
+            x1[t] = (uint32_t)p.layer * 65536u + (uint32_t)hs[t];
+            x2[t] = (uint32_t)sub;
+            x3[t] = (uint32_t)row;
+        }
+        philox_n<kTasks>(x0, x1, x2, x3, p.keys);
+#pragma unroll
+        for (int t = 0; t < kTasks; ++t) w[t] = make_uint4(x0[t], x1[t], x2[t], x3[t]);
+    }
 #pragma unroll
     for (int t = 0; t < kTasks; ++t)
         if (__any_sync(0xffffffffu, live[t]))   // warp-uniform: a task past the end is skipped whole
             write_row<kScheme, kBits>(p, raw[t], slot[t], live[t], hs[t], row, sub,
-                                      kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab);
+                                      kGrouped ? xrows + (warp * 4 + (lane >> 3)) * kXRowStride : xrows, tab,
+                                      kPre ? &w[t] : nullptr);
 }
 
 // Bypass-pair calibration: a cluster of 8 CTAs of 32 warps per KV head.  Warp

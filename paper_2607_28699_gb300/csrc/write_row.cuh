@@ -86,9 +86,12 @@ constexpr int kXRowStride = 160;
 // One row (K or V) of one (token, KV head): 8 lanes, 16 channels each.
 // xrow: the unit's shared row (grouped scheme only); tab: the head's bypass
 // table, or nullptr (then each K row reads the pair list itself).
+// pre_w: this lane's dither word of the row when the caller drew it already
+// (8-bit dither; several rows' calls advanced together), else nullptr.
 template <int kScheme, int kBits>
 __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2], int slot, bool live_unit, int h,
-                                          int row, int sub, uint8_t* xrow, const BypassTable* tab) {
+                                          int row, int sub, uint8_t* xrow, const BypassTable* tab,
+                                          const uint4* pre_w = nullptr) {
     constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
     constexpr bool kDither = kScheme != WC_SCHEME_FP8_E4M3;
     const bool bad = slot >= p.num_pages * kPage;
@@ -148,7 +151,7 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
         uint32_t dw[8];
         if constexpr (kBits == 8) {
-            const uint4 w = philox(slot_u, c1, (uint32_t)sub, (uint32_t)row, p.keys);
+            const uint4 w = pre_w ? *pre_w : philox(slot_u, c1, (uint32_t)sub, (uint32_t)row, p.keys);
             dw[0] = w.x; dw[1] = w.y; dw[2] = w.z; dw[3] = w.w;
             if constexpr (kGrouped) {
                 // storage-position bytes -> this lane's channels 16 sub + i
