@@ -935,7 +935,7 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
 #pragma unroll
         for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
         int lam_exp = INT_MIN;
-        float sv_lim = 0.f;   // 2^(6 - lam_exp); 0 until the first positive scale
+        float sv_lim = 1.17549435e-38f;   // 2^(6 - lam_exp); until the first positive scale, FLT_MIN
 
         int first;
         const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);

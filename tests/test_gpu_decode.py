@@ -220,3 +220,34 @@ def test_decode_host_validation():
     with pytest.raises(wc.WitCertError) as e:
         wc.metered_decode_attention(wide, 0, q, bt, ctx, cache, ws)
     assert e.value.status == 2
+
+
+@pytest.mark.parametrize("ctx_lens", [[100, 40], [37]])
+def test_decode_zero_value_rows(ctx_lens):
+    """Value rows that are exactly zero have scale 0: pages whose every value
+    scale is 0 (the first pages of a sequence, or all of it) leave the P scale
+    unset until a positive one arrives; outputs and meters match the oracle."""
+    import paper_2607_28699_gb300 as wc
+    wl = W.Workload("zv", 1, 8, 2, ctx_lens, shuffle_pages=True, seed=12)
+    bt, sm, k, v, q = make_inputs(wl, 0)
+    v = v.clone()
+    v[:20] = 0                                   # the first page and a half of sequence 0
+    if len(ctx_lens) > 1:
+        v[ctx_lens[0]:] = 0                      # all of sequence 1
+    od, gd = descs(8, 2, wl.num_pages, seed=5)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, 0, k.numpy(), v.numpy(), sm, ocache)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
+    out, meter, raw = wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    offs = np.concatenate([[0], np.cumsum(ctx_lens)[:-1]])
+    for b, S in enumerate(ctx_lens):
+        r = OP.decode_sequence(od, 0, q.numpy()[b], bt[b], S, ocache, k.numpy()[offs[b]:offs[b] + S],
+                               v.numpy()[offs[b]:offs[b] + S])
+        assert np.all(np.isfinite(out[b].cpu().numpy()))
+        assert_close(out[b].cpu().numpy(), r["out"], f"out[{b}]")
+        assert_close(raw[b].cpu().numpy(), r["meter_raw"], f"meter_raw[{b}]")
+        assert_sound(raw[b].cpu().numpy(), r["meter_raw"], r["tv"], f"meter_raw[{b}]")
