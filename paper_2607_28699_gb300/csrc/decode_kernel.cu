@@ -1241,7 +1241,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int h = hq / p.group, hh = hq % p.group;
     const size_t unit = (size_t)b * p.num_kv_heads + h;
-    const int count = p.splits;   // split plan (the flattened plan has merge_flat_kernel)
+    const int count = p.splits;   // split plan with many splits (otherwise merge_warp_kernel)
     const float* base = p.partials + unit * p.splits * (kMaxGroup * kPartialStride) + hh * kPartialStride;
     const size_t split_stride = kMaxGroup * kPartialStride;
     __shared__ float red[kMergeWarps][38];
@@ -1414,12 +1414,17 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
 // instead of packed onto the first few SMs to free up.
 constexpr int kMergeSpreadSmem = 118784;
 
-// Merge under the flattened plan, where a unit has only a few partials (its
-// sequence's cuts): one warp per (sequence, query head, 32 output dims) folds
-// all of them in order with the same running-maximum update as merge_kernel,
-// so a CTA of 8 warps serves 8 outputs and needs no block barrier.
+// Merge where a unit has only a few partials: the flattened plan (its
+// sequence's cuts) and a split plan of at most kWarpMergeSplits splits (a
+// batch of sequences on the per-token kernel).  One warp per (sequence, query
+// head, 32 output dims) folds all of them in order with the same
+// running-maximum update as merge_kernel, so a CTA of 8 warps serves 8 outputs
+// and needs no block barrier, and a batch's merge is one wave of short warps
+// rather than several waves of CTAs with a block reduction each.
+constexpr int kWarpMergeSplits = 8;
+
 template <int kX>
-__global__ void __launch_bounds__(32 * kMergeWarps) merge_flat_kernel(const __grid_constant__ DecodeParams p) {
+__global__ void __launch_bounds__(32 * kMergeWarps) merge_warp_kernel(const __grid_constant__ DecodeParams p) {
     grid_dep_launch();   // the next kernel waits for this grid before reading its outputs
     grid_dep_wait();
     const int lane = threadIdx.x & 31;
@@ -1431,31 +1436,41 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_flat_kernel(const __gr
     const int h = hq / p.group, hh = hq % p.group;
     constexpr bool tier_b = (kX & kXTierB) != 0, vside = (kX & kXValue) != 0, repair = (kX & kXRepair) != 0;
 
-    // This unit's partials.  The batch's pages lie end to end (sequence b from
-    // P_b = sum_{b' < b} n_b', page counts of the clamped context lengths, as in
-    // the decode); share j of the splits / Hkv shares took positions
-    // [j R, (j + 1) R), R = ceil(total / shares), in each head, so the unit's
-    // segments are those of shares P_b / R .. (P_b + n_b - 1) / R, stored at
-    // partials h (shares + batch) + j + b, consecutive.
-    int before = 0, total = 0;
-    for (int i = lane; i < p.batch; i += 32) {
-        const int np = (max(0, min(__ldg(p.ctx_lens + i), p.max_pages * kPage)) + kPage - 1) / kPage;
-        total += np;
-        if (i < b) before += np;
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        before += __shfl_xor_sync(0xffffffffu, before, o);
-        total += __shfl_xor_sync(0xffffffffu, total, o);
-    }
     const int nb = (max(0, min(__ldg(p.ctx_lens + b), p.max_pages * kPage)) + kPage - 1) / kPage;
-    const int shares = max(1, p.splits / p.num_kv_heads);
-    const long long R = max(1LL, ((long long)total + shares - 1) / shares);
-    const long long j0 = before / R;
-    const int count = nb > 0 ? (int)(((long long)before + nb - 1) / R - j0 + 1) : 0;
-    const float* base = p.partials +
-                        ((size_t)h * (shares + p.batch) + (size_t)(j0 + b)) * (kMaxGroup * kPartialStride) +
-                        hh * kPartialStride;
+    int count;
+    const float* base;
+    if (p.pages_per_split > 0) {
+        // Split plan: the unit's splits are consecutive; those past the
+        // sequence's last page hold no pages (their maximum is -inf) and are
+        // not read.
+        count = min(p.splits, (nb + p.pages_per_split - 1) / p.pages_per_split);
+        base = p.partials + ((size_t)b * p.num_kv_heads + h) * p.splits * (kMaxGroup * kPartialStride) +
+               hh * kPartialStride;
+    } else {
+        // Flattened plan.  The batch's pages lie end to end (sequence b from
+        // P_b = sum_{b' < b} n_b', page counts of the clamped context lengths, as
+        // in the decode); share j of the splits / Hkv shares took positions
+        // [j R, (j + 1) R), R = ceil(total / shares), in each head, so the unit's
+        // segments are those of shares P_b / R .. (P_b + n_b - 1) / R, stored at
+        // partials h (shares + batch) + j + b, consecutive.
+        int before = 0, total = 0;
+        for (int i = lane; i < p.batch; i += 32) {
+            const int np = (max(0, min(__ldg(p.ctx_lens + i), p.max_pages * kPage)) + kPage - 1) / kPage;
+            total += np;
+            if (i < b) before += np;
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) {
+            before += __shfl_xor_sync(0xffffffffu, before, o);
+            total += __shfl_xor_sync(0xffffffffu, total, o);
+        }
+        const int shares = max(1, p.splits / p.num_kv_heads);
+        const long long R = max(1LL, ((long long)total + shares - 1) / shares);
+        const long long j0 = before / R;
+        count = nb > 0 ? (int)(((long long)before + nb - 1) / R - j0 + 1) : 0;
+        base = p.partials + ((size_t)h * (shares + p.batch) + (size_t)(j0 + b)) * (kMaxGroup * kPartialStride) +
+               hh * kPartialStride;
+    }
 
     constexpr int kRows = 8;   // rows loaded per round before any is combined
     float M = -INFINITY, acc = 0.f, L = 0.f, Dn = 0.f, Db = 0.f, Vt = 0.f, Vm = 0.f;
@@ -1542,9 +1557,9 @@ static cudaError_t launch_merge(const DecodeParams& p, cudaStream_t stream) {
                                    (int)cudaSharedmemCarveoutMaxShared);
         (void)cudaGetLastError();   // a refused hint leaves no sticky error behind
     });
-    if (p.pages_per_split == 0) {   // flattened plan
+    if (p.pages_per_split == 0 || p.splits <= kWarpMergeSplits) {   // a few partials per unit
         const long warps = (long)p.batch * p.num_q_heads * (kHeadDim / 32);
-        return launch_pdl(merge_flat_kernel<kX>, dim3((unsigned)((warps + kMergeWarps - 1) / kMergeWarps)),
+        return launch_pdl(merge_warp_kernel<kX>, dim3((unsigned)((warps + kMergeWarps - 1) / kMergeWarps)),
                           dim3(32 * kMergeWarps), 0, stream, p);
     }
     const dim3 grid(kHeadDim / 32, p.num_q_heads, p.batch);
