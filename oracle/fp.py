@@ -31,7 +31,8 @@ def fp16_ru(x):
     x = np.asarray(x, dtype=np.float64)
     if np.any(x < 0) or np.any(np.isnan(x)):
         raise ValueError("fp16_ru is defined here for non-negative values only")
-    h = x.astype(np.float16)
+    with np.errstate(over="ignore"):   # above the largest binary16 the least one >= x is +inf
+        h = x.astype(np.float16)
     below = h.astype(np.float64) < x
     bits = h.view(np.uint16).copy()
     bits[below] += 1            # next binary16 above a non-negative value

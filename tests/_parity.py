@@ -14,7 +14,8 @@ def close(gpu, ref, rtol=RTOL, atol=ATOL):
     gpu = np.asarray(gpu, dtype=np.float64)
     ref = np.asarray(ref, dtype=np.float64)
     both_inf = np.isinf(gpu) & np.isinf(ref) & (np.sign(gpu) == np.sign(ref))
-    ok = both_inf | (np.abs(gpu - ref) <= atol + rtol * np.abs(ref))
+    with np.errstate(invalid="ignore"):   # inf - inf: judged by both_inf
+        ok = both_inf | (np.abs(gpu - ref) <= atol + rtol * np.abs(ref))
     return ok
 
 
