@@ -265,17 +265,15 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
         const int nbt = (nb + 7) >> 3;   // bypass tiles of 8 dims
 
         // ---- per-group sums of q (bypassed channels left out), band norms ---------
-        float qs = 0.f, qq = 0.f, qsum_all = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
+        float qs = 0.f, qq = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
             const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&qn[i]));
             const bool b0 = (nmask >> (2 * i)) & 1u, b1 = (nmask >> (2 * i + 1)) & 1u;
             qs += (b0 ? 0.f : f.x) + (b1 ? 0.f : f.y);
             qq = fmaf(b0 ? 0.f : f.x, f.x, fmaf(b1 ? 0.f : f.y, f.y, qq));
-            qsum_all += f.x + f.y;
             part[i >> 2] = fmaf(f.x, f.x, fmaf(f.y, f.y, part[i >> 2]));   // channels 32c + 8(i>>2) .. +7
         }
-        (void)qsum_all;
         // kappa sum_g q and ||q_g'||^2 of group G for this thread's softmax heads 2c, 2c+1
         float zo[4][2], qn2[4][2];
 #pragma unroll
