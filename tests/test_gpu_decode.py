@@ -133,6 +133,40 @@ def test_decode_flattened_plan_batches(ctx_lens, hq, hkv):
         assert_close(np.maximum(meter[b], r_up["meter"]), r_up["meter"], f"meter[{b}]")
 
 
+@pytest.mark.parametrize("scheme,bits", [(1, 8), (0, 10)])
+def test_decode_split_plan_batch_few_splits(scheme, bits):
+    """A batch on the per-token kernel (fp8, the 10-bit dither) takes the split
+    plan; here 8 splits of 24 pages per sequence, so the merge runs one warp per
+    output over the splits that hold the sequence's pages.  Empty and short
+    sequences beside long ones: every sequence against the oracle, empty ones
+    give out = 0 and meter 0."""
+    import paper_2607_28699_gb300 as wc
+    ctx_lens = [0, 3000, 5, 1200, 0, 16, 2049]
+    wl = W.Workload("s", 1, 28, 4, ctx_lens, shuffle_pages=True, seed=12)
+    bt, sm, k, v, q = make_inputs(wl, 0)
+    od, gd = descs(28, 4, wl.num_pages, scheme, bits, 0, 5)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, 0, k.numpy(), v.numpy(), sm, ocache)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
+    out, meter, raw = wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, meter, raw = out.cpu().numpy(), meter.cpu().numpy(), raw.cpu().numpy()
+    offs = np.concatenate([[0], np.cumsum(ctx_lens)[:-1]])
+    for b, S in enumerate(ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(meter[b] == 0) and np.all(raw[b] == 0)
+            continue
+        o = offs[b]
+        r = OP.decode_sequence(od, 0, q.numpy()[b], bt[b], S, ocache, k.numpy()[o:o + S], v.numpy()[o:o + S])
+        assert_close(out[b], r["out"], f"out[{b}]")
+        assert_close(raw[b], r["meter_raw"], f"meter_raw[{b}]")
+        assert_close(meter[b], r["meter"], f"meter[{b}]")
+        assert_sound(raw[b], r["meter_raw"], r["tv"], f"meter_raw[{b}]")
+
+
 def test_decode_flattened_plan_bad_ctx_sets_status():
     """Out-of-range context lengths in a batch are clamped and reported."""
     import paper_2607_28699_gb300 as wc
