@@ -316,7 +316,7 @@ class Setup:
 
     def decode_all_repair(self, select=True):
         """The same calls emitting the per-page meter terms, the gate, then the
-        block-level repair selection of every cell the gate flagged (§6.4)."""
+        block-level repair selection of every cell the gate flagged (§6.3.5)."""
         wc, wl = self.wc, self.wl
         L, B, Hq = wl.n_layers, wl.batch, wl.n_q_heads
         if not hasattr(self, "page_terms"):
@@ -531,7 +531,7 @@ def run_ours(args, rank, world, local):
                   "delta_req": st.TIER_B_DELTA_REQ, "kept_frac_at_tau": float((mb <= st.tau).float().mean()),
                   "meter_b_raw_median": float(mb.median())}
 
-    # ---- the same calls emitting the repair terms, gate, repair selection (§6.4) ----
+    # ---- the same calls emitting the repair terms, gate, repair selection (§6.3.5) ----
     def graph_ms(fn, per):
         g = capture(fn)
         for _ in range(args.warmup):

@@ -327,7 +327,7 @@ wc_status wc_metered_decode_attention_append(const wc_cache_desc* desc, int32_t 
 
 /*
  * Metered decode attention with the per-page terms of block-level repair
- * selection (§6.4 "Block-level paging").  Same computation, arguments and
+ * selection (§6.3.5 "Block-level paging").  Same computation, arguments and
  * outputs as wc_metered_decode_attention, plus for every sequence b, query
  * head hq and logical page j < ceil(ctx_lens[b] / 16):
  *   page_terms[b][hq][j]  = (m_j, d_j) fp32: page j's share of D = A - 1,
@@ -353,7 +353,7 @@ wc_status wc_metered_decode_attention_repair(const wc_cache_desc* desc, int32_t 
                                              void* stream);
 
 /*
- * Block-level repair selection (§6.4 "Block-level paging").  With p~ held
+ * Block-level repair selection (§6.3.5 "Block-level paging").  With p~ held
  * fixed, paging in the exact keys of logical page j (witness 0) lowers D by
  * exactly C_j, so the fewest pages that bring the meter to tau are the
  * largest contributions.  For every cell (b, hq), with n = ceil(ctx_lens[b]/16):
@@ -426,7 +426,7 @@ wc_status wc_metered_decode_attention_g32(const wc_cache_desc* desc, int32_t lay
                                           void* workspace, size_t workspace_bytes, void* stream);
 
 /*
- * Bypass-pair calibration (§6.2.3 "Fixed-channel outlier bypass": the
+ * Bypass-pair calibration (§6.2.5 "Fixed-channel outlier bypass": the
  * massive-activation RoPE pairs are stable across tokens, so a fixed set per
  * (layer, KV head) chosen from a prefix suffices).  For each KV head h,
  * pairs[h][0 .. m-1] = the m RoPE pairs of largest energy

@@ -24,7 +24,7 @@ meter      exact / compressed attention, total variation (§3 setup), the
            Tier-B sub-Gaussian bound, per-token and grouped (§4.2), the
            e-form meter (§3 Thm. "Sound replacement"), the value term,
            output bound and joint gate (§3, §4.2), block-level repair
-           selection (§6.4), gate (§6 meter loop box).
+           selection (§6.3.5), gate (§6 meter loop box).
 pipeline   the write path over a paged cache (per-token, fp8 and grouped
            schemes) and the metered decode step, composed from the
            functions above.

@@ -40,7 +40,7 @@ formula): pass_V holds when the value term sum_t p~_t rho^v_t is at most
 tau_V max_t ||v_t||, and the joint gate keeps a cell iff pass_K (meter_raw
 <= tau_K) and pass_V, both decided in float32.
 
-§6.4 "Block-level paging": the e-form certificate is block decomposable.
+§6.3.5 "Block-level paging": the e-form certificate is block decomposable.
 With p~ held fixed, replacing page j's keys by their exact values sets c_t = 0
 for its tokens and lowers D = A - 1 by exactly C_j = sum_{t in j} p~_t
 expm1(c_t).  Paging in pages by decreasing C_j until 1/2 D (D + 2) <= tau

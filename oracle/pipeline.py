@@ -212,7 +212,7 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
     ``out_exact`` [Hq, d]; with ``delta_loc`` (dithered INT8 only) also the
     Tier-B meters ``meter_b``/``meter_b_raw`` [Hq] (§4.2); with ``repair_tau``
     also ``contrib`` [Hq, pages] (page contributions to D) and ``repair``
-    (per query head: the logical pages to page in, in order, §6.4).
+    (per query head: the logical pages to page in, in order, §6.3.5).
     """
     G = desc.num_q_heads // desc.num_kv_heads
     d = desc.head_dim

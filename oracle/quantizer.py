@@ -21,7 +21,7 @@ fp16 subnormal 2^-24 (then clipping can occur, and the witness, being the
 actual residual, stays sound); amax = 0 gives s = 0, code 0, x^ = 0.
 
 Grouped scales with a fixed-channel outlier bypass (§6.2.3 "Storage side",
-Table "granularity"; "Fixed-channel outlier bypass", Tables "amax" and
+Table "granularity"; §6.2.5 "Fixed-channel outlier bypass", Tables "amax" and
 "bypassbudget"): one fp16 scale per token and group of G_c contiguous
 channels (G_c = 32 by default), s_g = fp16_rn(fp32(amax_g) / 126.5f) by the
 rule above, where amax_g leaves out the bypassed channels; the bypassed

@@ -15,7 +15,7 @@ namespace {
 // Extra outputs compiled into a decode kernel (template bit mask).
 constexpr int kXTierB = 1;   // Tier-B meter (§4.2)
 constexpr int kXValue = 2;   // value-side witness terms and output bound (§3, §4.2)
-constexpr int kXRepair = 4;  // per-page meter terms for block-level repair selection (§6.4)
+constexpr int kXRepair = 4;  // per-page meter terms for block-level repair selection (§6.3.5)
 constexpr int kXAppend = 8;  // the decode writes the step's new token before reading it
 constexpr int kXFlat = 16;   // warp-specialized kernel under the flattened split plan
 // failure-detection test (warp-specialized kernel, split plan): one page's

@@ -1,5 +1,5 @@
 // Metered decode attention over the grouped-scale cache (§6.2.3 "Storage
-// side" and "Fixed-channel outlier bypass"): one fp16 scale per token and
+// side" and §6.2.5 "Fixed-channel outlier bypass"): one fp16 scale per token and
 // 32-channel group, and the m key RoPE pairs of a (layer, KV head) stored
 // exactly.  Warp-specialized like the per-token kernel: 6 producer / 6 consumer
 // warp pairs per CTA, one CTA per SM (at 384 threads the consumer keeps its ~165

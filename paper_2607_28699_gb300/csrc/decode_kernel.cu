@@ -43,7 +43,7 @@ constexpr int kOffVw = 4416;             // value witness [16][2] fp16 (value si
 constexpr int kStageStride = 4480;       // stage buffer size
 constexpr int kSmemBytes = kWarps * kStages * kStageStride + kWarps * kStages * 8;
 
-// §6.4 "Block-level paging": the share of D of logical page lp for this
+// §6.3.5 "Block-level paging": the share of D of logical page lp for this
 // thread's softmax heads 2c, 2c+1, kept against the running maximum it was
 // summed under; with the final (M, L) the page contributes d 2^(m - M) / L.
 // dpg holds the thread's tokens g, g+8 on entry; the sum runs over the rows g.

@@ -1,4 +1,4 @@
-// Block-level repair selection (§6.4 "Block-level paging").  The e-form
+// Block-level repair selection (§6.3.5 "Block-level paging").  The e-form
 // certificate is block decomposable: with p~ held fixed, replacing the keys of
 // logical page j by their exact values (witness 0, so c_t = 0) lowers D = A - 1
 // by exactly C_j = sum_{t in j} p~_t (e^{c_t} - 1).  For each cell the gate sent

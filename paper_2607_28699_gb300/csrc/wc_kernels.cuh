@@ -44,7 +44,7 @@ struct DecodeParams {
     float* value_term;           // value side outputs, nullptr: not computed
     float* v_max;
     float* out_bound;
-    // Block-level repair selection (§6.4), nullptr: not emitted.  Per page j of
+    // Block-level repair selection (§6.3.5), nullptr: not emitted.  Per page j of
     // each (sequence, query head): (m_j, d_j), the page's share of D summed
     // against the running maximum m_j, so that it contributes d_j 2^(m_j - M) / L;
     // per (sequence, query head): (M, L), the final log2-domain maximum and sum.

@@ -8,7 +8,7 @@
 // (for the dither schemes) consumes exactly one Philox4x32-10 call per 16
 // channels.
 //
-// Grouped scheme (§6.2.3 "Storage side" and "Fixed-channel outlier bypass"):
+// Grouped scheme (§6.2.3 "Storage side" and §6.2.5 "Fixed-channel outlier bypass"):
 // one fp16 scale per 32-channel group (a lane pair), the group amax leaving
 // out the bypassed channels of the KV head's fixed RoPE pairs, which are
 // stored exactly (fp16, code 0).  A row is stored in a permuted channel order

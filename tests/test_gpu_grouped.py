@@ -1,5 +1,5 @@
 """GPU parity of the grouped-scale cache with the fixed-channel outlier-pair
-bypass (§6.2.3 "Storage side", "Fixed-channel outlier bypass"): the write
+bypass (§6.2.3 "Storage side", §6.2.5 "Fixed-channel outlier bypass"): the write
 kernel's codes (in storage order), group scales and exact bypassed values bit
 for bit against the oracle, its witness at most one fp16 step above; the
 decode's output, meter and grouped Tier-B meter against the oracle on

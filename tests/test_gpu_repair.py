@@ -1,4 +1,4 @@
-"""GPU parity of block-level repair selection (§6.4 "Block-level paging"):
+"""GPU parity of block-level repair selection (§6.3.5 "Block-level paging"):
 the decode with per-page terms leaves the plain outputs bit for bit, the page
 contributions C_j match the oracle's, the list is consistent with the
 kernel's own contributions (ordering; the count may differ only where the

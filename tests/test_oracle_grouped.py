@@ -1,5 +1,5 @@
 """Pins for the oracle's grouped-scale cache with the fixed-channel outlier
-bypass (§6.2.3 "Storage side" and "Fixed-channel outlier bypass"): one group
+bypass (§6.2.3 "Storage side" and §6.2.5 "Fixed-channel outlier bypass"): one group
 of 128 channels and no bypass is the per-token scheme; each 32-channel group
 is the per-token quantizer run on its own channels; bypassed channels are
 exact and leave the group amax (no clipping elsewhere); the byte accounts of

@@ -1,4 +1,4 @@
-"""Pins for the oracle's block-level repair selection (§6.4 "Block-level
+"""Pins for the oracle's block-level repair selection (§6.3.5 "Block-level
 paging"): the certificate is block decomposable, so paging in page j (its
 exact keys carry a zero witness) lowers A by exactly that page's contribution
 C_j with p~ held fixed; the plan is the fewest pages that bring the meter to
