@@ -88,7 +88,7 @@ typedef enum {
     WC_SCHEME_FP8_E4M3 = 1,
     /* Subtractive-dither INT8 with one fp16 scale per token and 32-channel
      * group and a fixed per-(layer, KV head) set of m key RoPE pairs stored
-     * exactly ("outlier bypass", left out of the group amax); §6.2.3.  8-bit
+     * exactly ("outlier bypass", left out of the group amax); §6.2.3, §6.2.5.  8-bit
      * dither only; written and read by the _g32 entry points. */
     WC_SCHEME_DITHER_INT8_G32 = 2
 } wc_scheme;
@@ -384,7 +384,7 @@ wc_status wc_repair_select(const float* page_terms, const float* softmax_norm,
                            float* d_after, uint32_t* dev_status, void* stream);
 
 /*
- * Write path of the grouped scheme (§6.2.3 "Storage side", "Fixed-channel
+ * Write path of the grouped scheme (§6.2.3 "Storage side", §6.2.5 "Fixed-channel
  * outlier bypass"): as wc_kv_quantize_witness, with for each row and group g
  * of 32 channels s_g = fp16_rn(fp32(amax_g) / 126.5f), amax_g over the
  * group's channels that are not bypassed (a key row's bypassed channels, the

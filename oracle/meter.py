@@ -11,8 +11,8 @@ sign convention p_t = p~_t exp(-eps_t) / Z, i.e. eps_t = z~_t - z_t.
 
 §3 Thm. "Sound replacement": A = E_p~[e^c] and TV <= 1/2 (A^2 - 1).
 The meter is reported as min(1, .) (§4.3) and evaluated without truncating
-c; +inf on overflow is sound and counts as over threshold (§6.2.3
-telemetry).  Here 1/2 (A^2 - 1) is computed as 1/2 D (D + 2) with
+c; +inf on overflow is sound and counts as over threshold (§6.2.5, on
+fp32 overflow).  Here 1/2 (A^2 - 1) is computed as 1/2 D (D + 2) with
 D = A - 1 = E_p~[expm1(c)], which is the same number without the
 cancellation of A^2 - 1 for small c (reading: the paper only asks for a
 numerically careful evaluation, "in the log domain").
