@@ -7,10 +7,12 @@
 // mean, so it merges exactly like the output; §6.2.2).
 //
 // Grid (splits, Hkv, batch); 8 warps per CTA, two CTAs per SM.  Each warp owns
-// a 3-stage ring of page buffers in shared memory filled by bulk asynchronous
-// copies (cp.async.bulk + mbarrier) that its lane 0 issues ahead of use; a
-// page is 16 tokens of one KV head (2 KiB K codes, 2 KiB V codes, scales,
-// witness).  Warps run independently until the CTA's closing merge.
+// a 3-stage ring of page buffers in shared memory that its lane 0 fills ahead
+// of use: the K and V code tiles (2 KiB each) by tensor-map TMA with the
+// 128-byte swizzle (so the 16-byte reads of a warp phase hit distinct banks),
+// scales and witness by bulk copies, all completing on the stage's mbarrier;
+// a page is 16 tokens of one KV head.  Warps run independently until the
+// CTA's closing merge.
 //
 // Per page a warp computes, on mma.sync (fp16 in, fp32 accumulate):
 //   QK:    S[token][head]  = code . q - h' . q                m16n8k16, A = codes / dither
@@ -38,10 +40,21 @@ constexpr int kThreads = 32 * kWarps;
 constexpr int kStages = 3;
 constexpr int kMinBlocks = 2;            // two CTAs (16 warps) per SM
 constexpr int kStageBytes = 4416;        // copy bytes: K codes | V codes | K scale | V scale | witness
-constexpr int kOffV = 2048, kOffKs = 4096, kOffVs = 4128, kOffW = 4160;
-constexpr int kOffVw = 4416;             // value witness [16][2] fp16 (value side)
-constexpr int kStageStride = 4480;       // stage buffer size
-constexpr int kSmemBytes = kWarps * kStages * kStageStride + kWarps * kStages * 8;
+// Shared memory: the K and V code tiles of every (warp, stage), [16][128] bytes
+// each, written by tensor-map TMA with the 128-byte swizzle (1024-byte aligned
+// regions), then each stage's scales and witness, then the barriers.
+constexpr int kTileRegion = kWarps * kStages * 2048;
+constexpr int kOffKs = 0, kOffVs = 32, kOffW = 64;   // within a stage's small part
+constexpr int kOffVw = 320;              // value witness [16][2] fp16 (value side)
+constexpr int kSmallStride = 384;
+constexpr int kSmemBytes = 2 * kTileRegion + kWarps * kStages * kSmallStride + kWarps * kStages * 8 + 1024;
+
+// The per-token kernel's parameters: the code tiles' tensor maps and the call.
+struct DkParams {
+    CUtensorMap k_map;   // k_codes as [num_pages * Hkv][16][128] bytes, box = one page of one head
+    CUtensorMap v_map;
+    DecodeParams p;
+};
 
 // §6.3.5 "Block-level paging": the share of D of logical page lp for this
 // thread's softmax heads 2c, 2c+1, kept against the running maximum it was
@@ -69,17 +82,21 @@ __device__ __forceinline__ void emit_skipped_page(const DecodeParams& p, int b, 
 }
 
 template <int kScheme, int kBits, int kX>
-__global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DecodeParams p) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DkParams dp) {
     constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
-    extern __shared__ __align__(128) uint8_t smem[];
+    const DecodeParams& p = dp.p;
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
+    uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
     const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
     const int G = p.group;
     constexpr bool kInt8 = (kScheme == WC_SCHEME_DITHER_INT8);
 
-    uint8_t* my_stages = smem + warp * kStages * kStageStride;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + kWarps * kStages * kStageStride) + warp * kStages;
+    uint8_t* my_k = smem + warp * kStages * 2048;   // this warp's K code tiles; its V tiles kTileRegion on
+    uint8_t* my_small = smem + 2 * kTileRegion + warp * kStages * kSmallStride;
+    uint64_t* bars =
+        reinterpret_cast<uint64_t*>(smem + 2 * kTileRegion + kWarps * kStages * kSmallStride) + warp * kStages;
     if (lane == 0)
         for (int s = 0; s < kStages; ++s) mbar_init(&bars[s], 1);
     fence_barrier_init();
@@ -128,12 +145,14 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
             return;
         }
-        uint8_t* st = my_stages + (k % kStages) * kStageStride;
-        const size_t ph = (size_t)phys * p.num_kv_heads + h;
+        const int s = k % kStages;
+        uint8_t* st = my_small + s * kSmallStride;
+        const int z = phys * p.num_kv_heads + h;
+        const size_t ph = (size_t)z;
         constexpr uint32_t bytes = (kInt8 ? kStageBytes : (2048 + 2048 + 256)) + (kValue ? 64 : 0);
         mbar_arrive_expect_tx(bar, bytes);
-        bulk_g2s(st, p.k_codes + ph * (kPage * kHeadDim), 2048, bar);
-        bulk_g2s(st + kOffV, p.v_codes + ph * (kPage * kHeadDim), 2048, bar);
+        tma_page(my_k + s * 2048, &dp.k_map, z, bar);
+        tma_page(my_k + kTileRegion + s * 2048, &dp.v_map, z, bar);
         if constexpr (kInt8) {
             bulk_g2s(st + kOffKs, p.k_scale + ph * kPage, 32, bar);
             bulk_g2s(st + kOffVs, p.v_scale + ph * kPage, 32, bar);
@@ -224,7 +243,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         }
         consumed = k + 1;
         if (page_ok) {
-            const uint8_t* st = my_stages + (k % kStages) * kStageStride;
+            const uint8_t* st = my_small + (k % kStages) * kSmallStride;
+            const uint8_t* kt = my_k + (k % kStages) * 2048;   // V tile at kt + kTileRegion
             const uint32_t slot0 = (uint32_t)phys * kPage;
             const int nvalid = min(kPage, ctx - lp * kPage);
 
@@ -234,8 +254,8 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             float dc[4] = {0.f, 0.f, 0.f, 0.f}, dd[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
             for (int gp = 0; gp < 2; ++gp) {                 // channels 32c + 16gp .. +15
-                const uint4 ka = *reinterpret_cast<const uint4*>(st + g * kHeadDim + 32 * c + 16 * gp);
-                const uint4 kb = *reinterpret_cast<const uint4*>(st + (g + 8) * kHeadDim + 32 * c + 16 * gp);
+                const uint4 ka = *reinterpret_cast<const uint4*>(kt + swz(g, 2 * c + gp));
+                const uint4 kb = *reinterpret_cast<const uint4*>(kt + swz(g + 8, 2 * c + gp));
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk) {
                     const int ks = 4 * gp + kk;              // channels 32c + 4ks .. +3
@@ -401,7 +421,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             uint4 vq[4];
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-                vq[j] = *reinterpret_cast<const uint4*>(st + kOffV + tv[j] * kHeadDim + 16 * g);
+                vq[j] = *reinterpret_cast<const uint4*>(kt + kTileRegion + swz(tv[j], g));
                 // an fp8 NaN byte in an unused tail slot would poison P = 0 columns
                 if (!kInt8 && tv[j] >= nvalid) vq[j] = make_uint4(0, 0, 0, 0);
             }
@@ -1588,8 +1608,13 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
         if (e != cudaSuccess) return e;
         configured = true;
     }
+    DkParams dp;
+    dp.p = p;
+    if (!encode_page_map(&dp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
+        !encode_page_map(&dp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
+        return cudaErrorInvalidValue;
     dim3 grid(p.splits, p.num_kv_heads, p.batch);
-    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kX>, grid, dim3(kThreads), kSmemBytes, stream, p);
+    cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kX>, grid, dim3(kThreads), kSmemBytes, stream, dp);
     if (e != cudaSuccess) return e;
     // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
