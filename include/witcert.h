@@ -269,16 +269,17 @@ wc_status wc_metered_decode_attention_v(const wc_cache_desc* desc, int32_t layer
  * provide the workspace wc_metered_decode_attention needs.
  *
  * Same computation, arguments and outputs as wc_metered_decode_attention,
- * without the workspace.  Its scratch is one fixed 4 MiB device array built
+ * without the workspace.  Its scratch is one fixed 16 MiB device array built
  * into the library; every GPU that loads the library keeps it until the
  * process exits.  The call never allocates or frees memory.
  *   dev_status  device uint32 that collects the WC_DEV_* bits (OR), required
  *               (not NULL: the built-in scratch has no word a caller can read);
  *               read and clear it with wc_read_status(dev_status, 1, ...).
  * Returns WC_ERR_UNSUPPORTED, launching nothing, when the decode would need
- * more scratch than 4 MiB (about 930 partial results: one per (KV head,
- * split) for one sequence; the SM count plus batch x Hkv for several
- * sequences; the count follows wc_workspace_size's plan).
+ * more scratch than 16 MiB (about 3700 partial results: one per (KV head,
+ * split) for one sequence; for several sequences the SM count (8 per SM's two
+ * CTAs for fp8 and the 10-bit dither) plus batch x Hkv; the count follows
+ * wc_workspace_size's plan).
  * The first call on each device, and the first after its context has been
  * recreated (cudaDeviceReset), looks up the scratch address
  * (cudaGetSymbolAddress); make that first call before any stream capture.

@@ -501,7 +501,7 @@ wc_status wc_read_status(void* workspace_or_word, int32_t is_status_word, uint32
 // ---------------------------------------------------------------------------
 namespace {
 
-constexpr size_t kNoAllocScratchBytes = size_t(4) << 20;   // 4 MiB per device
+constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;   // 16 MiB per device
 constexpr int kNoAllocMaxDevices = 64;
 
 // File-scope device scratch.  In host code this name is only a stand-in for

@@ -6,7 +6,9 @@
 // merged across context splits under log-sum-exp weights (A is a p~-weighted
 // mean, so it merges exactly like the output; §6.2.2).
 //
-// Grid (splits, Hkv, batch); 8 warps per CTA, two CTAs per SM.  Each warp owns
+// Grid (splits, Hkv, batch), or under the flattened plan (kXFlat: the 10-bit
+// dither on a batch that leaves SMs idle) one CTA per 8 warp shares of the
+// batch's pages; 8 warps per CTA, two CTAs per SM.  Each warp owns
 // a 3-stage ring of page buffers in shared memory that its lane 0 fills ahead
 // of use: the K and V code tiles (2 KiB each) by tensor-map TMA with the
 // 128-byte swizzle (so the 16-byte reads of a warp phase hit distinct banks),
@@ -81,6 +83,39 @@ __device__ __forceinline__ void emit_skipped_page(const DecodeParams& p, int b, 
             make_float2(-INFINITY, 0.f);
 }
 
+// q fragment of the B operand (head g, channels 32c + 2i, +1 in word i).
+__device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h, int G, int g, int c,
+                                            uint32_t (&qw)[16]) {
+    const bool row_valid = g < G;
+    const uint4* qsrc = reinterpret_cast<const uint4*>(
+        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
+        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+    }
+}
+
+// A warp's pages in order.  Split plan: pages warp, warp + 8, ... of one
+// sequence's split.  Flattened plan: a contiguous range of the batch's pages
+// laid end to end, sequence after sequence (sequences without pages hold
+// none of it).  dk_next is called only while the range has another page.
+struct DkWalk {
+    int b, lp, np;   // sequence, logical page, the sequence's page count
+};
+template <bool kFlat>
+__device__ __forceinline__ void dk_next(const DecodeParams& p, DkWalk& w) {
+    if constexpr (!kFlat) {
+        w.lp += kWarps;
+    } else if (++w.lp >= w.np) {
+        do {
+            ++w.b;
+            w.np = (clamped_ctx(p, w.b) + kPage - 1) / kPage;
+        } while (w.np == 0 && w.b + 1 < p.batch);
+        w.lp = 0;
+    }
+}
+
 template <int kScheme, int kBits, int kX>
 __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __grid_constant__ DkParams dp) {
     constexpr bool kTierB = (kX & kXTierB) != 0, kValue = (kX & kXValue) != 0, kRepair = (kX & kXRepair) != 0;
@@ -89,7 +124,12 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     uint8_t* smem = smem_raw + ((1024 - (smem_addr(smem_raw) & 1023)) & 1023);
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int g = lane >> 2, c = lane & 3;
-    const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+    // split plan: grid (splits, Hkv, batch); flattened plan (kXFlat): grid (CTAs),
+    // CTA c serving KV head c mod Hkv, each warp its own share of the batch's pages
+    constexpr bool kFlat = (kX & kXFlat) != 0;
+    const int split = kFlat ? 0 : (int)blockIdx.x;
+    const int h = kFlat ? (int)blockIdx.x % p.num_kv_heads : (int)blockIdx.y;
+    int b = kFlat ? 0 : (int)blockIdx.z;   // the sequence whose pages are being consumed
     const int G = p.group;
     constexpr bool kInt8 = (kScheme == WC_SCHEME_DITHER_INT8);
 
@@ -105,35 +145,104 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     grid_dep_launch();
     grid_dep_wait();   // q, page tables and the cache may come from the preceding kernel
 
-    // Independent loads first: context length, this warp's first page-table
-    // entries and the query fragments do not depend on one another.
-    const int p0 = split * p.pages_per_split;
-    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;
-    const int lim = min(p0 + p.pages_per_split, p.max_pages);
-    int ring[kStages];   // physical pages of this warp's next kStages pages
-#pragma unroll
-    for (int k = 0; k < kStages; ++k) {
-        const int lp = p0 + warp + kWarps * k;
-        ring[k] = lp < lim ? __ldg(bt_row + lp) : -1;
-    }
-    int ctx = __ldg(p.ctx_lens + b);
     const bool row_valid = g < G;
-    const uint4* qsrc = reinterpret_cast<const uint4*>(
-        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
-    uint32_t qw[16];   // head g, channels 32c + 2i, +1 in word i
+    const int p0 = split * p.pages_per_split;                          // split plan
+    const int32_t* bt_row = p.block_table + (size_t)b * p.max_pages;   // split plan
+    int ring[kStages];   // physical pages of this warp's next kStages pages
+    uint32_t qw[16];     // head g, channels 32c + 2i, +1 in word i
+    int ctx, n_my;
+    DkWalk cw, iw;       // flattened plan: the page being consumed, the next page to issue
+    if constexpr (!kFlat) {
+        // Independent loads first: context length, this warp's first page-table
+        // entries and the query fragments do not depend on one another.
+        const int lim = min(p0 + p.pages_per_split, p.max_pages);
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
-        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
+        for (int k = 0; k < kStages; ++k) {
+            const int lp = p0 + warp + kWarps * k;
+            ring[k] = lp < lim ? __ldg(bt_row + lp) : -1;
+        }
+        ctx = __ldg(p.ctx_lens + b);
+        load_q_frag(p, b, h, G, g, c, qw);
+        if (ctx < 0 || ctx > p.max_pages * kPage) {
+            if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+            ctx = max(0, min(ctx, p.max_pages * kPage));
+        }
+        const int npages = (ctx + kPage - 1) / kPage;
+        const int p1 = min(p0 + p.pages_per_split, npages);
+        n_my = (p1 - p0 - warp > 0) ? (p1 - p0 - warp + kWarps - 1) / kWarps : 0;
+        cw = iw = DkWalk{b, 0, 0};
+    } else {
+        // Warp share J = (c / Hkv) * 8 + warp takes pages [J R, (J + 1) R) of the
+        // batch's pages laid end to end, R = ceil(total / shares), shares =
+        // splits / Hkv; a scan of the page counts finds where each range starts.
+        __shared__ int s_wtot[kWarps];
+        __shared__ long long s_start[kWarps];
+        const int t = threadIdx.x, per = (p.batch + kThreads - 1) / kThreads;
+        int loc = 0;
+        bool bad = false;
+        for (int i = 0; i < per; ++i) {
+            const int bb = t * per + i;
+            if (bb < p.batch) {
+                const int cx = __ldg(p.ctx_lens + bb);
+                bad |= cx < 0 || cx > p.max_pages * kPage;
+                loc += (max(0, min(cx, p.max_pages * kPage)) + kPage - 1) / kPage;
+            }
+        }
+        if (bad && blockIdx.x == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
+        int inc = loc;   // inclusive scan over the warp
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int v = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += v;
+        }
+        if (lane == 31) s_wtot[warp] = inc;
+        __syncthreads();
+        int before = 0, total = 0;
+#pragma unroll
+        for (int w = 0; w < kWarps; ++w) {
+            const int v = s_wtot[w];
+            total += v;
+            if (w < warp) before += v;
+        }
+        const int excl = before + inc - loc;   // pages of the sequences before this thread's
+        const int shares = max(1, p.splits / p.num_kv_heads);
+        const long long R = max(1LL, ((long long)total + shares - 1) / shares);
+        const long long j0 = (long long)((int)blockIdx.x / p.num_kv_heads) * kWarps;
+        for (int w = 0; w < kWarps; ++w) {
+            const long long lo = (j0 + w) * R;
+            if (lo < total && excl <= lo && lo < (long long)excl + loc) {
+                long long acc = excl;   // exactly one thread: the one whose sequences hold lo
+                for (int i = 0; i < per; ++i) {
+                    const int bb = t * per + i;
+                    if (bb >= p.batch) break;
+                    const int np = (clamped_ctx(p, bb) + kPage - 1) / kPage;
+                    if (lo < acc + np) {
+                        s_start[w] = ((long long)bb << 32) | (long long)(lo - acc);
+                        break;
+                    }
+                    acc += np;
+                }
+            }
+        }
+        __syncthreads();
+        const long long lo = (j0 + warp) * R;
+        n_my = (int)max(0LL, min((long long)total, lo + R) - lo);
+        if (n_my > 0) {
+            const long long st = s_start[warp];
+            cw.b = (int)(st >> 32);
+            cw.lp = (int)(st & 0xffffffffLL);
+            cw.np = (clamped_ctx(p, cw.b) + kPage - 1) / kPage;
+        } else {
+            cw = DkWalk{0, 0, 0};
+        }
+        iw = cw;
+#pragma unroll
+        for (int k = 0; k < kStages; ++k) {
+            ring[k] = k < n_my ? __ldg(p.block_table + (size_t)iw.b * p.max_pages + iw.lp) : -1;
+            if (k + 1 < n_my) dk_next<true>(p, iw);
+        }
+        ctx = 0;
     }
-
-    if (ctx < 0 || ctx > p.max_pages * kPage) {
-        if (threadIdx.x == 0 && split == 0 && h == 0) atomicOr(p.status, WC_DEV_BAD_CTX);
-        ctx = max(0, min(ctx, p.max_pages * kPage));
-    }
-    const int npages = (ctx + kPage - 1) / kPage;
-    const int p1 = min(p0 + p.pages_per_split, npages);
-    const int n_my = (p1 - p0 - warp > 0) ? (p1 - p0 - warp + kWarps - 1) / kWarps : 0;
     const uint32_t c1 = (uint32_t)p.layer * 65536u + (uint32_t)h;
 
     // ---- per-warp stage ring --------------------------------------------------
@@ -164,7 +273,11 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
 #pragma unroll
     for (int k = 0; k < kStages; ++k) issue(k, ring[k]);
 
-    // ---- band norms and the bound operand ----------------------------------------
+    // ---- per sequence: band norms and the bound operand ----------------------------
+    // (once under the split plan; at each sequence's first page under the flattened plan)
+    float alpha0, alpha1, zoff0, zoff1;
+    uint32_t a_hi, a_lo;   // B operand of the bound: a[head g][bands 2c, 2c+1]
+    auto query_setup = [&]() {
     float qsum = 0.f, part[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int i = 0; i < 16; ++i) {
@@ -176,7 +289,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     qsum += __shfl_xor_sync(0xffffffffu, qsum, 2);
     // Tier B (§4.2): u_t = alpha s_t with alpha = sqrt(2 log(2S/delta) ||q||^2 / (12 d)),
     // for this thread's softmax heads 2c and 2c+1
-    float alpha0 = 0.f, alpha1 = 0.f;
+    alpha0 = alpha1 = 0.f;
     if constexpr (kTierB) {
         float qn2 = part[0] + part[1] + part[2] + part[3];   // ||q_g||^2 over channels 32c .. 32c+31
         qn2 += __shfl_xor_sync(0xffffffffu, qn2, 1);
@@ -201,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         band_a = part[0] + part[1];   // dims 32c .. 32c+15 = band 2c
         band_b = part[2] + part[3];
     }
-    uint32_t a_hi = 0, a_lo = 0;   // B operand of the bound: a[head g][bands 2c, 2c+1]
+    a_hi = a_lo = 0;
     if (row_valid) {
         const float x0 = sqrtf(band_a) * kRsd, x1 = sqrtf(band_b) * kRsd;
         const __half h0 = __float2half_rn(x0), h1 = __float2half_rn(x1);
@@ -210,30 +323,101 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
     }
     // this thread's softmax heads are 2c and 2c+1: kappa * sum(q) for each
     constexpr float kKappa = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
-    const float zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
-    const float zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
+    zoff0 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c);
+    zoff1 = kKappa * __shfl_sync(0xffffffffu, qsum, 8 * c + 4);
+    };
+    if constexpr (!kFlat) query_setup();
 
     // ---- running state (heads 2c, 2c+1) ----------------------------------------------
     // Log2-domain softmax reference, moved lazily: only when a page's max
     // exceeds it by more than 8 (P may reach 2^8 in between).
-    float m_run[2] = {-INFINITY, -INFINITY};
-    float l_part[2] = {0.f, 0.f}, d_part[2] = {0.f, 0.f}, spv_part[2] = {0.f, 0.f};
-    float db_part[2] = {0.f, 0.f};   // Tier-B meter accumulator (kTierB)
-    float vt_part[2] = {0.f, 0.f};   // value side: sum p~ rho^v (kValue)
-    float vmax = 0.f;                // value side: max ||v|| over this thread's tokens
+    float m_run[2], l_part[2], d_part[2], spv_part[2];
+    float db_part[2];   // Tier-B meter accumulator (kTierB)
+    float vt_part[2];   // value side: sum p~ rho^v (kValue)
+    float vmax;         // value side: max ||v|| over this thread's tokens
     float acc[8][4];
+    int lam_exp;        // P * s_v * 2^lam_exp stays below 2^14 (fp16): s_v * 2^lam_exp < 2^6
+    auto reset_state = [&]() {
+        m_run[0] = m_run[1] = -INFINITY;
+        l_part[0] = l_part[1] = d_part[0] = d_part[1] = spv_part[0] = spv_part[1] = 0.f;
+        db_part[0] = db_part[1] = vt_part[0] = vt_part[1] = 0.f;
+        vmax = 0.f;
 #pragma unroll
-    for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
-    // P * s_v * 2^lam_exp stays below 2^14 (fp16): s_v * 2^lam_exp < 2^6.
-    int lam_exp = kInt8 ? INT_MIN : 6;
+        for (int i = 0; i < 8; ++i) acc[i][0] = acc[i][1] = acc[i][2] = acc[i][3] = 0.f;
+        lam_exp = kInt8 ? INT_MIN : 6;
+    };
+    reset_state();
     bool failed = false;
     int consumed = 0;
+    // ---- a warp's rows: totals for heads 2c, 2c+1 (reduced over the token rows g),
+    // then its partial [head][kPartialStride] at wb (shared memory for the CTA merge
+    // of the split plan, the workspace under the flattened plan)
+    auto warp_rows = [&](float* wb) {
+#pragma unroll
+        for (int o = 4; o < 32; o <<= 1)
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
+                d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
+                if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
+                if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
+                spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
+            }
+        if constexpr (kValue)
+            for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+        const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
+        const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
+#pragma unroll
+        for (int e = 0; e < 2; ++e) {
+            float* row = wb + (2 * c + e) * kPartialStride + 16 * g;   // dims 16g .. 16g+15
+            const float add = kap * spv_part[e];
+#pragma unroll
+            for (int q4 = 0; q4 < 4; ++q4) {
+                float4 v;
+                v.x = fmaf(acc[2 * q4][e], inv_lam, add);
+                v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
+                v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
+                v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
+                *reinterpret_cast<float4*>(row + 4 * q4) = v;
+            }
+            if (g == 0) {
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
+                wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
+                if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
+                if constexpr (kValue) {
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
+                    wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
+                }
+            }
+        }
+    };
+    // flattened plan: warp share J's part of sequence b is partial h (shares + batch) + J + b
+    // (unique; a unit's partials consecutive, as the merge reads them)
+    auto flat_partial = [&]() {
+        const int shares = max(1, p.splits / p.num_kv_heads);
+        const int J = ((int)blockIdx.x / p.num_kv_heads) * kWarps + warp;
+        return p.partials + ((size_t)h * (shares + p.batch) + J + b) * (kMaxGroup * kPartialStride);
+    };
 
     for (int k = 0; k < n_my; ++k) {
-        const int lp = p0 + warp + kWarps * k;
+        int lp, phys_issue;   // this page; the page-table entry of the page issued at the end of the iteration
+        if constexpr (kFlat) {
+            if (k == 0 || cw.b != b) {   // a sequence's first page of this warp (warp-uniform)
+                if (k > 0) warp_rows(flat_partial());
+                b = cw.b;
+                ctx = clamped_ctx(p, b);
+                load_q_frag(p, b, h, G, g, c, qw);
+                query_setup();
+                reset_state();
+            }
+            lp = cw.lp;
+            phys_issue = (k + kStages < n_my) ? __ldg(p.block_table + (size_t)iw.b * p.max_pages + iw.lp) : -1;
+        } else {
+            lp = p0 + warp + kWarps * k;
+            phys_issue = (k + kStages < n_my) ? __ldg(bt_row + lp + kWarps * kStages) : -1;
+        }
         const int phys = ring[0];
-        // page-table entry for the page issued at the end of this iteration
-        const int phys_issue = (k + kStages < n_my) ? __ldg(bt_row + lp + kWarps * kStages) : -1;
         const bool page_ok = phys >= 0 && phys < p.num_pages;
         const bool landed = mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
         if (!__all_sync(0xffffffffu, landed)) {   // warp-uniform decision
@@ -492,6 +676,10 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
         }
         __syncwarp();
         issue(k + kStages, phys_issue);
+        if constexpr (kFlat) {
+            if (k + kStages + 1 < n_my) dk_next<true>(p, iw);
+            if (k + 1 < n_my) dk_next<true>(p, cw);
+        }
 #pragma unroll
         for (int i = 0; i + 1 < kStages; ++i) ring[i] = ring[i + 1];
         ring[kStages - 1] = phys_issue;
@@ -502,52 +690,15 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
             (void)mbar_wait_bounded(&bars[k % kStages], (uint32_t)((k / kStages) & 1));
     }
 
-    // ---- warp totals for heads 2c, 2c+1 (reduce over the token rows g) ----------------
-#pragma unroll
-    for (int o = 4; o < 32; o <<= 1)
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            l_part[e] += __shfl_xor_sync(0xffffffffu, l_part[e], o);
-            d_part[e] += __shfl_xor_sync(0xffffffffu, d_part[e], o);
-            if constexpr (kTierB) db_part[e] += __shfl_xor_sync(0xffffffffu, db_part[e], o);
-            if constexpr (kValue) vt_part[e] += __shfl_xor_sync(0xffffffffu, vt_part[e], o);
-            spv_part[e] += __shfl_xor_sync(0xffffffffu, spv_part[e], o);
-        }
-    if constexpr (kValue)
-        for (int o = 1; o < 32; o <<= 1) vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
-    const float inv_lam = kInt8 ? pow2(lam_exp == INT_MIN ? 0 : -lam_exp) : pow2(-lam_exp);
-    const float kap = kInt8 ? DitherConst<kBits == 10 ? 10 : 8>::kappa : 0.f;
+    if constexpr (kFlat) {
+        if (n_my > 0) warp_rows(flat_partial());
+        return;
+    }
 
     // ---- CTA merge: warps -> shared, one partial per CTA -----------------------------
     __syncthreads();   // stage buffers are reused below
     float* mbuf = reinterpret_cast<float*>(smem);   // [warp][head][kPartialStride]
-    {
-        float* wb = mbuf + warp * kMaxGroup * kPartialStride;
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            float* row = wb + (2 * c + e) * kPartialStride + 16 * g;   // dims 16g .. 16g+15
-            const float add = kap * spv_part[e];
-#pragma unroll
-            for (int q4 = 0; q4 < 4; ++q4) {
-                float4 v;
-                v.x = fmaf(acc[2 * q4][e], inv_lam, add);
-                v.y = fmaf(acc[2 * q4][e + 2], inv_lam, add);
-                v.z = fmaf(acc[2 * q4 + 1][e], inv_lam, add);
-                v.w = fmaf(acc[2 * q4 + 1][e + 2], inv_lam, add);
-                *reinterpret_cast<float4*>(row + 4 * q4) = v;
-            }
-            if (g == 0) {
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 0] = m_run[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 1] = l_part[e];
-                wb[(2 * c + e) * kPartialStride + kHeadDim + 2] = d_part[e];
-                if constexpr (kTierB) wb[(2 * c + e) * kPartialStride + kHeadDim + 3] = db_part[e];
-                if constexpr (kValue) {
-                    wb[(2 * c + e) * kPartialStride + kHeadDim + 4] = vt_part[e];
-                    wb[(2 * c + e) * kPartialStride + kHeadDim + 5] = vmax;
-                }
-            }
-        }
-    }
+    warp_rows(mbuf + warp * kMaxGroup * kPartialStride);
     __syncthreads();
     const size_t unit = (size_t)b * p.num_kv_heads + h;
     float* part_out = p.partials + (unit * p.splits + split) * (kMaxGroup * kPartialStride);
@@ -687,18 +838,6 @@ __device__ __forceinline__ void consumer_sync() {   // the 8 consumer warps only
 }
 
 
-// q fragment of the B operand (head g, channels 32c + 2i, +1 in word i).
-__device__ __forceinline__ void load_q_frag(const DecodeParams& p, int b, int h, int G, int g, int c,
-                                            uint32_t (&qw)[16]) {
-    const bool row_valid = g < G;
-    const uint4* qsrc = reinterpret_cast<const uint4*>(
-        p.q + ((size_t)b * p.num_q_heads + (size_t)h * G + (row_valid ? g : 0)) * kHeadDim + 32 * c);
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 v = row_valid ? __ldg(qsrc + i) : make_uint4(0, 0, 0, 0);
-        qw[4 * i] = v.x; qw[4 * i + 1] = v.y; qw[4 * i + 2] = v.z; qw[4 * i + 3] = v.w;
-    }
-}
 
 template <int kX>
 __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_constant__ WsParams wp) {
@@ -1413,11 +1552,21 @@ DecodePlan plan_decode(int batch, int num_kv_heads, int max_pages, int num_sms, 
     pl.splits = (int)std::max<long>(1, (max_pages + best_pps - 1) / best_pps);
     long partials = units * pl.splits;
     // A batch of several sequences (lengths unknown to the host, often ragged)
-    // takes the flattened plan: Hkv x floor(SMs / Hkv) CTAs, one per SM, each
-    // an equal share of one KV head's pages.
-    if ((use_ws(scheme, bits) || scheme == WC_SCHEME_DITHER_INT8_G32) && batch > 1 &&
-        (long long)batch * max_pages < (1LL << 31)) {
-        pl.splits = num_kv_heads * std::max(1, num_sms / num_kv_heads);   // a share per num_kv_heads CTAs
+    // takes the flattened plan: Hkv x floor(resident CTAs / Hkv) CTAs, all
+    // resident, each taking equal shares of one KV head's pages; a share per CTA
+    // for the warp-specialized kernels (one CTA per SM), a share per warp for
+    // the per-token kernel (two CTAs of 8 warps per SM).  The per-token kernel
+    // takes it only for the 10-bit dither and only when the split plan would
+    // leave resident CTA slots empty: a warp's share ends in a partial of its
+    // own (4.5 KB), which costs less than the idle SMs only where pages are
+    // expensive (the dither regenerated in the warp); split-plan CTAs are
+    // scheduled as SMs free up, which already evens out a ragged batch that
+    // fills a wave, and fp8 pages are cheap.
+    const bool per_warp = ctas_per_sm(scheme, bits) > 1;
+    const bool flat_ok = !per_warp || (scheme == WC_SCHEME_DITHER_INT8 && pl.splits * units < slots);
+    if (batch > 1 && (long long)batch * max_pages < (1LL << 31) && flat_ok) {
+        const int ctas = num_kv_heads * std::max(1, (int)(slots / num_kv_heads));
+        pl.splits = per_warp ? ctas * kWarps : ctas;   // shares: the merge reads splits / Hkv per head
         pl.pages_per_split = 0;
         partials = pl.splits + units;
     }
@@ -1613,12 +1762,28 @@ static cudaError_t launch_one(const DecodeParams& p, cudaStream_t stream) {
     if (!encode_page_map(&dp.k_map, p.k_codes, p.num_pages, p.num_kv_heads) ||
         !encode_page_map(&dp.v_map, p.v_codes, p.num_pages, p.num_kv_heads))
         return cudaErrorInvalidValue;
-    dim3 grid(p.splits, p.num_kv_heads, p.batch);
+    // split plan: (splits, Hkv, batch); flattened plan: one CTA per 8 warp shares
+    const dim3 grid = (kX & kXFlat) ? dim3(p.splits / kWarps) : dim3(p.splits, p.num_kv_heads, p.batch);
     cudaError_t e = launch_pdl(decode_kernel<kScheme, kBits, kX>, grid, dim3(kThreads), kSmemBytes, stream, dp);
     if (e != cudaSuccess) return e;
     // the merge is a programmatic dependent too: its CTAs are scheduled while
     // the decode grid drains and wait (griddepcontrol.wait) for all of it
-    return launch_merge<kX>(p, stream);
+    return launch_merge<kX & ~kXFlat>(p, stream);
+}
+
+// The per-token kernel for the extras in x (Tier B only with the dither).
+template <int kScheme, int kBits, int kF>
+static cudaError_t launch_one_x(const DecodeParams& p, int x, cudaStream_t stream) {
+    if constexpr (kScheme == WC_SCHEME_FP8_E4M3) {
+        return x == kXValue  ? launch_one<kScheme, kBits, kXValue | kF>(p, stream)
+             : x == kXRepair ? launch_one<kScheme, kBits, kXRepair | kF>(p, stream)
+                             : launch_one<kScheme, kBits, kF>(p, stream);
+    } else {
+        return x == kXTierB  ? launch_one<kScheme, kBits, kXTierB | kF>(p, stream)
+             : x == kXValue  ? launch_one<kScheme, kBits, kXValue | kF>(p, stream)
+             : x == kXRepair ? launch_one<kScheme, kBits, kXRepair | kF>(p, stream)
+                             : launch_one<kScheme, kBits, kF>(p, stream);
+    }
 }
 
 // cuTensorMapEncodeTiled through the runtime's driver entry point (the
@@ -1709,19 +1874,15 @@ cudaError_t launch_decode(const DecodeParams& p, int scheme, int bits, cudaStrea
     // requested by separate entry points, never together (checked by the caller)
     const int x = (p.meter_b ? kXTierB : 0) | (p.value_term ? kXValue : 0) | (p.page_terms ? kXRepair : 0) |
                   (p.k_new ? kXAppend : 0);
-    if (scheme == WC_SCHEME_FP8_E4M3)
-        return x == kXValue  ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXValue>(p, stream)
-             : x == kXRepair ? launch_one<WC_SCHEME_FP8_E4M3, 8, kXRepair>(p, stream)
-                             : launch_one<WC_SCHEME_FP8_E4M3, 8, 0>(p, stream);
+    if (scheme == WC_SCHEME_FP8_E4M3)   // always the split plan (plan_decode)
+        return p.pages_per_split == 0 ? cudaErrorNotSupported : launch_one_x<WC_SCHEME_FP8_E4M3, 8, 0>(p, x, stream);
     if (p.stall_page >= 0)   // failure-detection test (checked by the caller: 8-bit dither, no extras)
         return use_ws(scheme, bits) && p.pages_per_split > 0 && x == 0 ? launch_ws<kXStall>(p, stream)
                                                                         : cudaErrorNotSupported;
     if (use_ws(scheme, bits))   // pages_per_split == 0: the flattened plan
         return p.pages_per_split == 0 ? launch_ws_x<kXFlat>(p, x, stream) : launch_ws_x<0>(p, x, stream);
-    return x == kXTierB  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXTierB>(p, stream)
-         : x == kXValue  ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXValue>(p, stream)
-         : x == kXRepair ? launch_one<WC_SCHEME_DITHER_INT8, 10, kXRepair>(p, stream)
-                         : launch_one<WC_SCHEME_DITHER_INT8, 10, 0>(p, stream);
+    return p.pages_per_split == 0 ? launch_one_x<WC_SCHEME_DITHER_INT8, 10, kXFlat>(p, x, stream)
+                                  : launch_one_x<WC_SCHEME_DITHER_INT8, 10, 0>(p, x, stream);
 }
 
 }  // namespace wc

@@ -93,20 +93,24 @@ def test_decode_many_splits_long_context():
     _compare(*_run(wl, bits=10, layer=5))
 
 
+@pytest.mark.parametrize("scheme,bits", [(0, 8), (1, 8), (0, 10)])
 @pytest.mark.parametrize("ctx_lens,hq,hkv", [
     ([0, 1, 16, 17, 40, 0, 33, 5] * 25, 8, 2),      # 200 short sequences: CTAs walk many segments
     ([3000, 1, 0, 16, 2049, 17, 0, 700], 28, 4),     # one long sequence among short and empty ones
     ([0, 5], 8, 2),
     ([(37 * i) % 41 for i in range(600)], 8, 2),    # more sequences than the CTA's threads: several each
 ])
-def test_decode_flattened_plan_batches(ctx_lens, hq, hkv):
-    """A batch of several sequences runs the flattened split plan (each CTA an
-    equal share of all units' pages, cut at unit boundaries): every sequence
-    against the oracle, empty sequences give out = 0 and meter 0."""
+def test_decode_flattened_plan_batches(ctx_lens, hq, hkv, scheme, bits):
+    """A batch of several sequences: the warp-specialized kernel runs the
+    flattened split plan (each CTA an equal share of all units' pages, cut at
+    unit boundaries), the per-token kernel (fp8, 10-bit dither) the split plan
+    or, for the 10-bit dither when that leaves SMs idle, a flattened plan with a
+    share per warp: every sequence against the oracle, empty sequences give
+    out = 0 and meter 0."""
     import paper_2607_28699_gb300 as wc
     wl = W.Workload("f", 1, hq, hkv, ctx_lens, shuffle_pages=True, seed=9)
     bt, sm, k, v, q = make_inputs(wl, 0)
-    od, gd = descs(hq, hkv, wl.num_pages, 0, 8, 0, 3)
+    od, gd = descs(hq, hkv, wl.num_pages, scheme, bits, 0, 3)
     ocache = OP.empty_cache(od)
     OP.write_tokens(od, 0, k.numpy(), v.numpy(), sm, ocache)
     gcache = wc.LayerCache.empty(gd)
@@ -134,12 +138,15 @@ def test_decode_flattened_plan_batches(ctx_lens, hq, hkv):
 
 
 @pytest.mark.parametrize("scheme,bits", [(1, 8), (0, 10)])
-def test_decode_split_plan_batch_few_splits(scheme, bits):
-    """A batch on the per-token kernel (fp8, the 10-bit dither) takes the split
-    plan; here 8 splits of 24 pages per sequence, so the merge runs one warp per
-    output over the splits that hold the sequence's pages.  Empty and short
-    sequences beside long ones: every sequence against the oracle, empty ones
-    give out = 0 and meter 0."""
+def test_decode_per_token_kernel_batch(scheme, bits):
+    """A batch on the per-token kernel.  The 10-bit dither here takes the
+    flattened plan with one share per warp (the split plan would fill 224 of
+    304 CTA slots): each warp walks a contiguous run of the batch's pages
+    across sequence boundaries and writes one partial per sequence it touched.
+    fp8 keeps the split plan (8 splits, merged one warp per output over the
+    splits that hold pages).  Empty and short sequences beside long ones, the
+    oracle decoding the same stored cache: every sequence against it, empty
+    ones give out = 0 and meter 0."""
     import paper_2607_28699_gb300 as wc
     ctx_lens = [0, 3000, 5, 1200, 0, 16, 2049]
     wl = W.Workload("s", 1, 28, 4, ctx_lens, shuffle_pages=True, seed=12)

@@ -78,7 +78,7 @@ def test_noalloc_decode_matches_workspace_and_oracle_twice(scheme, ctx_lens, lay
 def test_noalloc_rejects_work_beyond_its_scratch_and_a_null_status():
     import paper_2607_28699_gb300 as wc
     f = _noalloc_fn()
-    # many short sequences: the plan needs more partials than 4 MiB holds
+    # many short sequences: the plan needs more partials than 16 MiB holds
     batch, max_pages = 4096, 64
     _, gd = descs(32, 8, 16, seed=1)
     cache = wc.LayerCache.empty(gd)
