@@ -44,10 +44,11 @@ def test_tier_b_matches_oracle_config1_shape(bits, layout):
     _run(W.config(1, ctx_scale=0.3), bits, layout)
 
 
+@pytest.mark.parametrize("bits", [8, 10])   # the 10-bit dither: the per-token kernel's per-warp plan
 @pytest.mark.parametrize("delta", [1e-2, 1e-9])
-def test_tier_b_batch_mixed_shuffled_gqa7(delta):
+def test_tier_b_batch_mixed_shuffled_gqa7(delta, bits):
     wl = W.Workload("m", 1, 28, 4, [4100, 77, 1, 2500, 16, 999], shuffle_pages=True, seed=6)
-    _run(wl, layer=3, delta=delta)
+    _run(wl, bits=bits, layer=3, delta=delta)
 
 
 def test_tier_b_many_splits():

@@ -16,9 +16,9 @@ from tests._parity import assert_close, assert_sound, descs, gpu_cache_to_numpy,
 pytestmark = pytest.mark.gpu
 
 
-def _setup(wl, scheme, layer, seed):
+def _setup(wl, scheme, layer, seed, bits=8):
     bt, sm, k, v, q = make_inputs(wl, layer)
-    od, gd = descs(wl.n_q_heads, wl.n_kv_heads, wl.num_pages, scheme, 8, 0, seed)
+    od, gd = descs(wl.n_q_heads, wl.n_kv_heads, wl.num_pages, scheme, bits, 0, seed)
     ocache = OP.empty_cache(od)
     OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
     return bt, sm, k, v, q, od, gd, ocache
@@ -43,12 +43,12 @@ def test_value_witness_write(scheme):
     assert np.all(gw >= ow) and np.all((gw == ow) | (gw == up))
 
 
-@pytest.mark.parametrize("scheme", [0, 1])
-def test_value_side_decode_and_joint_gate(scheme):
+@pytest.mark.parametrize("scheme,bits", [(0, 8), (1, 8), (0, 10)])   # 10-bit: the per-warp plan
+def test_value_side_decode_and_joint_gate(scheme, bits):
     import paper_2607_28699_gb300 as wc
     wl = W.Workload("d", 1, 28, 4, [4100, 77, 1, 2500, 16, 999], shuffle_pages=True, seed=6)
     layer = 3
-    bt, sm, k, v, q, od, gd, ocache = _setup(wl, scheme, layer, 7)
+    bt, sm, k, v, q, od, gd, ocache = _setup(wl, scheme, layer, 7, bits)
     gcache = numpy_cache_to_gpu(ocache, gd, value_witness=True)     # identical stored inputs on both sides
     ws = wc.Workspace(gd, wl.batch, wl.max_pages)
     ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
