@@ -174,12 +174,13 @@ def test_decode_per_token_kernel_batch(scheme, bits):
         assert_sound(raw[b], r["meter_raw"], r["tv"], f"meter_raw[{b}]")
 
 
-def test_decode_flattened_plan_bad_ctx_sets_status():
+@pytest.mark.parametrize("bits", [8, 10])   # 10: the per-token kernel's per-warp plan
+def test_decode_flattened_plan_bad_ctx_sets_status(bits):
     """Out-of-range context lengths in a batch are clamped and reported."""
     import paper_2607_28699_gb300 as wc
     wl = W.Workload("fb", 1, 8, 2, [64, 30], seed=2)
     bt, sm, k, v, q = make_inputs(wl)
-    od, gd = descs(8, 2, wl.num_pages)
+    od, gd = descs(8, 2, wl.num_pages, bits=bits)
     cache = wc.LayerCache.empty(gd)
     wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
     ws = wc.Workspace(gd, 2, wl.max_pages)
@@ -223,19 +224,22 @@ def test_decode_zero_context_and_repeat_calls():
     assert wc.read_status(ws) == 0
 
 
-def test_decode_bad_page_and_bad_ctx_set_status():
+@pytest.mark.parametrize("bits,ctx_lens", [(8, [64]), (10, [64]), (10, [64, 40])])   # [64, 40]: per-warp plan
+def test_decode_bad_page_and_bad_ctx_set_status(bits, ctx_lens):
     import paper_2607_28699_gb300 as wc
-    wl = W.Workload("b", 1, 8, 2, [64], seed=2)
+    wl = W.Workload("b", 1, 8, 2, ctx_lens, seed=2)
     bt, sm, k, v, q = make_inputs(wl)
-    od, gd = descs(8, 2, wl.num_pages)
+    od, gd = descs(8, 2, wl.num_pages, bits=bits)
     cache = wc.LayerCache.empty(gd)
     wc.kv_quantize_witness(gd, 0, k.cuda(), v.cuda(), torch.from_numpy(sm).cuda(), cache)
-    ws = wc.Workspace(gd, 1, wl.max_pages)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
     bt_bad = torch.from_numpy(bt).cuda().clone()
     bt_bad[0, 1] = 10_000
-    ctx = torch.tensor([64], dtype=torch.int32, device="cuda")
+    ctx = torch.tensor(ctx_lens, dtype=torch.int32, device="cuda")
     wc.metered_decode_attention(gd, 0, q.cuda(), bt_bad, ctx, cache, ws)
     assert wc.read_status(ws) & wc.DEV_BAD_PAGE
+    if len(ctx_lens) > 1:
+        return
     ctx_bad = torch.tensor([65], dtype=torch.int32, device="cuda")    # > max_pages * 16
     wc.metered_decode_attention(gd, 0, q.cuda(), torch.from_numpy(bt).cuda(), ctx_bad, cache, ws)
     assert wc.read_status(ws) & wc.DEV_BAD_CTX
