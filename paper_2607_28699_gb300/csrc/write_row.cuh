@@ -207,6 +207,44 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         // exactly below (about one warp in fifty, and rows with tiny amax).
         auto fast_pass = [&](auto with_residual) -> float {
             float dev = 0.0f;
+            if constexpr (!kGrouped && kBits == 8) {
+                // Channel pairs on the packed fp32x2 path: each lane of __ffma2_rn /
+                // __fadd2_rn rounds like the scalar fmaf / add, so est, t, k and r are
+                // the scalar pass's bits.  est - k and k - xi are taken as fma(-1, k,
+                // est) and fma(-1, xi, k) (exact products, the same roundings), and
+                // r = fma(-s, k - xi, x) is the residual with its sign flipped.  The
+                // squared residuals sum in two chains per half; the 2^-18 margin of
+                // norm_up_fp16 covers the fp32 error of any summation order.
+                const float2 inv2 = make_float2(inv_s, inv_s), ns2 = make_float2(-s, -s);
+                const float2 m1 = make_float2(-1.0f, -1.0f), c128 = make_float2(128.0f, 128.0f);
+                const float2 off = make_float2(-128.498046875f, -128.498046875f);
+                const float2 pb = make_float2(kBias, kBias), nb = make_float2(-kBias, -kBias);
+                float2 alo = make_float2(0.0f, 0.0f), ahi = make_float2(0.0f, 0.0f);
+#pragma unroll
+                for (int i = 0; i < 16; i += 2) {
+                    const float2 f = make_float2(__uint_as_float(prmt(dw[i >> 2], 0x3F800000u, xi_sel(i))),
+                                                 __uint_as_float(prmt(dw[(i + 1) >> 2], 0x3F800000u, xi_sel(i + 1))));
+                    const float2 xi = __ffma2_rn(f, c128, off);   // (j + 1/2)/256 - 1/2, as xi_of
+                    const float2 x2 = make_float2(x[i], x[i + 1]);
+                    const float2 est = __ffma2_rn(x2, inv2, xi);
+                    const float2 t = __fadd2_rn(est, pb);
+                    const float2 k = __fadd2_rn(t, nb);
+                    const float2 d = __ffma2_rn(k, m1, est);
+                    dev = fmaxf(dev, fmaxf(fabsf(d.x), fabsf(d.y)));
+                    tb[i] = __float_as_uint(t.x);
+                    tb[i + 1] = __float_as_uint(t.y);
+                    if constexpr (decltype(with_residual)::value) {
+                        const float2 r = __ffma2_rn(ns2, __ffma2_rn(xi, m1, k), x2);
+                        if (i < 8) alo = __ffma2_rn(r, r, alo);
+                        else ahi = __ffma2_rn(r, r, ahi);
+                    }
+                }
+                if constexpr (decltype(with_residual)::value) {
+                    lo = alo.x + alo.y;
+                    hi = ahi.x + ahi.y;
+                }
+                return dev;
+            }
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
                 const bool byp = kGrouped && ((bmask >> i) & 1u);   // exact channel: code 0, no residual
