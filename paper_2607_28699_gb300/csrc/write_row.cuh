@@ -244,23 +244,24 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
                     hi = ahi.x + ahi.y;
                 }
                 return dev;
-            }
+            } else {
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-                const bool byp = kGrouped && ((bmask >> i) & 1u);   // exact channel: code 0, no residual
-                const float xi = xi_of(i);
-                const float est = byp ? 0.0f : fmaf(x[i], inv_s, xi);   // s = 0: x = 0, est = xi, k = 0
-                const float t = est + kBias;
-                const float k = t - kBias;
-                dev = fmaxf(dev, fabsf(est - k));
-                tb[i] = __float_as_uint(t);
-                if constexpr (decltype(with_residual)::value) {
-                    const float r = byp ? 0.0f : fmaf(s, k - xi, -x[i]);   // x^ - x, one rounding
-                    if (i < 8) lo = fmaf(r, r, lo);
-                    else hi = fmaf(r, r, hi);
+                for (int i = 0; i < 16; ++i) {
+                    const bool byp = kGrouped && ((bmask >> i) & 1u);   // exact channel: code 0, no residual
+                    const float xi = xi_of(i);
+                    const float est = byp ? 0.0f : fmaf(x[i], inv_s, xi);   // s = 0: x = 0, est = xi, k = 0
+                    const float t = est + kBias;
+                    const float k = t - kBias;
+                    dev = fmaxf(dev, fabsf(est - k));
+                    tb[i] = __float_as_uint(t);
+                    if constexpr (decltype(with_residual)::value) {
+                        const float r = byp ? 0.0f : fmaf(s, k - xi, -x[i]);   // x^ - x, one rounding
+                        if (i < 8) lo = fmaf(r, r, lo);
+                        else hi = fmaf(r, r, hi);
+                    }
                 }
+                return dev;
             }
-            return dev;
         };
         bool exact = need_clamp;
         if (!exact) {
