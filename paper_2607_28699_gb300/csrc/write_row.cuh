@@ -16,8 +16,8 @@ namespace {
 // Quantizer: code = round-half-even of the exact real v = x/s + xi, clamped to
 // [-127, 127].  With s a normal fp16, s >= (amax / 126.5)(1 - 2^-24)(1 - 2^-11),
 // so |x/s| <= 126.57 and |v| < 127.07: the clamp cannot bind.  The fp32
-// estimate est = fma(x, RN(1/s), xi) then differs from v by at most
-// |x/s| 2^-24 (the reciprocal) + ulp(est)/2 = 7.6e-6 + 3.9e-6 < 1.2e-5, so
+// estimate est = fma(x, 1/s, xi), 1/s as recip_scale gives it, then differs from v by at most
+// |x/s| (2^-24 + 2^-46) (the reciprocal) + ulp(est)/2 < 7.6e-6 + 3.9e-6 < 1.2e-5, so
 // rounding est gives round(v) unless est lies within 1.2e-5 of a half-integer.
 // The fast pass flags estimates within 2e-5 of a tie (4 elements in 10^5).
 // Flagged rows, and rows whose scale is an fp16 subnormal (where the clamp
@@ -31,6 +31,28 @@ __device__ __forceinline__ float exact_round(float x, float s, float xi, float k
     if (up > 0.0f || (up == 0.0f && k_odd)) k += 1.0f;
     else if (dn < 0.0f || (dn == 0.0f && k_odd)) k -= 1.0f;
     return fminf(127.0f, fmaxf(-127.0f, k));
+}
+
+// fp32(amax) / 126.5 rounded to nearest even, for amax a non-negative fp16 value
+// or +inf: q0 = amax * RN(1/126.5), then one correction with the exact remainder
+// amax - q0 * 126.5 (Markstein, IBM J. Res. Dev. 34(1), 1990).  For every finite
+// fp16 amax the result equals the IEEE quotient (checked exhaustively with exact
+// rational arithmetic in tests/test_write_scale.py).
+__device__ __forceinline__ float div_126_5(float amax) {
+    constexpr float kInv = 0x1.03091cp-7f;   // RN(1 / 126.5)
+    const float q0 = amax * kInv;
+    const float r = fmaf(-q0, 126.5f, amax);
+    return amax == INFINITY ? amax : fmaf(r, kInv, q0);
+}
+
+// 1/s for a positive fp16 scale s (0 for +inf): rcp.approx (at most one ulp of
+// error) refined by one Newton-Raphson step y (2 - s y), within 2^-24 + 2^-46 of
+// 1/s relative, the error the estimate bound above allows for the reciprocal.
+__device__ __forceinline__ float recip_scale(float s) {
+    if (!(s < INFINITY)) return 0.0f;
+    float y;
+    asm("rcp.approx.f32 %0, %1;" : "=f"(y) : "f"(s));
+    return fmaf(y, fmaf(-s, y, 1.0f), y);
 }
 
 // Norm for a witness, rounded up to fp16: the smallest fp16 h with
@@ -141,10 +163,10 @@ __device__ __forceinline__ void write_row(const WriteParams& p, uint4 (&raw)[2],
         // the row (8 lanes) or the 32-channel group (a lane pair)
 #pragma unroll
         for (int o = 1; o < (kGrouped ? 2 : 8); o <<= 1) amax = fmaxf(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-        __half sh = __float2half_rn(__fdiv_rn(amax, 126.5f));
+        __half sh = __float2half_rn(div_126_5(amax));
         if (__half_as_ushort(sh) == 0 && amax > 0.0f) sh = __ushort_as_half((unsigned short)1);
         s = __half2float(sh);
-        const float inv_s = s > 0.0f ? __frcp_rn(s) : 0.0f;
+        const float inv_s = s > 0.0f ? recip_scale(s) : 0.0f;
 
         // dither words for channels 16*sub .. 16*sub + 15
         const uint32_t slot_u = (uint32_t)max(slot, 0);
