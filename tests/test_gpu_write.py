@@ -80,6 +80,43 @@ def test_write_edge_rows():
         _compare(ocache, gpu_cache_to_numpy(gcache))
 
 
+def test_write_scale_every_fp16_exponent():
+    """Rows whose amax takes fp16 values across every exponent (subnormals to
+    65504, 64 mantissas each, the largest and smallest included): the scale's
+    quotient and the reciprocal behind the fast rounding pass, checked on the
+    device through bit-exact scales and codes."""
+    import paper_2607_28699_gb300 as wc
+    rng = np.random.default_rng(21)
+    bits = []
+    for e in range(31):
+        mant = np.unique(np.concatenate([[0, 1, 1023], rng.integers(0, 1024, size=61)]))[:64]
+        bits.extend(int((e << 10) | int(m)) for m in mant)
+    amax = np.array(bits, dtype=np.uint16).view(np.float16).astype(np.float64)
+    amax = amax[amax > 0]
+    n = (amax.size + 1) // 2
+    amax = np.resize(amax, 2 * n).reshape(n, 2)
+    x = rng.normal(size=(n, 2, 128)) * (amax[..., None] / 3.0)
+    x = np.clip(x, -amax[..., None], amax[..., None]).astype(np.float16)
+    x = np.clip(x.astype(np.float64), -amax[..., None], amax[..., None])
+    idx = rng.integers(0, 128, size=(n, 2))
+    sign = np.where(rng.random((n, 2)) < 0.5, -1.0, 1.0)
+    np.put_along_axis(x, idx[..., None], (sign * amax)[..., None], axis=2)
+    k = x.astype(np.float16)
+    assert np.array_equal(np.abs(k.astype(np.float64)).max(axis=2), amax)
+    v = k[::-1].copy()
+    slots = np.arange(n, dtype=np.int32)
+    num_pages = (n + 15) // 16
+    for bits_ in (8, 10):
+        od, gd = descs(4, 2, num_pages, 0, bits_, 0, seed=29)
+        ocache = OP.empty_cache(od)
+        OP.write_tokens(od, 1, k, v, slots, ocache)
+        gcache = wc.LayerCache.empty(gd)
+        wc.kv_quantize_witness(gd, 1, torch.from_numpy(k).cuda(), torch.from_numpy(v).cuda(),
+                               torch.from_numpy(slots).cuda(), gcache)
+        torch.cuda.synchronize()
+        _compare(ocache, gpu_cache_to_numpy(gcache))
+
+
 @pytest.mark.parametrize("n_tok", [1, 5, 15, 16, 17])
 @pytest.mark.parametrize("hkv", [1, 4, 8])
 def test_write_small_batches_match_oracle(n_tok, hkv):
