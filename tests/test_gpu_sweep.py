@@ -82,3 +82,88 @@ def test_random_shapes_match_oracle(i):
         else:
             assert_close(raw[b], r["meter_raw"], f"meter_raw[{b}]")
             assert_close(meter[b], r["meter"], f"meter[{b}]")
+
+
+def _lens(r, batch, top):
+    lens = [0 if r.random() < 0.15 else int(r.integers(1, top)) for _ in range(batch)]
+    if max(lens) == 0:
+        lens[0] = int(r.integers(1, top))
+    return lens
+
+
+@pytest.mark.parametrize("i", range(10))
+def test_random_shapes_grouped_cache_and_tier_b(i):
+    """The grouped-scale cache (§6.2.3, §6.2.5) with 0-8 bypassed pairs: its
+    write bit for bit, its decode and grouped Tier-B meter against the oracle."""
+    import paper_2607_28699_gb300 as wc
+    from tests.test_gpu_grouped import _check_write, _write_both
+    r = np.random.default_rng(5000 + i)
+    hkv = int(r.choice([1, 2, 4]))
+    group = int(r.integers(1, 9))
+    m = int(r.choice([0, 1, 2, 3, 4, 8]))
+    layout = int(r.integers(0, 2))
+    wl = W.Workload(f"gsweep{i}", 1, group * hkv, hkv, _lens(r, int(r.integers(1, 11)), 2200),
+                    shuffle_pages=bool(r.random() < 0.5), seed=70 + i)
+    layer = int(r.integers(0, 28))
+    print(f"[gsweep {i}] Hq={wl.n_q_heads} Hkv={hkv} m={m} layout={layout} lens={wl.ctx_lens}")
+    bt, k, v, q, od, gd, ocache, gwrite = _write_both(wl, layer, m, layout, 90 + i)
+    _check_write(ocache, gwrite)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    delta = 10.0 ** -float(r.integers(2, 6))
+    res = wc.metered_decode_attention_tier_b(gd, layer, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws,
+                                             delta)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, raw, raw_b = res[0].cpu().numpy(), res[2].cpu().numpy(), res[4].cpu().numpy()
+    offs = np.concatenate([[0], np.cumsum(wl.ctx_lens)[:-1]])
+    for b, S in enumerate(wl.ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(raw[b] == 0) and np.all(raw_b[b] == 0)
+            continue
+        o = offs[b]
+        ref = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, k[o:o + S], v[o:o + S], delta_loc=delta)
+        assert_close(out[b], ref["out"], f"out[{b}]")
+        assert_close(raw[b], ref["meter_raw"], f"meter_raw[{b}]")
+        assert_sound(raw[b], ref["meter_raw"], ref["tv"], f"meter_raw[{b}]")
+        assert_close(raw_b[b], ref["meter_b_raw"], f"meter_b_raw[{b}]")
+        assert_sound(raw_b[b], ref["meter_b_raw"], None, f"meter_b_raw[{b}]")
+
+
+@pytest.mark.parametrize("i", range(8))
+def test_random_shapes_tier_b_per_token_cache(i):
+    """Tier B (§4.2) on the per-token dithered cache, 8- and 10-bit dither."""
+    import paper_2607_28699_gb300 as wc
+    r = np.random.default_rng(6000 + i)
+    hkv = int(r.choice([1, 2, 4]))
+    group = int(r.integers(1, 9))
+    bits = 8 if i % 2 == 0 else 10
+    layout = int(r.integers(0, 2))
+    wl = W.Workload(f"bsweep{i}", 1, group * hkv, hkv, _lens(r, int(r.integers(1, 11)), 2600),
+                    shuffle_pages=bool(r.random() < 0.5), seed=80 + i)
+    layer = int(r.integers(0, 28))
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    od, gd = descs(wl.n_q_heads, wl.n_kv_heads, wl.num_pages, 0, bits, layout, 40 + i)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    delta = 10.0 ** -float(r.integers(2, 6))
+    res = wc.metered_decode_attention_tier_b(gd, layer, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws,
+                                             delta)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, raw_b = res[0].cpu().numpy(), res[4].cpu().numpy()
+    offs = np.concatenate([[0], np.cumsum(wl.ctx_lens)[:-1]])
+    for b, S in enumerate(wl.ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(raw_b[b] == 0)
+            continue
+        o = offs[b]
+        ref = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, k.numpy()[o:o + S], v.numpy()[o:o + S],
+                                 delta_loc=delta)
+        assert_close(out[b], ref["out"], f"out[{b}]")
+        assert_close(raw_b[b], ref["meter_b_raw"], f"meter_b_raw[{b}]")
+        assert_sound(raw_b[b], ref["meter_b_raw"], None, f"meter_b_raw[{b}]")
