@@ -167,3 +167,87 @@ def test_random_shapes_tier_b_per_token_cache(i):
         assert_close(out[b], ref["out"], f"out[{b}]")
         assert_close(raw_b[b], ref["meter_b_raw"], f"meter_b_raw[{b}]")
         assert_sound(raw_b[b], ref["meter_b_raw"], None, f"meter_b_raw[{b}]")
+
+
+@pytest.mark.parametrize("i", range(8))
+def test_random_shapes_fused_append(i):
+    """The step's write fused into its decode: cache and outputs bit for bit
+    those of the separate write and decode, on random shapes (one new token
+    per sequence, some sequences without one)."""
+    import paper_2607_28699_gb300 as wc
+    r = np.random.default_rng(7000 + i)
+    hkv = int(r.choice([1, 2, 4]))
+    group = int(r.integers(1, 9))
+    lens = [int(r.integers(1, 3000)) for _ in range(int(r.integers(1, 11)))]
+    wl = W.Workload(f"asweep{i}", 1, group * hkv, hkv, lens, shuffle_pages=bool(r.random() < 0.5), seed=90 + i)
+    layer = int(r.integers(0, 28))
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    last = np.cumsum(wl.ctx_lens) - 1
+    prefix = np.setdiff1d(np.arange(len(sm)), last)
+    gd = wc.CacheDesc(num_q_heads=wl.n_q_heads, num_kv_heads=hkv, num_pages=wl.num_pages,
+                      rope_layout=int(r.integers(0, 2)), seed=60 + i)
+    kd, vd, smd = k.cuda(), v.cuda(), torch.from_numpy(sm).cuda()
+    base = wc.LayerCache.empty(gd)
+    if prefix.size:
+        pi = torch.from_numpy(prefix).cuda()
+        wc.kv_quantize_witness(gd, layer, kd[pi].contiguous(), vd[pi].contiguous(), smd[pi].contiguous(), base)
+    li = torch.from_numpy(last).cuda()
+    k_new, v_new, s_new = kd[li].contiguous(), vd[li].contiguous(), smd[li].contiguous()
+    skip = r.random(len(lens)) < 0.2
+    s_new[torch.from_numpy(skip).cuda()] = -1                       # no new token for these sequences
+    keep = ~skip
+    clone = lambda c: wc.LayerCache(c.k_codes.clone(), c.v_codes.clone(), c.k_scale.clone(), c.v_scale.clone(),
+                                    c.k_witness.clone())
+    a, b = clone(base), clone(base)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    qd, btd = q.cuda(), torch.from_numpy(bt).cuda()
+    ws_a, ws_b = wc.Workspace(gd, wl.batch, wl.max_pages), wc.Workspace(gd, wl.batch, wl.max_pages)
+    if keep.any():
+        ki = torch.from_numpy(np.nonzero(keep)[0]).cuda()
+        wc.kv_quantize_witness(gd, layer, k_new[ki].contiguous(), v_new[ki].contiguous(), s_new[ki].contiguous(), a)
+    ra = wc.metered_decode_attention(gd, layer, qd, btd, ctx, a, ws_a)
+    rb = wc.metered_decode_attention_append(gd, layer, qd, btd, ctx, b, ws_b, k_new, v_new, s_new)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws_a) == 0 and wc.read_status(ws_b) == 0
+    for name in ("k_codes", "v_codes", "k_scale", "v_scale", "k_witness"):
+        assert torch.equal(getattr(a, name), getattr(b, name)), name
+    for x, y in zip(ra, rb):
+        assert torch.equal(x, y)
+
+
+@pytest.mark.parametrize("i", range(8))
+def test_random_shapes_value_side(i):
+    """Value witness, value term, max ||v|| and the output bound (§3, §4.2)
+    against the oracle on random shapes, all three read schemes."""
+    import paper_2607_28699_gb300 as wc
+    r = np.random.default_rng(8000 + i)
+    hkv = int(r.choice([1, 2, 4]))
+    group = int(r.integers(1, 9))
+    scheme, bits = SCHEMES[i % len(SCHEMES)]
+    wl = W.Workload(f"vsweep{i}", 1, group * hkv, hkv, _lens(r, int(r.integers(1, 11)), 2600),
+                    shuffle_pages=bool(r.random() < 0.5), seed=110 + i)
+    layer = int(r.integers(0, 28))
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    od, gd = descs(wl.n_q_heads, hkv, wl.num_pages, scheme, bits, 0, 20 + i)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
+    gcache = numpy_cache_to_gpu(ocache, gd, value_witness=True)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    res = wc.metered_decode_attention_v(gd, layer, q.cuda(), torch.from_numpy(bt).cuda(), ctx, gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    out, vterm, vmax, bound = (res[j].cpu().numpy() for j in (0, 3, 4, 5))
+    offs = np.concatenate([[0], np.cumsum(wl.ctx_lens)[:-1]])
+    for b, S in enumerate(wl.ctx_lens):
+        if S == 0:
+            assert np.all(out[b] == 0) and np.all(vterm[b] == 0) and np.all(bound[b] == 0)
+            continue
+        o = offs[b]
+        ref = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, k.numpy()[o:o + S], v.numpy()[o:o + S])
+        assert_close(out[b], ref["out"], f"out[{b}]")
+        assert_close(vterm[b], ref["value_term"], f"value_term[{b}]")
+        assert_sound(vterm[b], ref["value_term"], None, f"value_term[{b}]")
+        assert np.array_equal(vmax[b].astype(np.float64), ref["v_max"])
+        assert_close(bound[b], ref["out_bound"], f"out_bound[{b}]")
+        assert np.all(bound[b] >= ref["out_err"])
