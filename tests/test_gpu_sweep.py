@@ -251,3 +251,46 @@ def test_random_shapes_value_side(i):
         assert np.array_equal(vmax[b].astype(np.float64), ref["v_max"])
         assert_close(bound[b], ref["out_bound"], f"out_bound[{b}]")
         assert np.all(bound[b] >= ref["out_err"])
+
+
+@pytest.mark.parametrize("i", range(6))
+def test_random_shapes_repair_selection(i):
+    """Block-level repair selection (§6.3.5) on random shapes: the per-page
+    contributions against the oracle's, the plain outputs untouched, and each
+    flagged cell's list consistent with the kernel's contributions and a top
+    set of the oracle's that brings the meter to tau."""
+    import paper_2607_28699_gb300 as wc
+    from tests.test_gpu_repair import _check_selection
+    r = np.random.default_rng(9000 + i)
+    hkv = int(r.choice([1, 2, 4]))
+    group = int(r.integers(1, 9))
+    scheme, bits = SCHEMES[i % len(SCHEMES)]
+    lens = [int(r.integers(1, 2600)) for _ in range(int(r.integers(1, 9)))]
+    wl = W.Workload(f"rsweep{i}", 1, group * hkv, hkv, lens, shuffle_pages=bool(r.random() < 0.5), seed=130 + i)
+    layer = int(r.integers(0, 28))
+    bt, sm, k, v, q = make_inputs(wl, layer)
+    od, gd = descs(wl.n_q_heads, hkv, wl.num_pages, scheme, bits, 0, 30 + i)
+    ocache = OP.empty_cache(od)
+    OP.write_tokens(od, layer, k.numpy(), v.numpy(), sm, ocache)
+    gcache = numpy_cache_to_gpu(ocache, gd)
+    ws = wc.Workspace(gd, wl.batch, wl.max_pages)
+    ctx = torch.tensor(wl.ctx_lens, dtype=torch.int32, device="cuda")
+    qd, btd = q.cuda(), torch.from_numpy(bt).cuda()
+    res = wc.metered_decode_attention_repair(gd, layer, qd, btd, ctx, gcache, ws)
+    plain = wc.metered_decode_attention(gd, layer, qd, btd, ctx, gcache, ws)
+    torch.cuda.synchronize()
+    assert wc.read_status(ws) == 0
+    for x, y in zip(plain, res[:3]):
+        assert torch.equal(x, y)
+    meter_raw = res[2].cpu().numpy()
+    tau = float(np.median(meter_raw)) * float(r.uniform(0.2, 0.9))
+    contrib, pages, n_rep, d_after = wc.repair_select(res[3], res[4], ctx, tau)
+    torch.cuda.synchronize()
+    contrib, pages, n_rep, d_after = (t.cpu().numpy() for t in (contrib, pages, n_rep, d_after))
+    for b, S in enumerate(wl.ctx_lens):
+        ref = OP.decode_sequence(od, layer, q.numpy()[b], bt[b], S, ocache, repair_tau=tau)
+        n = (S + 15) // 16
+        assert_close(contrib[b, :, :n], ref["contrib"], f"contrib[{b}]", atol=1e-6)
+        for hq in range(wl.n_q_heads):
+            _check_selection(contrib[b, hq, :n], pages[b, hq, :n_rep[b, hq]], n, d_after[b, hq], tau,
+                             ref["contrib"][hq])
