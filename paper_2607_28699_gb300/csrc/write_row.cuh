@@ -45,9 +45,12 @@ __device__ __forceinline__ float div_126_5(float amax) {
     return amax == INFINITY ? amax : fmaf(r, kInv, q0);
 }
 
-// 1/s for a positive fp16 scale s (0 for +inf): rcp.approx (at most one ulp of
-// error) refined by one Newton-Raphson step y (2 - s y), within 2^-24 + 2^-46 of
-// 1/s relative, the error the estimate bound above allows for the reciprocal.
+// 1/s for a positive fp16 scale s (0 for +inf): rcp.approx (documented within
+// one ulp) refined by one Newton-Raphson step y (2 - s y).  The step squares the
+// approximation's relative error e (to e^2 < 2^-46 for |e| <= 2^-23; below 2^-24
+// still for any |e| <= 2^-12) and its final fma rounds once, so the result lies
+// within 2^-24 + 2^-46 of 1/s relative: the reciprocal error the estimate bound
+// above allows.
 __device__ __forceinline__ float recip_scale(float s) {
     if (!(s < INFINITY)) return 0.0f;
     float y;
