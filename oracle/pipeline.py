@@ -228,6 +228,13 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
         res["repair"] = [None] * desc.num_q_heads
     if tier_b and desc.scheme == SCHEME_FP8_E4M3:
         raise ValueError("Tier B needs the dithered INT8 cache (a controlled quantizer)")
+    if ctx_len == 0:
+        # An empty context attends to nothing: out = 0 and meter = meter_raw = 0
+        # (A = 1 in the e-form), no pages to repair (the reading used for context 0).
+        res["A"][:] = 1.0
+        if repair_tau is not None:
+            res["repair"] = [np.zeros(0, dtype=np.int64) for _ in range(desc.num_q_heads)]
+        return res
     page, off = slots // desc.page_size, slots % desc.page_size
     for h in range(desc.num_kv_heads):
         khat, vhat, w = reconstruct(desc, layer, h, slots, cache)

@@ -91,3 +91,18 @@ def test_write_path_is_position_free_and_deterministic():
     write_tokens(desc, 0, k[:5], v[:5], np.array([-1, 3, -1, 4, -1]), c2)
     assert np.count_nonzero(c2["k_codes"][0, :, [0, 1, 2, 5]]) == 0
     assert np.count_nonzero(c2["k_codes"][0, :, 3]) > 0
+
+
+@pytest.mark.parametrize("scheme", [0, 1])
+def test_empty_context_attends_to_nothing(scheme):
+    """Context 0 (the reading for an empty sequence): out = 0, meters 0, no
+    pages to repair; a one-token context next to it is an ordinary decode."""
+    wl, bt, k, v, q, desc, cache = _small(scheme)
+    r0 = decode_sequence(desc, 0, q[0], bt[0], 0, cache, k[:0], v[:0], repair_tau=0.1,
+                         delta_loc=1e-3 if scheme == 0 else None)
+    for name in ("out", "meter", "meter_raw", "tv", "value_term", "out_bound", "meter_b_raw"):
+        assert np.all(r0[name] == 0), name
+    assert all(len(x) == 0 for x in r0["repair"])
+    r1 = decode_sequence(desc, 0, q[0], bt[0], 1, cache, k[:1], v[:1])
+    assert np.all(r1["meter_raw"] >= r1["tv"])
+    assert np.allclose(np.abs(r1["out"]).sum(axis=1) > 0, True)
