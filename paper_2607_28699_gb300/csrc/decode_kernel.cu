@@ -805,9 +805,8 @@ struct WsParams {
 
 // Append (kXAppend): the step's new token of sequence b, the last of its
 // context, is quantized and stored by the producer warp that stages the
-// sequence's last page, before that page's copies are issued (under the split
-// plan before the warp's first page, under the flattened plan just before the
-// page).  Its slot must
+// sequence's last page, before it issues the copies of the segment that holds
+// that page.  Its slot must
 // be that of the context's last token (else WC_DEV_BAD_APPEND, not written),
 // so no other CTA reads it.  Lanes 0-7 hold the row (write path layout); the
 // generic-proxy stores are fenced against the async-proxy copies that follow.
@@ -934,11 +933,11 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
             int first;
             const int n_seg = ws_seg_pages<kWsPairs>(cs, pw, first);
             int phys_next = kFlat ? (n_seg > 0 ? __ldg(bt_row + first) : -1) : phys_first;
-            if constexpr (kAppend && !kFlat) {
-                // Split plan: the stream that stages the sequence's last page stores the
-                // new token before its first page (not inside the page loop), so its
-                // write overlaps the other streams' first pages and the loop carries
-                // no write code.  Its copies are issued after the token's stores.
+            if constexpr (kAppend) {
+                // The stream that stages the sequence's last page in this segment stores
+                // the new token before the segment's first page (not inside the page
+                // loop), so its write overlaps the other streams' pages and the loop
+                // carries no write code.  Its copies are issued after the token's stores.
                 const int lpl = npages - 1;
                 if (n_seg > 0 && lpl >= first && (lpl - first) % kWsPairs == 0 && lpl < cs.e) {
                     const int phl = __ldg(bt_row + lpl);
@@ -960,9 +959,6 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 if (i + 1 < n_seg) phys_next = __ldg(bt_row + lp + kWsPairs);
                 const bool ok = phys >= 0 && phys < p.num_pages;
                 uint8_t* st = stages + s * kWsStageBytes;
-                if constexpr (kAppend && kFlat) {   // the sequence's last page: store the new token first
-                    if (ok && lp == npages - 1) append_new_token(wp, b, h, phys, ctx, lane);
-                }
                 if constexpr (kStall) {   // failure-detection test: this page is never staged
                     if (lp == p.stall_page) {
                         issued = k + 1;
