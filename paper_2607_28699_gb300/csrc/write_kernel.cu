@@ -47,15 +47,16 @@ constexpr int kPerHeadMinTokens = 16;                     // per-head grid from 
 //  else:     one index over units u = token * Hkv + h, a task = 4 consecutive
 //            units, so a one-token write of up to 8 KV heads is a single CTA
 //            (decode steps, where every SM the next decode needs counts).
-// Resident CTAs per SM the register budget is sized for: six for the 8-bit
-// dither, whose packed fast pass keeps its 80 registers without spilling
-// (seven would cap it at 72), the register counts the other variants need
-// otherwise.
-__host__ __device__ constexpr int write_min_blocks(int scheme, int bits) {
-    return scheme == WC_SCHEME_DITHER_INT8 && bits == 8 ? 6 : scheme == WC_SCHEME_FP8_E4M3 ? 10 : 7;
+// Resident CTAs per SM the register budget is sized for: seven (72 registers)
+// for the dithered schemes, ten for fp8.  The 8-bit dither's packed fast pass
+// then spills 4 bytes; the extra warps per SM still take 4-5% off a prefill
+// write against six CTAs at 80 registers, and eight (64 registers, 48 bytes of
+// spill) are slower again.
+__host__ __device__ constexpr int write_min_blocks(int scheme) {
+    return scheme == WC_SCHEME_FP8_E4M3 ? 10 : 7;
 }
 template <int kScheme, int kBits, bool kPerHead>
-__global__ void __launch_bounds__(128, write_min_blocks(kScheme, kBits)) write_kernel(const __grid_constant__ WriteParams p) {
+__global__ void __launch_bounds__(128, write_min_blocks(kScheme)) write_kernel(const __grid_constant__ WriteParams p) {
     constexpr bool kGrouped = kScheme == WC_SCHEME_DITHER_INT8_G32;
     __shared__ __align__(16) uint8_t xrows[kGrouped ? 4 * 4 * kXRowStride : 16];   // [warp][unit][row]
     __shared__ BypassTable btab;
