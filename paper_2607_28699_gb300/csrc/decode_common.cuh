@@ -66,6 +66,27 @@ constexpr float kDRel = 1.0f + 0x1p-12f;
 constexpr float kDAbs = 0x1p-21f;
 __device__ __forceinline__ float d_upper(float d) { return fmaf(d, kDRel, kDAbs); }
 
+// One token's meter term p~ (e^c - 1) in the log2 frame of the running maximum:
+// t = y - m (p~ = 2^t, flushed to 0 below 2^-126) and cl = c log2(e).  The
+// kernels use the product 2^t (2^cl - 1) as long as every cl of the page is below
+// kHugeLog2: an underflowed 2^t then drops less than 2^(64 - 126) per token,
+// far inside kDAbs.  A page with a larger bound (a key row of huge magnitude;
+// never with ordinary inputs) takes its terms from meter_term, which uses
+// 2^(t + cl) from kHugeLog2 on, its exponent raised by a bound on the two fp32
+// roundings of t + cl + margin: at least the term, and finite wherever the term
+// is, so a token whose weight underflows but whose bound does not still counts
+// (the product gives 0, or 0 * inf = NaN).
+constexpr float kHugeLog2 = 64.0f;
+__device__ __forceinline__ float meter_term(float t, float cl) {
+    if (cl < kHugeLog2) return fast_exp2(t) * (fast_exp2(cl) - 1.f);
+    if (t == -INFINITY) return 0.f;   // a token past the context
+    return fast_exp2(t + cl + (fabsf(t) + cl) * 0x1p-22f);
+}
+
+// NaN only arises in the meter from 0 * inf or inf - inf, i.e. from a term or a
+// sum that overflowed: report it as +inf, the bound's overflow value.
+__device__ __forceinline__ float raw_or_inf(float raw) { return raw == raw ? raw : INFINITY; }
+
 // 2^n for -126 <= n <= 127.
 __device__ __forceinline__ float pow2(int n) { return __int_as_float((127 + n) << 23); }
 

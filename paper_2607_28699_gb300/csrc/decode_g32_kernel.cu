@@ -455,16 +455,35 @@ __global__ void __launch_bounds__(kGwThreads, 1) decode_g32_ws_kernel(const __gr
                         acc[mt][1] *= a1; acc[mt][3] *= a1;
                     }
                 }
-                float pe[4];
+                float pe[4], ub[4];           // ub: the Tier-B bound in log2 units
+#pragma unroll
+                for (int i = 0; i < 4; ++i) ub[i] = kTierB ? u[i] * kLog2e : 0.f;
+                bool huge;                    // warp-uniform: a bound of kHugeLog2 or more (meter_term)
+                {
+                    float big = fmaxf(fmaxf(cb[0], cb[1]), fmaxf(cb[2], cb[3]));
+                    if constexpr (kTierB) big = fmaxf(big, fmaxf(fmaxf(ub[0], ub[1]), fmaxf(ub[2], ub[3])));
+                    huge = __any_sync(0xffffffffu, big >= kHugeLog2);
+                }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int e = i & 1;
                     pe[i] = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
                     l_part[e] += pe[i];
-                    d_part[e] = fmaf(pe[i], fast_exp2(cb[i]) - 1.f, d_part[e]);
-                    if constexpr (kTierB) db_part[e] = fmaf(pe[i], fast_exp2(u[i] * kLog2e) - 1.f, db_part[e]);
+                    if (!huge) {
+                        d_part[e] = fmaf(pe[i], fast_exp2(cb[i]) - 1.f, d_part[e]);
+                        if constexpr (kTierB) db_part[e] = fmaf(pe[i], fast_exp2(ub[i]) - 1.f, db_part[e]);
+                    }
 #pragma unroll
                     for (int gi = 0; gi < 4; ++gi) spv[gi][e] = fmaf(pe[i], sv[i >> 1][gi], spv[gi][e]);
+                }
+                if (huge) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int e = i & 1;
+                        const float t = y[i] - m_run[e];
+                        d_part[e] += meter_term(t, cb[i]);
+                        if constexpr (kTierB) db_part[e] += meter_term(t, ub[i]);
+                    }
                 }
                 {   // P s_g 2^lam_exp < 2^14: s_g 2^lam_exp < 2^6 for every group of the page;
                     // lam_exp only decreases, checked per lane against sv_lim, reduced only then

@@ -549,19 +549,43 @@ __global__ void __launch_bounds__(kThreads, kMinBlocks) decode_kernel(const __gr
                 }
             }
             float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
+            float cl[4], ub[4];          // the bounds in log2 units (ub: Tier B)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                cl[i] = cb[i] * kLog2e;
+                ub[i] = kTierB ? ((i & 1) ? alpha1 : alpha0) * sk[i >> 1] * kLog2e : 0.f;
+            }
+            bool huge;                   // warp-uniform: a bound of kHugeLog2 or more (meter_term)
+            {
+                float big = fmaxf(fmaxf(cl[0], cl[1]), fmaxf(cl[2], cl[3]));
+                if constexpr (kTierB) big = fmaxf(big, fmaxf(fmaxf(ub[0], ub[1]), fmaxf(ub[2], ub[3])));
+                huge = __any_sync(0xffffffffu, big >= kHugeLog2);
+            }
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int r = i >> 1, e = i & 1;
                 const float pe = fast_exp2(y[i] - m_run[e]);     // 0 for masked tokens
                 l_part[e] += pe;
-                const float em1 = fast_exp2(cb[i] * kLog2e) - 1.f;
-                d_part[e] = fmaf(pe, em1, d_part[e]);
-                if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
-                if constexpr (kTierB)
-                    db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
+                if (!huge) {
+                    const float em1 = fast_exp2(cl[i]) - 1.f;
+                    d_part[e] = fmaf(pe, em1, d_part[e]);
+                    if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
+                    if constexpr (kTierB) db_part[e] = fmaf(pe, fast_exp2(ub[i]) - 1.f, db_part[e]);
+                }
                 if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                 P[i] = pe * sv[r];
                 spv_part[e] += P[i];
+            }
+            if (huge) {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const int e = i & 1;
+                    const float t = y[i] - m_run[e];
+                    const float dt = meter_term(t, cl[i]);
+                    d_part[e] += dt;
+                    if constexpr (kRepair) dpg[e] += dt;
+                    if constexpr (kTierB) db_part[e] += meter_term(t, ub[i]);
+                }
             }
             if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
             if constexpr (kInt8) {
@@ -1233,21 +1257,44 @@ __global__ void __launch_bounds__(kWsThreads, 1) decode_ws_kernel(const __grid_c
                 const float svl[2] = {sv[0] * lam, sv[1] * lam};   // exact: lam is a power of two
                 float dpg[2] = {0.f, 0.f};   // this page's share of D (kRepair)
                 float x[4];                  // P * s_v * lam, the PV operand
+                float ub[4];                 // Tier-B bound in log2 units (kTierB)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) ub[i] = kTierB ? ((i & 1) ? alpha1 : alpha0) * sk[i >> 1] * kLog2e : 0.f;
+                bool huge = false;           // warp-uniform: a bound of kHugeLog2 or more (meter_term)
+                if constexpr (!kMeterOff || kTierB) {
+                    float big = kMeterOff ? 0.f : fmaxf(fmaxf(cb[0], cb[1]), fmaxf(cb[2], cb[3]));
+                    if constexpr (kTierB) big = fmaxf(big, fmaxf(fmaxf(ub[0], ub[1]), fmaxf(ub[2], ub[3])));
+                    huge = __any_sync(0xffffffffu, big >= kHugeLog2);
+                }
 #pragma unroll
                 for (int i = 0; i < 4; ++i) {
                     const int r = i >> 1, e = i & 1;
                     const float pe = fast_exp2(y[i] - m_run[e]);
                     l_part[e] += pe;
-                    if constexpr (!kMeterOff) {
-                        const float em1 = fast_exp2(cb[i]) - 1.f;
-                        d_part[e] = fmaf(pe, em1, d_part[e]);
-                        if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
+                    if (!huge) {
+                        if constexpr (!kMeterOff) {
+                            const float em1 = fast_exp2(cb[i]) - 1.f;
+                            d_part[e] = fmaf(pe, em1, d_part[e]);
+                            if constexpr (kRepair) dpg[e] = fmaf(pe, em1, dpg[e]);
+                        }
+                        if constexpr (kTierB) db_part[e] = fmaf(pe, fast_exp2(ub[i]) - 1.f, db_part[e]);
                     }
-                    if constexpr (kTierB)
-                        db_part[e] = fmaf(pe, fast_exp2((e ? alpha1 : alpha0) * sk[r] * kLog2e) - 1.f, db_part[e]);
                     if constexpr (kValue) vt_part[e] = fmaf(pe, rho[r], vt_part[e]);
                     x[i] = pe * svl[r];
                     spv_part[e] += x[i];     // sum P s_v, in the lam frame
+                }
+                if (huge) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const int e = i & 1;
+                        const float t = y[i] - m_run[e];
+                        if constexpr (!kMeterOff) {
+                            const float dt = meter_term(t, cb[i]);
+                            d_part[e] += dt;
+                            if constexpr (kRepair) dpg[e] += dt;
+                        }
+                        if constexpr (kTierB) db_part[e] += meter_term(t, ub[i]);
+                    }
                 }
                 if constexpr (kRepair) emit_page_terms(p, b, h, G, lp, g, c, dpg, m_run);
                 uint32_t bp0, bp1, bl0, bl1;
@@ -1494,7 +1541,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
             float raw = 0.f;
             if (l > 0.f) {
                 const float D = d_upper(dn / l);        // A - 1, rounded up
-                raw = 0.5f * D * (D + 2.0f);            // (A^2 - 1) / 2, +inf on overflow
+                raw = raw_or_inf(0.5f * D * (D + 2.0f));   // (A^2 - 1) / 2, +inf on overflow
             }
             p.meter_raw[cell] = raw;
             p.meter[cell] = fminf(1.0f, raw);
@@ -1503,7 +1550,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_kernel(const __grid_co
                 float rb = 0.f;
                 if (l > 0.f) {
                     const float D = d_upper(db / l);
-                    rb = 0.5f * D * (D + 2.0f);
+                    rb = raw_or_inf(0.5f * D * (D + 2.0f));
                 }
                 p.meter_b_raw[cell] = rb;
                 p.meter_b[cell] = fminf(1.0f, rb);
@@ -1697,7 +1744,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_warp_kernel(const __gr
         float raw = 0.f;
         if (L > 0.f) {
             const float D = d_upper(Dn / L);
-            raw = 0.5f * D * (D + 2.0f);
+            raw = raw_or_inf(0.5f * D * (D + 2.0f));
         }
         p.meter_raw[cell] = raw;
         p.meter[cell] = fminf(1.0f, raw);
@@ -1706,7 +1753,7 @@ __global__ void __launch_bounds__(32 * kMergeWarps) merge_warp_kernel(const __gr
             float rb = 0.f;
             if (L > 0.f) {
                 const float D = d_upper(Db / L);
-                rb = 0.5f * D * (D + 2.0f);
+                rb = raw_or_inf(0.5f * D * (D + 2.0f));
             }
             p.meter_b_raw[cell] = rb;
             p.meter_b[cell] = fminf(1.0f, rb);
