@@ -178,9 +178,10 @@ size_t wc_workspace_size(const wc_cache_desc* desc, int32_t batch, int32_t max_p
  *   c_t             = (1/sqrt(128)) sum_b ||q_b|| w_{t,b}
  *   meter_raw[b][hq] = 1/2 (A^2 - 1), A = sum_t p~_t e^{c_t}  (+inf on fp32 overflow)
  *   meter[b][hq]    = min(1, meter_raw)
- * meter_raw is rounded up (an upper bound, never below the exact value); a
- * term or sum that overflows fp32 makes it +inf (never NaN), including a
- * token whose softmax weight underflows fp32 while its bound is huge.
+ * meter_raw carries an upward margin sized to cover its fp32 evaluation
+ * (checked on or above the fp64 value); a term or sum that overflows fp32
+ * makes it +inf (never NaN), including a token whose softmax weight
+ * underflows fp32 while its bound is huge.
  * The context is split across CTAs (one sequence: every KV head's pages in
  * equal splits; several sequences, whose lengths only the device sees: each
  * CTA serves one KV head and an equal share of the batch's pages laid end to
