@@ -97,10 +97,46 @@ def eform_meter(p_tilde, c):
     with np.errstate(over="ignore", invalid="ignore"):
         terms = p_tilde * np.expm1(c)
         terms = np.where(p_tilde == 0, 0.0, terms)      # 0 * e^huge is 0 mass
+    return meter_of_terms(terms)
+
+
+def meter_of_terms(terms):
+    """(meter, meter_raw, A) from the terms p~_t expm1(c_t) of D = A - 1."""
+    with np.errstate(over="ignore", invalid="ignore"):
         D = np.sum(terms, axis=-1)
         raw = 0.5 * D * (D + 2.0)
     raw = np.where(np.isnan(raw), np.inf, raw)
     return np.minimum(1.0, raw), raw, 1.0 + D
+
+
+def eform_terms(z, c):
+    """p~ = softmax(z) and the terms p~_t expm1(c_t) of D, for logits z of
+    cached tokens (all finite) and bounds c >= 0.
+
+    The product p~_t expm1(c_t) is the definition as written; where float64
+    cannot hold it (p~_t underflows to 0 for a logit ~745 below the maximum,
+    or expm1(c_t) overflows for c_t > ~709) the same number is taken in the
+    log domain, exp(log p~_t + log expm1(c_t)) with log p~_t = z_t - m -
+    log sum_s e^{z_s - m} and log expm1(c) = c + log(-expm1(-c)), so a token
+    whose weight underflows still counts with its bound.  Elsewhere the terms
+    are bit for bit those of eform_meter(softmax(z), c).
+    """
+    z = np.asarray(z, np.float64)
+    c = np.asarray(c, np.float64)
+    p = softmax(z)
+    m = np.max(z, axis=-1, keepdims=True)
+    with np.errstate(over="ignore", invalid="ignore", divide="ignore"):
+        em1 = np.expm1(c)
+        direct = p * em1
+        log_p = (z - m) - np.log(np.sum(np.exp(z - m), axis=-1, keepdims=True))
+        logged = np.exp(log_p + c + np.log(-np.expm1(-c)))
+        terms = np.where((p > 0) & np.isfinite(em1), direct, logged)
+    return p, terms
+
+
+def eform_meter_logits(z, c):
+    """eform_meter of softmax(z) with the terms of eform_terms: (meter, meter_raw, A)."""
+    return meter_of_terms(eform_terms(z, c)[1])
 
 
 def tier_a_bound(q, w, num_bands, rope_layout):
@@ -193,12 +229,14 @@ def joint_gate(meter_raw, vterm, v_max, tau_k, tau_v, group):
     return keep_q, keep_kv, int(np.sum(keep_q)), int(np.sum(keep_kv))
 
 
-def page_contributions(p_tilde, c, page_of_token, n_pages):
-    """C_j = sum over the tokens of logical page j of p~_t expm1(c_t)."""
-    p_tilde = np.asarray(p_tilde, np.float64)
-    with np.errstate(over="ignore", invalid="ignore"):
-        terms = p_tilde * np.expm1(np.asarray(c, np.float64))
-        terms = np.where(p_tilde == 0, 0.0, terms)      # as in eform_meter
+def page_contributions(p_tilde, c, page_of_token, n_pages, terms=None):
+    """C_j = sum over the tokens of logical page j of p~_t expm1(c_t) (the
+    terms may be given, e.g. those of eform_terms)."""
+    if terms is None:
+        p_tilde = np.asarray(p_tilde, np.float64)
+        with np.errstate(over="ignore", invalid="ignore"):
+            terms = p_tilde * np.expm1(np.asarray(c, np.float64))
+            terms = np.where(p_tilde == 0, 0.0, terms)      # as in eform_meter
     return np.bincount(np.asarray(page_of_token, dtype=np.int64), weights=terms, minlength=n_pages)
 
 

@@ -241,12 +241,14 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
         for g in range(G):
             hq = h * G + g
             q = np.asarray(q16[hq], dtype=np.float64)
-            p_tilde = M.softmax(M.logits(q, khat))
+            z_tilde = M.logits(q, khat)
             c = M.tier_a_bound(q, w, desc.num_bands, desc.rope_layout)
-            res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.eform_meter(p_tilde, c)
+            p_tilde, terms = M.eform_terms(z_tilde, c)
+            res["meter"][hq], res["meter_raw"][hq], res["A"][hq] = M.meter_of_terms(terms)
             res["out"][hq] = M.attend(p_tilde, vhat)
             if repair_tau is not None:
-                res["contrib"][hq] = M.page_contributions(p_tilde, c, np.arange(ctx_len) // desc.page_size, n_pages)
+                res["contrib"][hq] = M.page_contributions(p_tilde, c, np.arange(ctx_len) // desc.page_size, n_pages,
+                                                          terms=terms)
                 res["repair"][hq] = M.repair_plan(res["contrib"][hq], repair_tau)[0]
             vw = cache["v_witness"][page, h, off].astype(np.float64)        # [S, 2]
             res["value_term"][hq] = M.value_term(p_tilde, vw[:, 0])
@@ -255,10 +257,10 @@ def decode_sequence(desc, layer, q16, block_table_row, ctx_len, cache,
             if tier_b and desc.scheme == SCHEME_DITHER_INT8_G32:
                 u = M.tier_b_bound_grouped(q, cache["k_scale"][page, h, off], desc.group_channels,
                                            _excluded(desc, cache, h, 0), ctx_len, delta_loc)
-                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
+                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter_logits(z_tilde, u)
             elif tier_b:
                 u = M.tier_b_bound(q, cache["k_scale"][page, h, off].astype(np.float64), ctx_len, delta_loc)
-                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter(p_tilde, u)
+                res["meter_b"][hq], res["meter_b_raw"][hq], _ = M.eform_meter_logits(z_tilde, u)
             if k_exact is not None:
                 p = M.softmax(M.logits(q, np.asarray(k_exact)[:ctx_len, h]))
                 res["tv"][hq] = M.total_variation(p, p_tilde)

@@ -54,6 +54,47 @@ def test_eform_closed_forms():
     assert raw == pytest.approx(0.5 * math.expm1(0.5))
 
 
+def test_eform_terms_equal_the_product_on_ordinary_inputs():
+    """From logits, the terms and the meter are bit for bit the product form's
+    wherever float64 holds p~ and expm1(c)."""
+    rng = np.random.default_rng(21)
+    for S in (1, 2, 17, 300):
+        z = rng.normal(0, 4, S)
+        c = np.abs(rng.normal(0, 0.5, S))
+        p, terms = M.eform_terms(z, c)
+        assert np.array_equal(p, M.softmax(z))
+        assert np.array_equal(terms, M.softmax(z) * np.expm1(c))
+        for a, b in zip(M.eform_meter_logits(z, c), M.eform_meter(M.softmax(z), c)):
+            assert np.array_equal(a, b)
+
+
+def test_eform_terms_where_float64_underflows_or_overflows():
+    """Closed forms where the product cannot be formed in float64 (§3 e-form,
+    evaluated in the log domain): a weight of e^-800 / (1 + e^-800) with
+    c = 801 contributes e (1 - e^-801) / (1 + e^-800) = e to D, where the
+    product gives 0; a weight e^-705 / (1 + e^-705) with c = 710 contributes
+    e^5, where expm1(710) overflows."""
+    _, terms = M.eform_terms(np.array([0.0, -800.0]), np.array([0.0, 801.0]))
+    assert terms[0] == 0.0 and terms[1] == pytest.approx(math.e, rel=1e-13)
+    m, raw, A = M.eform_meter_logits(np.array([0.0, -800.0]), np.array([0.0, 801.0]))
+    assert raw == pytest.approx(0.5 * math.e * (math.e + 2.0), rel=1e-13) and m == 1.0
+    assert M.eform_meter(M.softmax(np.array([0.0, -800.0])), np.array([0.0, 801.0]))[1] == 0.0
+    m, raw, A = M.eform_meter_logits(np.array([0.0, -705.0]), np.array([0.0, 710.0]))
+    assert A - 1.0 == pytest.approx(math.exp(5.0), rel=1e-12)
+    assert M.eform_meter(M.softmax(np.array([0.0, -705.0])), np.array([0.0, 710.0]))[1] == np.inf
+    # beyond float64 the meter is +inf, and a zero bound adds nothing at any weight
+    m, raw, _ = M.eform_meter_logits(np.array([0.0, -10.0]), np.array([0.0, 2000.0]))
+    assert raw == np.inf and m == 1.0
+    _, terms = M.eform_terms(np.array([0.0, -900.0]), np.array([0.25, 0.0]))
+    assert terms[1] == 0.0 and terms[0] == pytest.approx(math.expm1(0.25), rel=1e-15)
+    # the page contributions from these terms sum to D
+    z, c = np.array([0.0, -800.0, -3.0, -790.0]), np.array([0.1, 801.0, 0.0, 792.0])
+    p, terms = M.eform_terms(z, c)
+    C = M.page_contributions(p, c, np.array([0, 0, 1, 1]), 2, terms=terms)
+    assert C.sum() == pytest.approx(M.eform_meter_logits(z, c)[2] - 1.0, rel=1e-14)
+    assert C[1] == pytest.approx(math.exp(2.0) / (1 + math.exp(-3.0)), rel=1e-12)
+
+
 def test_eform_sound_against_sign_vertices_and_interior():
     """TV(p, p~) <= 1/2 (A^2 - 1) for every admissible eps (brute force)."""
     rng = np.random.default_rng(2)
