@@ -15,7 +15,10 @@ c; +inf on overflow is sound and counts as over threshold (§6.2.5, on
 fp32 overflow).  Here 1/2 (A^2 - 1) is computed as 1/2 D (D + 2) with
 D = A - 1 = E_p~[expm1(c)], which is the same number without the
 cancellation of A^2 - 1 for small c (reading: the paper only asks for a
-numerically careful evaluation, "in the log domain").
+numerically careful evaluation, "in the log domain").  From logits
+(eform_terms, the pipeline's form) a term p~_t expm1(c_t) that float64
+cannot form as a product (p~_t underflowing, expm1(c_t) overflowing) is taken
+in the log domain, so it keeps its value instead of 0 or +inf.
 
 §4.1 Thm. "Sound black-box logit bound": |eps_t| = |q . r_t| / sqrt(d)
 <= (1/sqrt(d)) sum_b ||q_b|| w_{t,b} =: c_t.
