@@ -75,3 +75,25 @@ def test_reference_arm_under_torchrun_prints_one_line_from_rank_zero():
     assert len(lines) == 1, r.stdout[-2000:]
     d = json.loads(lines[0])
     assert d["impl"] == "reference" and d["n_gpus"] == 2 and d["value"] > 0
+
+
+def test_traffic_row_used_only_at_its_kernel_source(tmp_path, monkeypatch):
+    """roofline.traffic comes from profiles/traffic.txt only for the decode
+    source the row was captured at; any other source gives null."""
+    import hashlib
+    b = _bench_module()
+    root = tmp_path
+    (root / "paper_2607_28699_gb300" / "csrc").mkdir(parents=True)
+    (root / "profiles").mkdir()
+    src = root / "paper_2607_28699_gb300" / "csrc" / "decode_kernel.cu"
+    src.write_bytes(b"// kernel A\n")
+    sha = hashlib.sha256(b"// kernel A\n").hexdigest()[:16]
+    (root / "profiles" / "traffic.txt").write_text(
+        "# kernel  source_sha256_16  workload  bytes_per_launch\n"
+        f"decode_kernel {sha} wl-a 123456\n"
+        "decode_kernel 0000000000000000 wl-b 999\n")
+    monkeypatch.setattr(b, "ROOT", str(root))
+    assert b._traffic("wl-a") == 123456
+    assert b._traffic("wl-b") is None and b._traffic("wl-c") is None
+    src.write_bytes(b"// kernel B\n")          # the kernel changed since the capture
+    assert b._traffic("wl-a") is None
